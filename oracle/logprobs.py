@@ -1,0 +1,70 @@
+"""FP8 token scoring: logits, log-probs, ratios, dLoss/dlogits -- oracle side.
+
+Test infrastructure only (see ``oracle/__init__.py``).
+
+§2.1 defines the token ratio r_t = pi_theta(y_t|h_t) / pi_old(y_t|h_t); in the
+full-pipeline FP8 setting of §3 both probabilities come from FP8-quantised
+forward passes.  For the lm_head this is
+
+  z[t, v]   = sum_k  X_tilde_h[t, k] * X_tilde_W[v, k]       (dequantised, Eq. 3)
+  logp_t    = z[t, y_t] - log sum_v exp(z[t, v])             (temperature 1)
+  r_t       = exp(logp_new_t - logp_old_t)
+
+evaluated here in float64 from the dequantised operands (mathematically equal
+to the per-block scaled sum sum_kb S_h S_W sum_k q_h q_W).
+
+Readings: temperature 1 (the paper evaluates at temperature 1.0 and states no
+training temperature); the lm_head input and weight are both FP8-quantised at
+the same granularity.
+
+dLoss/dlogits follows from the chain rule through log-softmax:
+  dL/dz[t, v] = g_t * (1{v == y_t} - exp(z[t, v] - lse_t)),  g_t = dL/dlogp_t.
+"""
+
+import numpy as np
+
+from . import quantize as Q
+
+
+def logits(h_codes, h_scales, w_codes, w_scales, gran, rows=None):
+    """z = X_tilde_h @ X_tilde_W^T in float64 (optionally for a subset of rows)."""
+    xh = Q.dequantize(h_codes, h_scales, gran, Q.ACT)
+    if rows is not None:
+        xh = xh[np.asarray(rows)]
+    xw = Q.dequantize(w_codes, w_scales, gran, Q.WEIGHT)
+    return xh @ xw.T
+
+
+def log_softmax_gather(z, targets):
+    """(logp, lse): lse_t = log sum_v exp z[t, v]; logp_t = z[t, y_t] - lse_t."""
+    z = np.asarray(z, dtype=np.float64)
+    y = np.asarray(targets, dtype=np.int64)
+    if np.any(y < 0) or np.any(y >= z.shape[1]):
+        raise ValueError("target outside [0, V)")
+    m = np.max(z, axis=1)
+    lse = m + np.log(np.sum(np.exp(z - m[:, None]), axis=1))
+    zy = z[np.arange(z.shape[0]), y]
+    return zy - lse, lse
+
+
+def token_logprobs(h_codes, h_scales, w_codes, w_scales, gran, targets, rows=None):
+    """Per-token log-prob (and lse) of the target under the FP8 lm_head."""
+    z = logits(h_codes, h_scales, w_codes, w_scales, gran, rows)
+    y = np.asarray(targets)
+    if rows is not None:
+        y = y[np.asarray(rows)]
+    return log_softmax_gather(z, y)
+
+
+def importance_ratios(logp_new, logp_old):
+    """r_t = exp(logp_new - logp_old) (§2.1), float64."""
+    return np.exp(np.asarray(logp_new, np.float64) - np.asarray(logp_old, np.float64))
+
+
+def dlogits(z, targets, lse, g):
+    """dL/dz[t, v] = g_t (1{v == y_t} - exp(z[t, v] - lse_t)), float64."""
+    z = np.asarray(z, dtype=np.float64)
+    p = np.exp(z - np.asarray(lse, np.float64)[:, None])
+    onehot = np.zeros_like(p)
+    onehot[np.arange(z.shape[0]), np.asarray(targets, np.int64)] = 1.0
+    return np.asarray(g, np.float64)[:, None] * (onehot - p)

@@ -1,0 +1,71 @@
+"""Clipped PPO surrogate with TIS weights (Eq. 1, Eq. 4, §2.1) -- oracle side.
+
+Test infrastructure only (see ``oracle/__init__.py``).
+
+Eq. 1 / Eq. 4 per token, with calibrated bounds [L, H] in place of
+[1 - eps, 1 + eps] (§4):
+
+    l_t = -w_t * min(r_t A_t, clip(r_t, L, H) A_t),   clip(r, L, H) = min(max(r, L), H)
+
+Clip semantics (§2.1): a token's gradient is zeroed when A_t > 0 and r_t >= H,
+or A_t < 0 and r_t <= L -- these are the "clipped" tokens counted in the clip
+fractions.
+
+Readings:
+* Aggregation is the token mean over valid tokens: loss = sum_{mask} l_t /
+  sum mask (the DAPO token-level loss, used for GRPO as well).  sum mask = 0
+  gives loss 0.
+* The gradient returned is g_t = dloss / dlogp_t, with r_t = exp(logp_t -
+  logp_old_t) so dr/dlogp = r: g_t = -w_t A_t r_t / sum mask on unclipped valid
+  tokens and 0 elsewhere.
+* w_t = 1 when no TIS weights are given.
+* Everything here is float64.
+"""
+
+import numpy as np
+
+CLIP_HI = 1  # bit set in the clip mask: A > 0 and r >= H
+CLIP_LO = 2  # bit set in the clip mask: A < 0 and r <= L
+
+
+def clip_mask(r, adv, mask, lo, hi):
+    """Per-token clip bits, compared in float32 as the inputs are float32."""
+    r = np.asarray(r, np.float32)
+    adv = np.asarray(adv, np.float32)
+    valid = np.asarray(mask) != 0
+    up = valid & (adv > 0) & (r >= np.float32(hi))
+    dn = valid & (adv < 0) & (r <= np.float32(lo))
+    return (up * CLIP_HI + dn * CLIP_LO).astype(np.uint8)
+
+
+def clipped_surrogate(r, adv, mask, w, lo, hi):
+    """Token-mean clipped surrogate loss, per-token terms, grad and counts."""
+    r32 = np.asarray(r, np.float32)
+    a32 = np.asarray(adv, np.float32)
+    valid = np.asarray(mask) != 0
+    r64 = r32.astype(np.float64)
+    a64 = a32.astype(np.float64)
+    w64 = np.ones_like(r64) if w is None else np.asarray(w, np.float32).astype(np.float64)
+    lo64, hi64 = float(np.float32(lo)), float(np.float32(hi))
+    clipped_r = np.minimum(np.maximum(r64, lo64), hi64)
+    term = -w64 * np.minimum(r64 * a64, clipped_r * a64)
+    term = np.where(valid, term, 0.0)
+    n_valid = int(valid.sum())
+    cm = clip_mask(r32, a32, valid, lo, hi)
+    clipped = cm != 0
+    loss_sum = float(np.sum(term))
+    loss = loss_sum / n_valid if n_valid else 0.0
+    grad = np.where(valid & ~clipped, -w64 * a64 * r64, 0.0)
+    grad = grad / n_valid if n_valid else np.zeros_like(grad)
+    n_pos = int(np.sum(valid & (a32 > 0)))
+    n_neg = int(np.sum(valid & (a32 < 0)))
+    c_pos = int(np.sum((cm & CLIP_HI) != 0))
+    c_neg = int(np.sum((cm & CLIP_LO) != 0))
+    return {
+        "loss": loss, "loss_sum": loss_sum, "terms": term, "grad": grad,
+        "clip_mask": cm, "n_valid": n_valid, "n_pos": n_pos, "n_neg": n_neg,
+        "clipped_pos": c_pos, "clipped_neg": c_neg,
+        "clip_frac_pos": c_pos / n_pos if n_pos else 0.0,
+        "clip_frac_neg": c_neg / n_neg if n_neg else 0.0,
+        "clip_frac": (c_pos + c_neg) / n_valid if n_valid else 0.0,
+    }

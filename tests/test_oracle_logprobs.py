@@ -1,0 +1,121 @@
+"""Pins for the oracle's FP8 logits / log-prob / dlogits (§2.1, Eq. 3).
+
+Closed forms (W = 0, V = 1), one-hot weight rows (catches a transposed or
+mis-indexed operand), scale-exchange invariance between the two operands'
+block scales (catches a dropped or misplaced scale), SciPy's log_softmax, the
+normalisation of the softmax, and a finite-difference check of dlogits.
+"""
+
+import numpy as np
+import pytest
+import scipy.special
+
+from oracle import e4m3
+from oracle import logprobs as L
+from oracle import quantize as Q
+
+
+def _codes(rng, shape):
+    c = rng.integers(0, 256, size=shape).astype(np.uint8)
+    c[(c == 0x7F) | (c == 0xFF)] = 0x38
+    return c
+
+
+@pytest.mark.parametrize("gran", [Q.TENSOR, Q.ROWWISE, Q.BLOCK])
+def test_zero_weight_gives_uniform(gran):
+    rng = np.random.default_rng(0)
+    T, H, V = 5, 256, 37
+    hc = _codes(rng, (T, H))
+    hs = {Q.TENSOR: np.float32([0.5]), Q.ROWWISE: np.full(T, 0.25, np.float32),
+          Q.BLOCK: np.full((T, 2), 0.125, np.float32)}[gran]
+    wc = np.zeros((V, H), np.uint8)
+    ws = {Q.TENSOR: np.float32([1.0]), Q.ROWWISE: np.ones(V, np.float32),
+          Q.BLOCK: np.ones((1, 2), np.float32)}[gran]
+    y = rng.integers(0, V, T)
+    logp, lse = L.token_logprobs(hc, hs, wc, ws, gran, y)
+    assert np.allclose(logp, -np.log(V), rtol=0, atol=1e-14)
+
+
+def test_single_word_vocab():
+    rng = np.random.default_rng(1)
+    hc = _codes(rng, (4, 128))
+    wc = _codes(rng, (1, 128))
+    logp, _ = L.token_logprobs(hc, np.float32([0.01]), wc, np.float32([0.02]), Q.TENSOR, [0, 0, 0, 0])
+    assert np.all(logp == 0.0)
+
+
+def test_one_hot_rows_pick_dequantised_hidden_entries():
+    rng = np.random.default_rng(2)
+    T, H, V = 6, 256, 9
+    hc = _codes(rng, (T, H))
+    hs = rng.uniform(0.01, 2, size=(T, H // 128)).astype(np.float32)
+    cols = rng.integers(0, H, V)
+    wc = np.zeros((V, H), np.uint8)
+    wc[np.arange(V), cols] = 0x38  # code for 1.0
+    ws = np.ones((1, H // 128), np.float32)
+    z = L.logits(hc, hs, wc, ws, Q.BLOCK)
+    expect = e4m3.decode(hc)[:, cols] * hs[:, cols // 128]
+    assert np.array_equal(z, expect)
+
+
+def test_block_scale_exchange_invariance():
+    rng = np.random.default_rng(3)
+    T, H, V = 7, 384, 200
+    hc, wc = _codes(rng, (T, H)), _codes(rng, (V, H))
+    hs = rng.uniform(0.01, 1, size=(T, 3)).astype(np.float32)
+    ws = rng.uniform(0.01, 1, size=(2, 3)).astype(np.float32)
+    z0 = L.logits(hc, hs, wc, ws, Q.BLOCK)
+    hs2, ws2 = hs.copy(), ws.copy()
+    hs2[:, 1] *= 4
+    ws2[:, 1] /= 4
+    assert np.allclose(L.logits(hc, hs2, wc, ws2, Q.BLOCK), z0, rtol=1e-13, atol=1e-13)
+    ws3 = ws.copy()
+    ws3[:, 1] *= 2  # changing one scale must change the result
+    assert not np.allclose(L.logits(hc, hs, wc, ws3, Q.BLOCK), z0)
+    # equal block scales per row reduce block mode to row mode
+    hs_row = rng.uniform(0.01, 1, size=T).astype(np.float32)
+    ws_row = np.full(V, 0.5, np.float32)
+    zr = L.logits(hc, hs_row, wc, ws_row, Q.ROWWISE)
+    zb = L.logits(hc, np.repeat(hs_row[:, None], 3, 1), wc, np.full((2, 3), 0.5, np.float32), Q.BLOCK)
+    assert np.allclose(zr, zb, rtol=1e-14, atol=1e-14)
+
+
+def test_log_softmax_matches_scipy_and_normalises():
+    rng = np.random.default_rng(4)
+    z = rng.standard_normal((8, 1000)) * 5
+    y = rng.integers(0, 1000, 8)
+    logp, lse = L.log_softmax_gather(z, y)
+    ref = scipy.special.log_softmax(z, axis=1)[np.arange(8), y]
+    assert np.allclose(logp, ref, rtol=0, atol=1e-12)
+    assert np.allclose(lse, scipy.special.logsumexp(z, axis=1), rtol=0, atol=1e-12)
+    all_logp = np.stack([L.log_softmax_gather(z, np.full(8, v))[0] for v in range(1000)], 1)
+    assert np.allclose(np.exp(all_logp).sum(1), 1.0, atol=1e-12)
+    with pytest.raises(ValueError):
+        L.log_softmax_gather(z, np.full(8, 1000))
+
+
+def test_dlogits_finite_difference():
+    rng = np.random.default_rng(5)
+    T, V = 3, 11
+    z = rng.standard_normal((T, V))
+    y = rng.integers(0, V, T)
+    g = rng.standard_normal(T)
+
+    def f(zz):
+        return float(np.sum(g * L.log_softmax_gather(zz, y)[0]))
+
+    _, lse = L.log_softmax_gather(z, y)
+    d = L.dlogits(z, y, lse, g)
+    h = 1e-6
+    for t in range(T):
+        for v in range(V):
+            zp, zm = z.copy(), z.copy()
+            zp[t, v] += h
+            zm[t, v] -= h
+            assert abs((f(zp) - f(zm)) / (2 * h) - d[t, v]) < 1e-8
+    assert np.allclose(d.sum(1), 0.0, atol=1e-14)
+
+
+def test_ratio_identity():
+    lp = np.random.default_rng(6).standard_normal(10)
+    assert np.all(L.importance_ratios(lp, lp) == 1.0)

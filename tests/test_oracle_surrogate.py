@@ -1,0 +1,80 @@
+"""Pins for the oracle's clipped surrogate (Eq. 1, Eq. 4, §2.1 clip semantics).
+
+A hand-worked table, the unclipped special case r = 1 (loss reduces to the
+TIS-weighted mean of -A), A = 0, the equality conventions, and the gradient
+against a central finite difference in float64.
+"""
+
+import os
+
+import numpy as np
+import pytest
+
+from oracle import surrogate as S
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def test_hand_worked_table():
+    rows = []
+    for line in open(os.path.join(GOLDEN, "surrogate_tiny.txt")):
+        line = line.split("#")[0].strip()
+        if line:
+            rows.append([float(x) for x in line.split()[:6]])
+    a = np.array(rows)
+    r, adv, w, mask, term, clipped = (a[:, i] for i in range(6))
+    out = S.clipped_surrogate(r, adv, mask, w, 0.8, 1.2)
+    assert np.allclose(out["terms"], term, rtol=0, atol=1e-6)
+    assert np.array_equal(out["clip_mask"] != 0, clipped != 0)
+    assert abs(out["loss"] - 0.3 / 7) < 1e-6
+    assert out["n_valid"] == 7 and out["clipped_pos"] == 2 and out["clipped_neg"] == 2
+
+
+def test_unclipped_ratio_one():
+    rng = np.random.default_rng(0)
+    adv = rng.standard_normal(100).astype(np.float32)
+    w = rng.uniform(0.5, 2, 100).astype(np.float32)
+    mask = (rng.random(100) < 0.8).astype(np.uint8)
+    out = S.clipped_surrogate(np.ones(100, np.float32), adv, mask, w, 0.8, 1.2)
+    v = mask != 0
+    assert np.isclose(out["loss"], -np.sum(w[v].astype(np.float64) * adv[v]) / v.sum(), rtol=1e-14)
+    assert out["clipped_pos"] == 0 and out["clipped_neg"] == 0
+
+
+def test_zero_advantage_and_empty_mask():
+    out = S.clipped_surrogate(np.full(5, 3.0), np.zeros(5), np.ones(5), None, 0.8, 1.2)
+    assert out["loss"] == 0 and np.all(out["grad"] == 0) and np.all(out["clip_mask"] == 0)
+    out = S.clipped_surrogate(np.full(5, 3.0), np.ones(5), np.zeros(5), None, 0.8, 1.2)
+    assert out["loss"] == 0 and out["n_valid"] == 0
+
+
+@pytest.mark.parametrize("seed", range(5))
+def test_gradient_finite_difference(seed):
+    rng = np.random.default_rng(seed)
+    T = 40
+    logp_old = rng.normal(-3, 1, T)
+    logp = logp_old + rng.normal(0, 0.3, T)
+    adv = rng.standard_normal(T)
+    w = rng.uniform(0.5, 2, T)
+    mask = (rng.random(T) < 0.8).astype(np.uint8)
+    lo, hi = 0.8, 1.2
+    r = np.exp(logp - logp_old)
+    # keep away from the kinks so the finite difference is clean
+    near = (np.abs(r - lo) < 1e-3) | (np.abs(r - hi) < 1e-3)
+    logp[near] += 0.01
+
+    def loss(lp):
+        rr = np.exp(lp - logp_old)
+        lo64, hi64 = float(np.float32(lo)), float(np.float32(hi))
+        t = -w * np.minimum(rr * adv, np.clip(rr, lo64, hi64) * adv)
+        return np.sum(np.where(mask != 0, t, 0)) / max(1, mask.sum())
+
+    r = np.exp(logp - logp_old)
+    # gradient of the oracle, evaluated in float64 terms
+    out = S.clipped_surrogate(r, adv, mask, w, lo, hi)
+    h = 1e-7
+    for t in range(T):
+        e = np.zeros(T)
+        e[t] = h
+        fd = (loss(logp + e) - loss(logp - e)) / (2 * h)
+        assert abs(fd - out["grad"][t]) < 5e-6 * max(1, abs(fd)), t
