@@ -1,0 +1,431 @@
+"""Benchmark: scored tokens/s of the FP8 log-prob + Calibrated-Clipping path.
+
+One step = one pass of the whole hot path over one synthetic batch of the
+8B-shaped GRPO workload (T = 16384 tokens, hidden 4096, vocab 151936, 1x128 /
+128x128 block E4M3 scaling): quantise h, quantise W, FP8 GEMM with streaming
+logsumexp + target gather, combine into log-probs and ratios, calibrate the
+clip bounds, clipped surrogate with token-mean loss, clip counts and
+dloss/dlogp.  Inputs are resident in HBM when the timed region starts (the W
+codes alone, 622 MB, exceed L2, so no flush is needed); ``e2e`` repeats the
+measurement with the per-step inputs in pinned host memory, copied in and the
+result read back inside the timed region.
+
+--impl reference times the CPU oracle on the host cores instead (bounded
+samples of the same workload, extrapolated to a full step).
+Multi-GPU (torchrun): every rank runs its own replica of the workload (weak
+scaling, no collective on the data path); value = all tokens / max rank time.
+"""
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "scored tokens/sec (FP8 logprob+calibrated-clip loss) at 8B shape; % FP8 peak, % HBM"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+FP8_OVER_BF16 = 4.5 / 2.25  # nominal dense FP8 / BF16 tensor rates
+GRAN_NAMES = {0: "tensor", 1: "row", 2: "block"}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def workload_desc(w):
+    lm = f", length mask U[{w.length_mask[0]},{w.length_mask[1]}]" if w.length_mask else ""
+    flt = ", all-equal groups masked (DAPO filter)" if w.filter_equal_groups else ""
+    return (f"{w.name}: T={w.T}, H={w.H}, V={w.V}, {GRAN_NAMES[w.gran]} E4M3 scaling, "
+            f"{w.prompts}x{w.group} responses x {w.resp_len}, rewards Bern({w.reward_p}), "
+            f"eps_low={w.eps_low}, eps_high={w.eps_high}{lm}{flt}")
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    """nvidia-smi samples (200 ms) during the timed region."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ our arm
+def bf16_reference_logprobs(h, W, y, chunk=16384):
+    """Stand-in for the BF16 shadow pass that feeds r_bf16 (input preparation,
+    untimed): log-softmax of the bf16 h @ W^T with fp32 accumulation (TF32
+    multiplies are exact on bf16-valued operands)."""
+    import torch
+    prev = torch.backends.cuda.matmul.allow_tf32
+    torch.backends.cuda.matmul.allow_tf32 = True
+    T = h.shape[0]
+    m = torch.full((T,), -float("inf"), device=h.device)
+    s = torch.zeros(T, device=h.device)
+    zy = torch.zeros(T, device=h.device)
+    hf = h.float()
+    yl = y.long()
+    for v0 in range(0, W.shape[0], chunk):
+        z = hf @ W[v0:v0 + chunk].float().T
+        cm = z.max(dim=1).values
+        mn = torch.maximum(m, cm)
+        s = s * torch.exp(m - mn) + torch.exp(z - mn[:, None]).sum(1)
+        m = mn
+        inside = (yl >= v0) & (yl < v0 + z.shape[1])
+        idx = (yl - v0).clamp(0, z.shape[1] - 1)
+        zy = torch.where(inside, z.gather(1, idx[:, None])[:, 0], zy)
+        del z
+    torch.backends.cuda.matmul.allow_tf32 = prev
+    return zy - (m + torch.log(s))
+
+
+def kernels_per_step(gran, mode):
+    q = 2 if gran == 0 else 1
+    calib = 6 if mode == 1 else 18
+    return 2 * q + 2 + calib + 2
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+    from paper_2609_22870_gb300 import api, synth
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    w = synth.WORKLOADS[args.workload]
+    if args.gran is not None:
+        w = synth.granularity_sweep(args.gran) if args.workload == "grpo_8b" else w
+    T, H, V, gran = w.T, w.H, w.V, w.gran
+    h = synth.hidden_states(w, dev)
+    W = synth.lm_head_weight(w, dev)
+    y = synth.targets(w, dev)
+    adv, mask = synth.rollout(w)
+    noise = synth.old_policy_noise(w)
+    logp_bf16 = bf16_reference_logprobs(h, W, y)
+    logp_old = (logp_bf16 + noise.to(dev)).float()
+    r_bf16 = torch.exp(logp_bf16 - logp_old).float()
+    coef = torch.exp(logp_old).float()  # TIS weight 1 (sampler = old policy) times pi_sampler
+    adv_d, mask_d = adv.to(dev), mask.to(dev)
+    opts = api.calib_opts(mode=args.calib_mode)
+    b = api.StepBuffers(T, H, V, gran, dev)
+    stream = torch.cuda.current_stream()
+
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(7)]
+
+    def step(record=False):
+        if record:
+            ev[0].record(stream)
+        api.quantize(h, gran, api.ROLE_ACT, b.h_codes, b.h_scales, b.q_ws)
+        if record:
+            ev[1].record(stream)
+        api.quantize(W, gran, api.ROLE_WEIGHT, b.w_codes, b.w_scales, b.q_ws)
+        if record:
+            ev[2].record(stream)
+        api.logit_partials(b.h_codes, b.h_scales, b.w_codes, b.w_scales, gran, y, b.lp_ws)
+        if record:
+            ev[3].record(stream)
+        api.combine_logprobs(T, H, V, gran, y, b.lp_ws, logp_old, b.logp, b.lse, b.ratio)
+        if record:
+            ev[4].record(stream)
+        api.calibrate_clip_bounds(b.ratio, r_bf16, adv_d, mask_d, coef, w.eps_low, w.eps_high, opts,
+                                  b.cal_res, b.cal_ws)
+        if record:
+            ev[5].record(stream)
+        api.clipped_surrogate(b.ratio, adv_d, mask_d, None, bounds=api.bounds_view(b.cal_res),
+                              stats=b.stats, workspace=b.sur_ws,
+                              out={"grad": b.grad, "clip_mask": b.clip_mask})
+        if record:
+            ev[6].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    api.check()
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    per_step_events = []
+    t0.record(stream)
+    for _ in range(args.steps):
+        ev[:] = [torch.cuda.Event(enable_timing=True) for _ in range(7)]
+        step(record=True)
+        per_step_events.append(list(ev))
+    t1.record(stream)
+    torch.cuda.synchronize()
+    stage = np.zeros(6)
+    for evs in per_step_events:
+        stage += [evs[i].elapsed_time(evs[i + 1]) for i in range(6)]
+    clk = clocks.stop()
+    elapsed_ms = t0.elapsed_time(t1)
+    api.check()
+
+    # same step through the public API with host buffers (copies inside the region)
+    pin = lambda t: t.cpu().pin_memory()  # noqa: E731
+    host = {"h": pin(h), "y": pin(y), "logp_old": pin(logp_old), "r_bf16": pin(r_bf16),
+            "adv": pin(adv), "mask": pin(mask), "coef": pin(coef)}
+    devin = {k: torch.empty_like(v, device=dev) for k, v in host.items()}
+    out_host = {"stats": torch.empty(b.stats.numel(), dtype=torch.uint8).pin_memory(),
+                "cal": torch.empty(b.cal_res.numel(), dtype=torch.uint8).pin_memory(),
+                "grad": torch.empty(T, dtype=torch.float32).pin_memory()}
+    h2d = sum(v.numel() * v.element_size() for v in host.values())
+    d2h = sum(v.numel() * v.element_size() for v in out_host.values())
+
+    def e2e_step():
+        for k in host:
+            devin[k].copy_(host[k], non_blocking=True)
+        api.score_calibrate_loss(devin["h"], W, devin["y"], devin["logp_old"], devin["r_bf16"],
+                                 devin["adv"], devin["mask"], devin["coef"], gran, w.eps_low,
+                                 w.eps_high, opts, b)
+        out_host["stats"].copy_(b.stats, non_blocking=True)
+        out_host["cal"].copy_(b.cal_res, non_blocking=True)
+        out_host["grad"].copy_(b.grad, non_blocking=True)
+
+    for _ in range(max(1, args.warmup)):
+        e2e_step()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / args.steps
+    api.check()
+    res = api.read_calib_result(b.cal_res)
+    st = api.read_clip_stats(b.stats)
+
+    ms = elapsed_ms / args.steps
+    if world > 1:
+        t = torch.tensor([ms, e2e_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms, e2e_ms = float(t[0]), float(t[1])
+    if rank != 0:
+        return None
+    stage /= args.steps
+    gemm_ms = stage[2]
+    flops = 2.0 * T * H * V
+    peaks, peak_src = load_peaks()
+    fp8_peak = peaks["bf16_tflops_sustained"] * FP8_OVER_BF16
+    achieved = flops / (gemm_ms * 1e-3) / 1e12
+    line = {
+        "metric": METRIC,
+        "value": world * T / (ms * 1e-3),
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "fp8_e4m3 (fp32 accumulate)",
+        "data": "synthetic",
+        "config": {"workload": workload_desc(w), "T": T, "H": H, "V": V,
+                   "granularity": GRAN_NAMES[gran],
+                   "calib_mode": "grid" if args.calib_mode == 1 else "exact",
+                   "parallelism": f"replicas x{world}",
+                   "l2": "inputs larger than L2 (W codes 622 MB, bf16 W 1.2 GB); no flush",
+                   "r_bf16": "from a torch bf16 reference scoring pass, untimed input preparation"},
+        "roofline": {"bound": "tensor", "kernel": "fp8_gemm_kernel (logit partials)",
+                     "achieved": achieved, "peak": fp8_peak, "unit": "TFLOP/s",
+                     "frac": achieved / fp8_peak,
+                     "peak_source": f"{peak_src} bf16 sustained x {FP8_OVER_BF16:g} (nominal FP8/BF16)",
+                     "traffic": None},
+        "stages_ms": {"quantize_h": stage[0], "quantize_w": stage[1], "gemm_lse": stage[2],
+                      "combine": stage[3], "calibrate": stage[4], "surrogate": stage[5]},
+        "e2e": {"value": world * T / (e2e_ms * 1e-3), "unit": "tokens/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "note": "h, targets, logp_old, r_bf16, adv, mask, coef copied in; stats, bounds, "
+                        "dloss/dlogp read back; lm_head W is resident model state"},
+        "gpu_launches": kernels_per_step(gran, args.calib_mode) * args.steps,
+        "clocks": clk,
+        "result": {"lo": res["lo_new"], "hi": res["hi_new"], "loss": st["loss"],
+                   "clip_frac_pos": st["clip_frac_pos"], "clip_frac_neg": st["clip_frac_neg"]},
+    }
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = oracle_step_estimate(w, budget_s=args.cpu_budget)
+    return line
+
+
+# ------------------------------------------------------------------ oracle arm
+def oracle_step_estimate(w, budget_s=20.0, seed=0):
+    """Times the CPU oracle on a bounded sample of the workload and extrapolates
+    to one full step: W quantisation and scoring are timed on a sample of
+    128-row vocabulary strips and token rows (cost linear in both), calibration
+    and the surrogate run on all T tokens (synthetic ratios of the same size)."""
+    import torch
+    from oracle import calibrate as OC
+    from oracle import logprobs as OL
+    from oracle import quantize as OQ
+    from oracle import surrogate as OS
+    from paper_2609_22870_gb300 import synth
+
+    rng = np.random.default_rng(seed)
+    n_rows = min(w.T, 512)
+    h = synth.normal_bf16(n_rows, w.H, 1.0, 1, "cpu").float().numpy()
+    t = time.perf_counter()
+    hq, hs = OQ.quantize(h, w.gran, OQ.ACT)
+    t_qh = (time.perf_counter() - t) / n_rows
+    order = rng.permutation(w.V // 128)
+    t_qw = t_gemm = 0.0
+    n_strips = 0
+    t_start = time.perf_counter()
+    for sidx in order:  # as many strips as the time budget allows
+        Wx = synth.normal_bf16(128, w.H, 0.02, int(sidx), "cpu").float().numpy()
+        t = time.perf_counter()
+        wq, ws = OQ.quantize(Wx, w.gran, OQ.WEIGHT)
+        t_qw += time.perf_counter() - t
+        t = time.perf_counter()
+        z = OL.logits(hq, hs, wq, ws, w.gran)
+        OL.log_softmax_gather(z, np.zeros(n_rows, np.int64))
+        t_gemm += time.perf_counter() - t
+        n_strips += 1
+        if time.perf_counter() - t_start >= budget_s:
+            break
+    frac = (w.V / 128) / n_strips
+    t_qw_full = t_qw * frac
+    t_score_full = t_gemm * frac * (w.T / n_rows)
+    adv, mask = synth.rollout(w)
+    r_bf, r_fp, coef = synth.ratio_inputs(w.T, 3)
+    t = time.perf_counter()
+    res = OC.calibrate_clip_bounds(r_fp.numpy(), r_bf.numpy(), adv.numpy(), mask.numpy(), coef.numpy(),
+                                   w.eps_low, w.eps_high)
+    t_cal = time.perf_counter() - t
+    t = time.perf_counter()
+    OS.clipped_surrogate(r_fp.numpy(), adv.numpy(), mask.numpy(), None, res["lo_new"], res["hi_new"])
+    t_loss = time.perf_counter() - t
+    step_s = t_qh * w.T + t_qw_full + t_score_full + t_cal + t_loss
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    return {"value": w.T / step_s, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": (f"{n_strips}/{w.V // 128} W strips of 128 rows quantised and scored against "
+                       f"{n_rows} token rows (numpy float64, BLAS threads up to {cores}); calibrate + "
+                       f"surrogate on all {w.T} tokens; full step extrapolated linearly "
+                       f"({step_s:.1f} s/step)"),
+            "step_seconds": step_s}
+
+
+def run_reference(args, rank, world):
+    from paper_2609_22870_gb300 import synth
+    if rank != 0:
+        return None
+    w = synth.WORKLOADS[args.workload]
+    per_step = max(2.0, 150.0 / max(1, args.steps + args.warmup))
+    for i in range(args.warmup):
+        oracle_step_estimate(w, budget_s=per_step, seed=100 + i)
+    vals = []
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        vals.append(oracle_step_estimate(w, budget_s=per_step, seed=i))
+    wall = time.perf_counter() - t0
+    v = statistics.median(x["value"] for x in vals)
+    step_s = statistics.median(x["step_seconds"] for x in vals)
+    cb = dict(vals[0])
+    cb["value"] = v
+    return {"impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_s * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "float64 (oracle)", "data": "synthetic",
+            "config": {"workload": workload_desc(w), "T": w.T, "H": w.H, "V": w.V,
+                       "granularity": GRAN_NAMES[w.gran]},
+            "cpu_baseline": cb, "sample_wall_seconds": wall,
+            "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="grpo_8b")
+    ap.add_argument("--gran", type=int, default=None, help="override granularity (0/1/2) of grpo_8b")
+    ap.add_argument("--calib-mode", type=int, default=0)
+    ap.add_argument("--cpu-budget", type=float, default=20.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(3, args.warmup)
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        line = run_reference(args, rank, world)
+    else:
+        import torch
+        if world > 1:
+            import torch.distributed as dist
+            torch.cuda.set_device(local_rank)
+            dist.init_process_group("nccl")
+        line = run_ours(args, rank, world, local_rank)
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+    if line is not None:
+        print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,305 @@
+/*
+ * fp8rl.h -- C ABI of libfp8rl.so: FP8 token scoring followed by Calibrated
+ * Clipping, as in "Towards Full Pipeline FP8 Reinforcement Learning for LLMs".
+ *
+ * The library runs every step on the GPU (NVIDIA GB300, sm_103a).  All tensor
+ * pointers are DEVICE pointers owned by the caller unless a comment says
+ * "host".  The library keeps no device allocation of its own besides a few
+ * status words; scratch memory comes from the caller as a workspace whose size
+ * the matching *_workspace_size() query returns (any alignment of 256 bytes or
+ * more; the library zeroes what it needs itself).
+ *
+ * Every compute call is asynchronous on `stream` (a cudaStream_t; NULL is the
+ * legacy default stream) and returns host-detectable errors synchronously:
+ * null pointers, unsupported shapes, misalignment, a short workspace, a
+ * failed launch.  Errors found by a kernel (bad target ids, non-finite or
+ * negative inputs where the method forbids them, an expired bounded wait) set
+ * a device status word and never trap; fp8rl_check() reports and clears it.
+ * Outputs of a call that flagged an error are unspecified (NaN where noted).
+ * No C++ exception crosses this interface.
+ *
+ * Paper references are to sections, equations and Algorithm 1 of the paper.
+ */
+#ifndef FP8RL_H_
+#define FP8RL_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum fp8rl_status {
+  FP8RL_OK = 0,
+  FP8RL_EINVAL = 1,     /* null pointer, unknown enum value, negative size       */
+  FP8RL_ESHAPE = 2,     /* shape outside what the call supports                  */
+  FP8RL_EALIGN = 3,     /* pointer or leading dimension not 16-byte aligned      */
+  FP8RL_EWORKSPACE = 4, /* workspace null or smaller than the size query         */
+  FP8RL_ECUDA = 5,      /* a CUDA runtime / driver call failed                   */
+  FP8RL_EDEVICE = 6,    /* a kernel flagged bad input data (from fp8rl_check)    */
+  FP8RL_ETIMEOUT = 7    /* a bounded in-kernel wait expired (from fp8rl_check)   */
+} fp8rl_status;
+
+/* Scaling granularity of Eq. 3 (§2.2): one scale per tensor, per row, or per
+ * block.  For the lm_head operands "row" means one scale per token of h[T][H]
+ * and one per vocabulary row (output channel) of W[V][H]; "block" means 1x128
+ * blocks of h and 128x128 blocks of W. */
+typedef enum fp8rl_gran {
+  FP8RL_GRAN_TENSOR = 0,
+  FP8RL_GRAN_ROWWISE = 1,
+  FP8RL_GRAN_BLOCK = 2
+} fp8rl_gran;
+
+/* Operand role, which fixes the block shape and scale layout in block mode. */
+typedef enum fp8rl_role {
+  FP8RL_ROLE_ACT = 0,    /* hidden states h[T][H]: 1x128 blocks    */
+  FP8RL_ROLE_WEIGHT = 1  /* lm_head weight W[V][H]: 128x128 blocks */
+} fp8rl_role;
+
+/* ---------------------------------------------------------------------- */
+/* Status                                                                   */
+/* ---------------------------------------------------------------------- */
+
+/* Synchronises `stream`, then reads and clears the device status words that
+ * kernels of this library set.  Returns FP8RL_ETIMEOUT if any bounded wait
+ * expired, else FP8RL_EDEVICE if any kernel flagged bad input, else
+ * FP8RL_ECUDA if the synchronisation failed, else FP8RL_OK. */
+fp8rl_status fp8rl_check(void* stream);
+
+/* Static description of a status code (never NULL). */
+const char* fp8rl_status_string(fp8rl_status status);
+
+/* Text of the last CUDA error seen by the calling host thread inside this
+ * library ("" if none).  Valid until the next call on the same thread. */
+const char* fp8rl_last_cuda_error(void);
+
+/* ---------------------------------------------------------------------- */
+/* a1/a2: scaled E4M3 quantisation (Eq. 3, §2.2)                            */
+/* ---------------------------------------------------------------------- */
+
+/* Number of float scales fp8rl_quantize writes for this shape (0 on bad
+ * arguments):
+ *   TENSOR              1                       scales[0]
+ *   ROWWISE             rows                    scales[r]
+ *   BLOCK, ROLE_ACT     rows * (cols/128)       scales[kb * rows + r]   (block-column major)
+ *   BLOCK, ROLE_WEIGHT  ceil(rows/128)*(cols/128) scales[rb * (cols/128) + kb]
+ */
+int64_t fp8rl_scales_count(int64_t rows, int64_t cols, fp8rl_gran gran, fp8rl_role role);
+
+size_t fp8rl_quantize_workspace_size(int64_t rows, int64_t cols, fp8rl_gran gran, fp8rl_role role);
+
+/* Eq. 3: S = max|X| / 448 over each block, codes = Q_FP8(X / S).
+ *   x       bf16 [rows][ld] row-major (first `cols` of each row are used);
+ *           16-byte aligned, ld % 8 == 0
+ *   codes   E4M3 bytes [rows][cols] row-major, 16-byte aligned
+ *   scales  float32, count and layout as fp8rl_scales_count() says
+ * S = fl32(amax / 448) (S = 1 when amax == 0); each code is the
+ * round-to-nearest-even, saturating (+-448) E4M3 encoding of the correctly
+ * rounded float32 quotient x / S.  Requires cols % 16 == 0, and cols % 128 == 0
+ * in block mode.  A tail block of W along rows (rows % 128 != 0) takes its
+ * amax over the rows present.  Non-finite x sets FP8RL_EDEVICE. */
+fp8rl_status fp8rl_quantize(const void* x, int64_t rows, int64_t cols, int64_t ld,
+                            fp8rl_gran gran, fp8rl_role role,
+                            uint8_t* codes, float* scales,
+                            void* workspace, size_t workspace_bytes, void* stream);
+
+/* ---------------------------------------------------------------------- */
+/* a3/a4: FP8 lm_head scoring with online logsumexp and target gather       */
+/* ---------------------------------------------------------------------- */
+
+/* The token ratio of §2.1 needs pi(y_t | h_t) under the FP8 forward pass of §3:
+ *   z[t][v]  = sum_k S_h S_W q_h[t][k] q_W[v][k]   (fp32 accumulation on the
+ *              FP8 tensor cores; in block mode per 128-wide K block)
+ *   lse[t]   = log sum_v exp(z[t][v])
+ *   logp[t]  = z[t][y_t] - lse[t]
+ *   ratio[t] = exp(logp[t] - logp_old[t])
+ * computed without ever storing z: each 128-column vocabulary chunk leaves
+ * one (max, sum-exp) pair per token in the workspace, merged afterwards.
+ *
+ *   h_codes/h_scales  from fp8rl_quantize(h[T][H], gran, FP8RL_ROLE_ACT)
+ *   w_codes/w_scales  from fp8rl_quantize(W[V][H], gran, FP8RL_ROLE_WEIGHT)
+ *   targets           int32 [T], each in [0, V)  (else FP8RL_EDEVICE, logp NaN)
+ *   logp_old          float [T] or NULL
+ *   logp              float [T] out
+ *   lse               float [T] out, or NULL
+ *   ratio             float [T] out, or NULL (needs logp_old)
+ * Requires T >= 1, V >= 1, H >= 16, H % 16 == 0 (H % 128 == 0 in block mode),
+ * code pointers 16-byte aligned.  Temperature 1. */
+size_t fp8rl_token_logprobs_workspace_size(int64_t T, int64_t H, int64_t V, fp8rl_gran gran);
+
+fp8rl_status fp8rl_token_logprobs(const uint8_t* h_codes, const float* h_scales,
+                                  const uint8_t* w_codes, const float* w_scales,
+                                  fp8rl_gran gran, int64_t T, int64_t H, int64_t V,
+                                  const int32_t* targets, const float* logp_old,
+                                  float* logp, float* lse, float* ratio,
+                                  void* workspace, size_t workspace_bytes, void* stream);
+
+/* The two halves of fp8rl_token_logprobs, for callers that time or overlap
+ * them separately: the FP8 GEMM with its streaming logsumexp epilogue leaves
+ * per-chunk partials and z[t][y_t] in the workspace; the combine merges them.
+ * Pass the same arguments and workspace to both, in this order. */
+fp8rl_status fp8rl_logit_partials(const uint8_t* h_codes, const float* h_scales,
+                                  const uint8_t* w_codes, const float* w_scales,
+                                  fp8rl_gran gran, int64_t T, int64_t H, int64_t V,
+                                  const int32_t* targets,
+                                  void* workspace, size_t workspace_bytes, void* stream);
+
+fp8rl_status fp8rl_combine_logprobs(int64_t T, int64_t H, int64_t V, fp8rl_gran gran,
+                                    const int32_t* targets, const float* logp_old,
+                                    float* logp, float* lse, float* ratio,
+                                    void* workspace, size_t workspace_bytes, void* stream);
+
+/* r_t = exp(logp_new_t - logp_old_t) (§2.1), float [T]. */
+fp8rl_status fp8rl_importance_ratios(const float* logp_new, const float* logp_old,
+                                     int64_t T, float* ratio, void* stream);
+
+/* ---------------------------------------------------------------------- */
+/* a5: Calibrated Clipping (§4, Eq. 5, Algorithm 1)                         */
+/* ---------------------------------------------------------------------- */
+
+typedef enum fp8rl_calib_mode {
+  FP8RL_CALIB_EXACT = 0, /* search every float32 threshold in I_L / I_H (default) */
+  FP8RL_CALIB_GRID = 1   /* Algorithm 1's grid with step `step`                  */
+} fp8rl_calib_mode;
+
+/* Host-side options; fp8rl_default_calib_opts() fills the paper's values. */
+typedef struct fp8rl_calib_opts {
+  int32_t mode;          /* fp8rl_calib_mode                                   */
+  int32_t reserved;      /* must be 0                                          */
+  double lo_min, lo_max; /* I_L = [0.5, 0.9]                                   */
+  double hi_min, hi_max; /* I_H = [1.2, 2.0]                                   */
+  double step;           /* Delta = 0.02 (grid mode)                           */
+  double delta_lo;       /* SmoothUpdate limit for L, 0.05                     */
+  double delta_hi;       /* SmoothUpdate limit for H, 0.1                      */
+  float lo_old, hi_old;  /* previous bounds; NaN = none (new = searched bound) */
+} fp8rl_calib_opts;
+
+/* Written to device memory by fp8rl_calibrate_clip_bounds.  The first two
+ * fields are the bounds to clip with, so (const float*)result can be passed as
+ * `bounds` to fp8rl_clipped_surrogate. */
+typedef struct fp8rl_calib_result {
+  float lo_new, hi_new;   /* SmoothUpdate(L_old, L*, dL), SmoothUpdate(H_old, H*, dH) */
+  float lo_star, hi_star; /* searched bounds L*, H*                                   */
+  float c_lo, c_hi;       /* reference bounds fl32(1 - eps_low), fl32(1 + eps_high)   */
+  int32_t flags;          /* FP8RL_CALIB_FLAG_* bits                                  */
+  int32_t shift;          /* fixed-point shift s of the Eq. 5 sums                    */
+  int64_t n_neg, n_pos;   /* valid tokens with A < 0, A > 0                           */
+  int64_t k_bf16;         /* #{A<0 : r_bf16 <= c_lo}  (alpha_low = k_bf16 / n_neg)    */
+  int64_t k_fp8;          /* #{A<0 : r_fp8 <= L*}                                     */
+  int64_t sum_pos_bf16;   /* N_bf  = sum_{A>0, r_bf16 < c_hi} q   (q = RNE(e 2^s))    */
+  int64_t sum_neg_bf16;   /* D_bf  = |sum_{A<0, r_bf16 > c_lo} q|                     */
+  int64_t sum_neg_fp8;    /* D_fp8 = |sum_{A<0, r_fp8 > L*} q|                        */
+  int64_t sum_pos_fp8;    /* P     = sum_{A>0, r_fp8 < H*} q                          */
+  double rho_bf16;        /* N_bf / D_bf                                              */
+  double rho_fp8;         /* P / D_fp8                                                */
+} fp8rl_calib_result;
+
+#define FP8RL_CALIB_FLAG_NO_NEG 1       /* no A<0 token: L* = c_lo (clamped to I_L) */
+#define FP8RL_CALIB_FLAG_NO_POS 2       /* no A>0 token: H* = c_hi (clamped to I_H) */
+#define FP8RL_CALIB_FLAG_ZERO_D_BF16 4  /* D_bf = 0: rho_BF16 undefined, H* = c_hi  */
+#define FP8RL_CALIB_FLAG_ZERO_D_FP8 8   /* D_fp8 = 0: rho_FP8 undefined, H* = c_hi  */
+
+void fp8rl_default_calib_opts(fp8rl_calib_opts* opts);
+
+size_t fp8rl_calibrate_workspace_size(int64_t T);
+
+/* Algorithm 1.  Inputs, float [T] unless noted:
+ *   r_fp8, r_bf16  importance ratios from the FP8 path and the BF16 shadow pass
+ *   adv            advantages A_t
+ *   mask           uint8 [T], 1 = valid token (NULL = all valid)
+ *   coef           w_t^TIS * pi_sampler(y_t|h_t) of Eq. 5 (NULL = 1)
+ *   opts           HOST pointer, NULL = fp8rl_default_calib_opts()
+ *   result         DEVICE pointer to one fp8rl_calib_result
+ * Stage 1 (§4): k = #{A<0 : r_bf16 <= c_lo}; L* minimises
+ * |#{A<0 : r_fp8 <= L} - k| over L in I_L (every float32 in EXACT mode, the
+ * grid in GRID mode); among minimisers the one nearest c_lo, then the smaller.
+ * Stage 2 (Eq. 5): e_t = (coef_t r_t) A_t in float64, rounded to integers
+ * q_t = RNE(e_t 2^s) with one shift s per call so no sum overflows; H*
+ * minimises |P(H) D_bf - N_bf D_fp8| (= |rho_FP8 - rho_BF16| D_bf D_fp8) over H
+ * in I_H, ties to the point nearest c_hi, then the smaller.  Then SmoothUpdate.
+ * Ratios and coef must be finite and >= 0, advantages finite (else
+ * FP8RL_EDEVICE).  T >= 0. */
+fp8rl_status fp8rl_calibrate_clip_bounds(const float* r_fp8, const float* r_bf16,
+                                         const float* adv, const uint8_t* mask,
+                                         const float* coef, int64_t T,
+                                         float eps_low, float eps_high,
+                                         const fp8rl_calib_opts* opts,
+                                         fp8rl_calib_result* result,
+                                         void* workspace, size_t workspace_bytes,
+                                         void* stream);
+
+/* ---------------------------------------------------------------------- */
+/* a6/a7: clipped surrogate, clip fractions, dLoss/dlogp (Eq. 1, Eq. 4)      */
+/* ---------------------------------------------------------------------- */
+
+/* Device-resident statistics of one fp8rl_clipped_surrogate call. */
+typedef struct fp8rl_clip_stats {
+  double loss;           /* sum_valid l_t / n_valid (0 when n_valid == 0) */
+  double loss_sum;       /* sum_valid l_t                                 */
+  int64_t n_valid, n_pos, n_neg;
+  int64_t clipped_pos;   /* A > 0 and r >= H   */
+  int64_t clipped_neg;   /* A < 0 and r <= L   */
+  float lo, hi;          /* bounds used        */
+  int32_t flags;         /* 1 = no valid token */
+  int32_t reserved;
+} fp8rl_clip_stats;
+
+#define FP8RL_CLIP_HI 1  /* clip-mask bit: A > 0 and r >= H */
+#define FP8RL_CLIP_LO 2  /* clip-mask bit: A < 0 and r <= L */
+
+size_t fp8rl_surrogate_workspace_size(int64_t T);
+
+/* l_t = -w_t min(r_t A_t, clip(r_t, L, H) A_t) (Eq. 1 with the TIS weight of
+ * Eq. 4 and calibrated bounds), loss = sum_valid l_t / n_valid (token mean,
+ * float64 accumulation, deterministic for a given T).
+ *   r, adv       float [T];  mask uint8 [T] or NULL;  w_tis float [T] or NULL (1)
+ *   lo, hi       bounds by value, used when `bounds` is NULL
+ *   bounds       DEVICE float[2] {L, H} or NULL (e.g. a fp8rl_calib_result*)
+ *   grad_logp    float [T] out or NULL: dloss/dlogp_t = -w A r / n_valid on
+ *                unclipped valid tokens, 0 elsewhere.  With lse from
+ *                fp8rl_token_logprobs this is dLoss/dlogits in factored form:
+ *                dLoss/dz[t][v] = grad_logp[t] (1{v == y_t} - exp(z[t][v] - lse[t])).
+ *   clip_mask    uint8 [T] out or NULL: FP8RL_CLIP_HI / FP8RL_CLIP_LO bits
+ *   stats        DEVICE pointer to one fp8rl_clip_stats */
+fp8rl_status fp8rl_clipped_surrogate(const float* r, const float* adv, const uint8_t* mask,
+                                     const float* w_tis, int64_t T, float lo, float hi,
+                                     const float* bounds, float* grad_logp, uint8_t* clip_mask,
+                                     fp8rl_clip_stats* stats,
+                                     void* workspace, size_t workspace_bytes, void* stream);
+
+/* Dense dLoss/dlogits for selected rows (a verification and debugging path;
+ * the hot path keeps the factored form above).  For i < n_rows, t = rows[i]:
+ *   out[i][v] = grad_logp[t] * (1{v == y_t} - exp(z[t][v] - lse[t])),  v < V,
+ * with z recomputed by the same FP8 GEMM as fp8rl_token_logprobs.
+ *   rows  int64 [n_rows] DEVICE, each in [0, T)    out float [n_rows][V] */
+size_t fp8rl_dlogits_workspace_size(int64_t n_rows, int64_t H, int64_t V, fp8rl_gran gran);
+
+fp8rl_status fp8rl_dlogits_rows(const uint8_t* h_codes, const float* h_scales,
+                                const uint8_t* w_codes, const float* w_scales,
+                                fp8rl_gran gran, int64_t T, int64_t H, int64_t V,
+                                const int32_t* targets, const float* lse,
+                                const float* grad_logp, const int64_t* rows, int64_t n_rows,
+                                float* out, void* workspace, size_t workspace_bytes,
+                                void* stream);
+
+/* ---------------------------------------------------------------------- */
+/* Bounded waits                                                            */
+/* ---------------------------------------------------------------------- */
+
+/* Every spin-wait in this library's kernels gives up after this many
+ * nanoseconds of GPU time (default 2e9), sets FP8RL_ETIMEOUT and returns after
+ * draining its own in-flight copies.  Process-wide; 0 restores the default. */
+void fp8rl_set_wait_limit_ns(uint64_t limit_ns);
+
+/* Launches one CTA that waits, with the bounded wait every kernel here uses,
+ * on a barrier nothing will signal; the wait expires after `limit_ns`, so a
+ * following fp8rl_check() returns FP8RL_ETIMEOUT and the context stays
+ * usable.  Used to test the timeout path without hanging a GPU. */
+fp8rl_status fp8rl_wait_selftest(uint64_t limit_ns, void* stream);
+
+#ifdef __cplusplus
+} /* extern "C" */
+#endif
+
+#endif /* FP8RL_H_ */

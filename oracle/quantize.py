@@ -80,17 +80,17 @@ def quantize(x, gran, role=ACT):
         s = scale_from_amax(np.max(np.abs(xb), axis=2))  # (rows, nkb)
         codes = _encode_block(xb, s[:, :, None]).reshape(rows, cols)
         return codes, s
-    # weight: 128 x 128 blocks, tail rows along V allowed
+    # weight: 128 x 128 blocks, tail rows along V allowed; one 128-row strip
+    # (all its blocks) at a time
     nrb = (rows + BLOCK_W - 1) // BLOCK_W
     s = np.empty((nrb, nkb), dtype=np.float32)
     codes = np.empty((rows, cols), dtype=np.uint8)
     for rb in range(nrb):
         r0, r1 = rb * BLOCK_W, min(rows, (rb + 1) * BLOCK_W)
-        for kb in range(nkb):
-            blk = x[r0:r1, kb * BLOCK_K:(kb + 1) * BLOCK_K]
-            sb = scale_from_amax(np.max(np.abs(blk)))
-            s[rb, kb] = sb
-            codes[r0:r1, kb * BLOCK_K:(kb + 1) * BLOCK_K] = _encode_block(blk, sb)
+        strip = x[r0:r1].reshape(r1 - r0, nkb, BLOCK_K)
+        sb = scale_from_amax(np.max(np.abs(strip), axis=(0, 2)))  # (nkb,)
+        s[rb] = sb
+        codes[r0:r1] = _encode_block(strip, sb[None, :, None]).reshape(r1 - r0, cols)
     return codes, s
 
 

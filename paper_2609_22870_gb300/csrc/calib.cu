@@ -1,0 +1,753 @@
+// a5: Calibrated Clipping (§4, Eq. 5, Algorithm 1) on the GPU.
+//
+// Stage 1 (lower-bound alignment): k = #{A<0 : r_bf16 <= c_lo}; L* is the
+// float32 threshold in I_L minimising |#{A<0 : r_fp8 <= L} - k|, nearest c_lo.
+// Stage 2 (upper-bound rebalancing, Eq. 5): with e_t = (coef_t r_t) A_t
+// rounded to integers q_t = RNE(e_t 2^s), N_bf, D_bf, D_fp8 are exact sums and
+// H* is the float32 in I_H minimising |P(H) D_bf - N_bf D_fp8|,
+// P(H) = sum_{A>0, r_fp8 < H} q, nearest c_hi.  Then SmoothUpdate.
+//
+// EXACT mode finds each optimum with a weighted radix select over the float32
+// bit patterns of the ratios (non-negative floats order like their bits):
+// three histogram passes (11, 11, 10 bits) locate the smallest ratio u whose
+// cumulative weight crosses the target, one more pass finds u's neighbours and
+// the pieces of the step function that contain the ends of the search
+// interval, and a single-block decide step turns them into the bound.  Counts
+// and fixed-point sums are integers, so every reduction order gives the same
+// bits and the result is reproducible to the last bit.  GRID mode histograms
+// the ratios over Algorithm 1's candidate thresholds instead.
+//
+// Passes are grid-stride kernels with shared-memory histograms flushed by
+// atomics; decide steps run in one block of 1024 threads.
+#include <cmath>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace fp8rl {
+namespace {
+
+__device__ uint32_t d_status;
+
+constexpr int kBuckets = 2048;
+
+constexpr unsigned kNone = 0xFFFFFFFFu;
+
+enum Stage : int {
+  kPrep = 0,    // counts, emax, input checks; L histogram digit 0 / L grid counts
+  kSums = 1,    // N_bf, D_bf; L digit 1 (exact) | D_fp8, k_fp8, H grid sums (grid)
+  kL2 = 2,      // L digit 2
+  kLNb = 3,     // L neighbours
+  kH0 = 4,      // D_fp8, k_fp8, H digit 0
+  kH1 = 5,
+  kH2 = 6,
+  kHNb = 7,     // H neighbours
+  kPFin = 8     // P(H*)
+};
+
+struct State {
+  // accumulated by passes (zeroed before the first pass)
+  unsigned long long n_neg, n_pos, k_bf16, k_fp8;
+  unsigned long long emax_bits;
+  unsigned long long s_pos_bf, s_neg_bf, s_neg_fp, s_pos_fp;  // int64 two's complement
+  unsigned int bad;
+  unsigned int nb_below1;  // 1 + max{key < u} (0 = none)
+  unsigned int nb_above;   // min{key > u}     (kNone = none)
+  unsigned int nb_mpiece;  // L: min{key > key(lo_min)}   H: min{key >= key(hi_min), q > 0}
+  unsigned int nb_Mpiece1; // L: 1 + max{key <= key(lo_max)}   H: 1 + max{key < key(hi_max), q > 0}
+  unsigned int pad0;
+  // written by decide steps
+  int shift;
+  int found;
+  unsigned int prefix;
+  unsigned int u_key;
+  long long below;
+  long long p_lt, p_le;
+  unsigned long long tgt_hi, tgt_lo;  // X as unsigned 128-bit
+  long long dmul;                     // D
+  float lo_star, hi_star;
+  int flags;
+  int h_active;  // stage 2 runs (not degenerate)
+  int pad1;
+  // histograms
+  unsigned long long h_cnt[kBuckets];
+  unsigned long long h_w[kBuckets];
+};
+
+struct Args {
+  const float* r_fp8;
+  const float* r_bf16;
+  const float* adv;
+  const uint8_t* mask;
+  const float* coef;
+  int64_t T;
+  float c_lo, c_hi;
+  float lo_min, lo_max, hi_min, hi_max;
+  float delta_lo, delta_hi;
+  float lo_old, hi_old;
+  int grid_mode;
+  double lo_grid0, hi_grid0, step;  // Algorithm 1 grids: fl32(x0 + i * step)
+  int n_lcand, n_hcand;
+  State* st;
+  fp8rl_calib_result* out;
+};
+
+__device__ __forceinline__ void flag(uint32_t bits) { atomicOr(&d_status, bits); }
+
+__device__ __forceinline__ unsigned key_of(float r) { return __float_as_uint(r) & 0x7FFFFFFFu; }
+
+// q_t = RNE(((coef r) A) 2^s) -- float64 product, exact scaling, RNE to int64.
+__device__ __forceinline__ long long fixed_term(float c, float r, float a, int s) {
+  const double e = (static_cast<double>(c) * static_cast<double>(r)) * static_cast<double>(a);
+  return __double2ll_rn(ldexp(e, s));
+}
+
+__device__ __forceinline__ bool digit_match(unsigned key, int digit, unsigned prefix) {
+  if (digit == 0) return true;
+  if (digit == 1) return (key >> 21) == prefix;
+  return (key >> 10) == prefix;
+}
+
+__device__ __forceinline__ unsigned digit_of(unsigned key, int digit) {
+  if (digit == 0) return key >> 21;
+  if (digit == 1) return (key >> 10) & 0x7FFu;
+  return key & 0x3FFu;
+}
+
+// Candidate i of an Algorithm 1 grid, fl32(x0 + i * step) in float64.
+__device__ __forceinline__ float cand_at(double x0, double step, int i) {
+  return static_cast<float>(x0 + static_cast<double>(i) * step);
+}
+
+// First candidate index i with r <= cand(i) (strict=false) or r < cand(i)
+// (strict=true); n if none.  Candidates ascend.
+__device__ __forceinline__ int first_cand(double x0, double step, int n, float r, bool strict) {
+  int lo = 0, hi = n;
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    const float c = cand_at(x0, step, mid);
+    const bool ok = strict ? (r < c) : (r <= c);
+    if (ok) hi = mid; else lo = mid + 1;
+  }
+  return lo;
+}
+
+template <typename T>
+__device__ __forceinline__ T warp_sum(T v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// ------------------------------------------------------------------ passes
+__global__ void __launch_bounds__(256) pass_kernel(Args a, int stage) {
+  __shared__ unsigned long long sh_cnt[kBuckets];
+  __shared__ long long sh_w[kBuckets];
+  State* st = a.st;
+  if ((stage == kH1 || stage == kH2 || stage == kHNb) && !st->h_active) return;
+  const bool grid_mode = a.grid_mode != 0;
+  const bool want_hist = grid_mode ? (stage == kPrep || stage == kSums)
+                                   : (stage == kPrep || stage == kSums || stage == kL2 ||
+                                      stage == kH0 || stage == kH1 || stage == kH2);
+  if (want_hist) {
+    for (int i = threadIdx.x; i < kBuckets; i += blockDim.x) {
+      sh_cnt[i] = 0;
+      sh_w[i] = 0;
+    }
+    __syncthreads();
+  }
+  const int shift = st->shift;
+  const float lo_star = st->lo_star, hi_star = st->hi_star;
+  const unsigned prefix = st->prefix, u = st->u_key;
+  int digit = 0;
+  if (stage == kSums || stage == kH1) digit = 1;
+  if (stage == kL2 || stage == kH2) digit = 2;
+  const unsigned key_lm = key_of(a.lo_min), key_lM = key_of(a.lo_max);
+  const unsigned key_hm = key_of(a.hi_min), key_hM = key_of(a.hi_max);
+
+  unsigned long long n_neg = 0, n_pos = 0, k_bf = 0, k_fp = 0;
+  long long s_pos_bf = 0, s_neg_bf = 0, s_neg_fp = 0, s_pos_fp = 0;
+  double emax = 0.0;
+  unsigned bad = 0;
+  unsigned nb_below1 = 0, nb_above = kNone, nb_m = kNone, nb_M1 = 0;
+
+  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < a.T;
+       t += (int64_t)gridDim.x * blockDim.x) {
+    const bool valid = a.mask ? a.mask[t] != 0 : true;
+    const float A = a.adv[t];
+    const float rf = a.r_fp8[t];
+    const bool neg = valid && A < 0.f, pos = valid && A > 0.f;
+    if (stage == kPrep) {
+      const float rb = a.r_bf16[t];
+      const float c = a.coef ? a.coef[t] : 1.f;
+      if (!(isfinite(A) && isfinite(rf) && isfinite(rb) && isfinite(c)) || rf < 0.f || rb < 0.f ||
+          c < 0.f)
+        bad = 1;
+      if (neg) {
+        ++n_neg;
+        if (rb <= a.c_lo) ++k_bf;
+      }
+      if (pos) ++n_pos;
+      if (neg || pos) {
+        const double eb = (static_cast<double>(c) * rb) * static_cast<double>(A);
+        const double ef = (static_cast<double>(c) * rf) * static_cast<double>(A);
+        emax = fmax(emax, fmax(fabs(eb), fabs(ef)));
+      }
+      if (neg) {
+        if (grid_mode) {
+          atomicAdd(&sh_cnt[first_cand(a.lo_grid0, a.step, a.n_lcand, rf, false)], 1ull);
+        } else {
+          const unsigned d = digit_of(key_of(rf), 0);
+          atomicAdd(&sh_cnt[d], 1ull);
+          atomicAdd(reinterpret_cast<unsigned long long*>(&sh_w[d]), 1ull);
+        }
+      }
+      continue;
+    }
+    if (stage == kSums) {
+      if (!(neg || pos)) continue;
+      const float rb = a.r_bf16[t];
+      const float c = a.coef ? a.coef[t] : 1.f;
+      const long long qb = fixed_term(c, rb, A, shift);
+      if (pos && rb < a.c_hi) s_pos_bf += qb;
+      if (neg && rb > a.c_lo) s_neg_bf += qb;
+      if (grid_mode) {
+        const long long qf = fixed_term(c, rf, A, shift);
+        if (neg && rf > lo_star) s_neg_fp += qf;
+        if (neg && rf <= lo_star) ++k_fp;
+        if (pos) {
+          const int j = first_cand(a.hi_grid0, a.step, a.n_hcand, rf, true);
+          atomicAdd(reinterpret_cast<unsigned long long*>(&sh_w[j]),
+                    static_cast<unsigned long long>(qf));
+          atomicAdd(&sh_cnt[j], 1ull);
+        }
+      } else if (neg) {
+        const unsigned key = key_of(rf);
+        if (digit_match(key, 1, prefix)) {
+          const unsigned d = digit_of(key, 1);
+          atomicAdd(&sh_cnt[d], 1ull);
+          atomicAdd(reinterpret_cast<unsigned long long*>(&sh_w[d]), 1ull);
+        }
+      }
+      continue;
+    }
+    if (stage == kL2 || stage == kLNb) {
+      if (!neg) continue;
+      const unsigned key = key_of(rf);
+      if (stage == kL2) {
+        if (digit_match(key, 2, prefix)) {
+          const unsigned d = digit_of(key, 2);
+          atomicAdd(&sh_cnt[d], 1ull);
+          atomicAdd(reinterpret_cast<unsigned long long*>(&sh_w[d]), 1ull);
+        }
+      } else {
+        if (key < u) nb_below1 = max(nb_below1, key + 1);
+        if (key > u) nb_above = min(nb_above, key);
+        if (key > key_lm) nb_m = min(nb_m, key);
+        if (key <= key_lM) nb_M1 = max(nb_M1, key + 1);
+      }
+      continue;
+    }
+    // H stages: Pos set, weights q_fp8
+    if (stage == kH0 && neg) {
+      const float c = a.coef ? a.coef[t] : 1.f;
+      if (rf > lo_star) s_neg_fp += fixed_term(c, rf, A, shift);
+      else ++k_fp;
+    }
+    if (!pos) continue;
+    const float c = a.coef ? a.coef[t] : 1.f;
+    const long long qf = fixed_term(c, rf, A, shift);
+    const unsigned key = key_of(rf);
+    if (stage == kPFin) {
+      if (rf < hi_star) s_pos_fp += qf;
+    } else if (stage == kHNb) {
+      if (qf > 0) {
+        if (key < u) nb_below1 = max(nb_below1, key + 1);
+        if (key > u) nb_above = min(nb_above, key);
+        if (key >= key_hm) nb_m = min(nb_m, key);
+        if (key < key_hM) nb_M1 = max(nb_M1, key + 1);
+      }
+    } else if (digit_match(key, digit, prefix)) {
+      const unsigned d = digit_of(key, digit);
+      atomicAdd(&sh_cnt[d], 1ull);
+      atomicAdd(reinterpret_cast<unsigned long long*>(&sh_w[d]), static_cast<unsigned long long>(qf));
+    }
+  }
+
+  // ---- flush: warp-aggregated scalars, then the block histogram
+  const int lane = threadIdx.x & 31;
+  n_neg = warp_sum(n_neg);
+  n_pos = warp_sum(n_pos);
+  k_bf = warp_sum(k_bf);
+  k_fp = warp_sum(k_fp);
+  s_pos_bf = warp_sum(s_pos_bf);
+  s_neg_bf = warp_sum(s_neg_bf);
+  s_neg_fp = warp_sum(s_neg_fp);
+  s_pos_fp = warp_sum(s_pos_fp);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) emax = fmax(emax, __shfl_xor_sync(0xffffffffu, emax, o));
+  bad = __reduce_or_sync(0xffffffffu, bad);
+  nb_below1 = __reduce_max_sync(0xffffffffu, nb_below1);
+  nb_above = __reduce_min_sync(0xffffffffu, nb_above);
+  nb_m = __reduce_min_sync(0xffffffffu, nb_m);
+  nb_M1 = __reduce_max_sync(0xffffffffu, nb_M1);
+  if (lane == 0) {
+    if (n_neg) atomicAdd(&st->n_neg, n_neg);
+    if (n_pos) atomicAdd(&st->n_pos, n_pos);
+    if (k_bf) atomicAdd(&st->k_bf16, k_bf);
+    if (k_fp) atomicAdd(&st->k_fp8, k_fp);
+    if (s_pos_bf) atomicAdd(&st->s_pos_bf, static_cast<unsigned long long>(s_pos_bf));
+    if (s_neg_bf) atomicAdd(&st->s_neg_bf, static_cast<unsigned long long>(s_neg_bf));
+    if (s_neg_fp) atomicAdd(&st->s_neg_fp, static_cast<unsigned long long>(s_neg_fp));
+    if (s_pos_fp) atomicAdd(&st->s_pos_fp, static_cast<unsigned long long>(s_pos_fp));
+    if (emax > 0.0) atomicMax(&st->emax_bits, static_cast<unsigned long long>(__double_as_longlong(emax)));
+    if (bad) {
+      atomicOr(&st->bad, 1u);
+      flag(kErrDevice);
+    }
+    if (nb_below1) atomicMax(&st->nb_below1, nb_below1);
+    if (nb_above != kNone) atomicMin(&st->nb_above, nb_above);
+    if (nb_m != kNone) atomicMin(&st->nb_mpiece, nb_m);
+    if (nb_M1) atomicMax(&st->nb_Mpiece1, nb_M1);
+  }
+  if (want_hist) {
+    __syncthreads();
+    for (int i = threadIdx.x; i < kBuckets; i += blockDim.x) {
+      if (sh_cnt[i]) {
+        atomicAdd(&st->h_cnt[i], sh_cnt[i]);
+        atomicAdd(&st->h_w[i], static_cast<unsigned long long>(sh_w[i]));
+      }
+    }
+  }
+}
+
+// ------------------------------------------------------------------ 128-bit
+struct U128 {
+  unsigned long long hi, lo;
+};
+__device__ __forceinline__ U128 mul_u64(unsigned long long a, unsigned long long b) {
+  return U128{__umul64hi(a, b), a * b};
+}
+__device__ __forceinline__ bool ge128(U128 a, U128 b) {
+  return a.hi > b.hi || (a.hi == b.hi && a.lo >= b.lo);
+}
+__device__ __forceinline__ bool lt128(U128 a, U128 b) { return !ge128(a, b); }
+__device__ __forceinline__ U128 sub128(U128 a, U128 b) {  // a >= b
+  U128 r;
+  r.lo = a.lo - b.lo;
+  r.hi = a.hi - b.hi - (a.lo < b.lo ? 1ull : 0ull);
+  return r;
+}
+__device__ __forceinline__ U128 absdiff128(U128 a, U128 b) { return ge128(a, b) ? sub128(a, b) : sub128(b, a); }
+
+__device__ __forceinline__ float next_up(float x) { return nextafterf(x, INFINITY); }
+__device__ __forceinline__ float next_down(float x) { return nextafterf(x, -INFINITY); }
+__device__ __forceinline__ float clampf(float x, float lo, float hi) { return fminf(fmaxf(x, lo), hi); }
+
+__device__ __forceinline__ float smooth(float b_old, float b_star, float delta) {
+  if (isnan(b_old)) return b_star;
+  float d = __fmul_rn(__fsub_rn(b_star, b_old), 0.5f);
+  d = fminf(fmaxf(d, -delta), delta);
+  return __fadd_rn(b_old, d);
+}
+
+// One step of the weighted radix select, by the whole block: smallest bucket
+// b with cnt[b] > 0 and (below + sum_{b' <= b} w[b']) * D >= X.
+__device__ void select_step(State* st, int bits, bool last) {
+  __shared__ long long sh_incl[kBuckets];
+  __shared__ long long warp_tot[32];
+  __shared__ int sh_best;
+  const int nb = 1 << bits;
+  const int tid = threadIdx.x;
+  const int per = kBuckets / blockDim.x;  // 2 buckets per thread
+  long long local[2] = {0, 0};
+  long long run = 0;
+  for (int j = 0; j < per; ++j) {
+    const int b = tid * per + j;
+    run += (b < nb) ? static_cast<long long>(st->h_w[b]) : 0;
+    local[j] = run;
+  }
+  // exclusive scan of per-thread totals
+  const int lane = tid & 31, wid = tid >> 5;
+  long long v = run;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const long long n = __shfl_up_sync(0xffffffffu, v, o);
+    if (lane >= o) v += n;
+  }
+  if (lane == 31) warp_tot[wid] = v;
+  if (tid == 0) sh_best = 0x7FFFFFFF;
+  __syncthreads();
+  if (wid == 0) {
+    long long w = (lane < (int)(blockDim.x >> 5)) ? warp_tot[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const long long n = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += n;
+    }
+    warp_tot[lane] = w;  // inclusive over warps
+  }
+  __syncthreads();
+  const long long before = (v - run) + (wid > 0 ? warp_tot[wid - 1] : 0);
+  const U128 X{st->tgt_hi, st->tgt_lo};
+  const unsigned long long D = static_cast<unsigned long long>(st->dmul);
+  for (int j = 0; j < per; ++j) {
+    const int b = tid * per + j;
+    const long long incl = before + local[j];
+    sh_incl[b] = incl;
+    if (b < nb && st->h_cnt[b] > 0) {
+      const long long cum = st->below + incl;
+      if (ge128(mul_u64(static_cast<unsigned long long>(cum), D), X)) atomicMin(&sh_best, b);
+    }
+  }
+  __syncthreads();
+  if (tid == 0) {
+    const int b = sh_best;
+    if (b == 0x7FFFFFFF) {
+      st->found = 0;
+    } else {
+      const long long excl = sh_incl[b] - static_cast<long long>(st->h_w[b]);
+      st->below += excl;
+      st->prefix = (st->prefix << bits) | static_cast<unsigned>(b);
+      if (last) {
+        st->u_key = st->prefix;
+        st->p_lt = st->below;
+        st->p_le = st->below + static_cast<long long>(st->h_w[b]);
+      }
+    }
+  }
+  __syncthreads();
+  for (int i = tid; i < kBuckets; i += blockDim.x) {
+    st->h_cnt[i] = 0;
+    st->h_w[i] = 0;
+  }
+}
+
+__device__ void reset_neighbours(State* st) {
+  st->nb_below1 = 0;
+  st->nb_above = kNone;
+  st->nb_mpiece = kNone;
+  st->nb_Mpiece1 = 0;
+}
+
+// Decides stage 2's target after D_fp8 is known; false when degenerate (H* is
+// then the reference bound clamped to I_H).
+__device__ bool begin_upper(const Args& a, State* st) {
+  const long long n_bf = static_cast<long long>(st->s_pos_bf);
+  const long long d_bf = llabs(static_cast<long long>(st->s_neg_bf));
+  const long long d_fp = llabs(static_cast<long long>(st->s_neg_fp));
+  int fl = st->flags;
+  if (st->n_pos == 0) fl |= FP8RL_CALIB_FLAG_NO_POS;
+  if (d_bf == 0) fl |= FP8RL_CALIB_FLAG_ZERO_D_BF16;
+  if (d_fp == 0) fl |= FP8RL_CALIB_FLAG_ZERO_D_FP8;
+  st->flags = fl;
+  const U128 X = mul_u64(static_cast<unsigned long long>(n_bf), static_cast<unsigned long long>(d_fp));
+  st->tgt_hi = X.hi;
+  st->tgt_lo = X.lo;
+  st->dmul = d_bf;
+  st->below = 0;
+  st->prefix = 0;
+  st->found = 1;
+  const bool active =
+      !(fl & (FP8RL_CALIB_FLAG_NO_POS | FP8RL_CALIB_FLAG_ZERO_D_BF16 | FP8RL_CALIB_FLAG_ZERO_D_FP8));
+  st->h_active = active;
+  if (!active) st->hi_star = clampf(a.c_hi, a.hi_min, a.hi_max);
+  return active;
+}
+
+__device__ void write_result(const Args& a, State* st) {
+  fp8rl_calib_result r;
+  r.lo_star = st->lo_star;
+  r.hi_star = st->hi_star;
+  r.lo_new = smooth(a.lo_old, st->lo_star, a.delta_lo);
+  r.hi_new = smooth(a.hi_old, st->hi_star, a.delta_hi);
+  r.c_lo = a.c_lo;
+  r.c_hi = a.c_hi;
+  r.flags = st->flags;
+  r.shift = st->shift;
+  r.n_neg = static_cast<int64_t>(st->n_neg);
+  r.n_pos = static_cast<int64_t>(st->n_pos);
+  r.k_bf16 = static_cast<int64_t>(st->k_bf16);
+  r.k_fp8 = static_cast<int64_t>(st->k_fp8);
+  r.sum_pos_bf16 = static_cast<int64_t>(st->s_pos_bf);
+  r.sum_neg_bf16 = llabs(static_cast<long long>(st->s_neg_bf));
+  r.sum_neg_fp8 = llabs(static_cast<long long>(st->s_neg_fp));
+  r.sum_pos_fp8 = static_cast<int64_t>(st->s_pos_fp);
+  r.rho_bf16 = r.sum_neg_bf16 ? static_cast<double>(r.sum_pos_bf16) / static_cast<double>(r.sum_neg_bf16) : NAN;
+  r.rho_fp8 = r.sum_neg_fp8 ? static_cast<double>(r.sum_pos_fp8) / static_cast<double>(r.sum_neg_fp8) : NAN;
+  *a.out = r;
+}
+
+__device__ void zero_hist(State* st) {
+  for (int i = threadIdx.x; i < kBuckets; i += blockDim.x) {
+    st->h_cnt[i] = 0;
+    st->h_w[i] = 0;
+  }
+}
+
+// L* from the unconstrained minimiser interval [lo, hi] of |C(L) - k| (closed
+// in float32) and the pieces of C containing the ends of I_L.
+__device__ float lower_from_interval(const Args& a, const State* st, float lo, float hi) {
+  if (fmaxf(lo, a.lo_min) <= fminf(hi, a.lo_max))
+    return clampf(a.c_lo, fmaxf(lo, a.lo_min), fminf(hi, a.lo_max));
+  if (hi < a.lo_min) {  // f increases across I_L: the piece containing lo_min
+    const float b = st->nb_mpiece != kNone ? next_down(__uint_as_float(st->nb_mpiece)) : INFINITY;
+    return clampf(a.c_lo, a.lo_min, fminf(b, a.lo_max));
+  }
+  // f decreases across I_L: the piece containing lo_max
+  const float b = st->nb_Mpiece1 ? __uint_as_float(st->nb_Mpiece1 - 1) : -INFINITY;
+  return clampf(a.c_lo, fmaxf(b, a.lo_min), a.lo_max);
+}
+
+__device__ float upper_from_interval(const Args& a, const State* st, float lo, float hi) {
+  if (fmaxf(lo, a.hi_min) <= fminf(hi, a.hi_max))
+    return clampf(a.c_hi, fmaxf(lo, a.hi_min), fminf(hi, a.hi_max));
+  if (hi < a.hi_min) {  // the piece (z, b] containing hi_min
+    const float b = st->nb_mpiece != kNone ? __uint_as_float(st->nb_mpiece) : INFINITY;
+    return clampf(a.c_hi, a.hi_min, fminf(b, a.hi_max));
+  }
+  // the piece containing hi_max
+  const float b = st->nb_Mpiece1 ? next_up(__uint_as_float(st->nb_Mpiece1 - 1)) : -INFINITY;
+  return clampf(a.c_hi, fmaxf(b, a.hi_min), a.hi_max);
+}
+
+__global__ void __launch_bounds__(1024) decide_kernel(Args a, int stage) {
+  State* st = a.st;
+  const int tid = threadIdx.x;
+  __shared__ int sh_go;
+
+  if (stage == kPrep) {
+    if (tid == 0) {
+      // fixed-point shift s = 62 - E - B: max|e| < 2^E, 2^B >= signed tokens
+      const double emax = __longlong_as_double(static_cast<long long>(st->emax_bits));
+      const unsigned long long nt = st->n_neg + st->n_pos;
+      int s = 0;
+      if (nt > 0 && emax > 0.0) {
+        int E;
+        frexp(emax, &E);
+        const int B = nt > 1 ? 64 - __clzll(static_cast<long long>(nt - 1)) : 0;
+        s = 62 - E - B;
+      }
+      st->shift = s;
+      st->flags = 0;
+      if (st->n_neg == 0) {
+        st->flags |= FP8RL_CALIB_FLAG_NO_NEG;
+        st->lo_star = clampf(a.c_lo, a.lo_min, a.lo_max);
+      }
+      st->tgt_hi = 0;
+      st->tgt_lo = st->k_bf16;
+      st->dmul = 1;
+      st->below = 0;
+      st->prefix = 0;
+      st->found = 1;
+      sh_go = st->n_neg > 0;
+      if (a.grid_mode && st->n_neg > 0) {
+        // cnt_le(L_i) is the prefix sum of the candidate histogram; minimise
+        // (|cnt - k|, |L_i - c_lo|, L_i) over the <= 2047 candidates
+        const long long k = static_cast<long long>(st->k_bf16);
+        long long cum = 0, best_f = -1;
+        double best_d = 0;
+        float best = 0;
+        for (int i = 0; i < a.n_lcand; ++i) {
+          cum += static_cast<long long>(st->h_cnt[i]);
+          const long long f = llabs(cum - k);
+          const float L = cand_at(a.lo_grid0, a.step, i);
+          const double d = fabs(static_cast<double>(L) - static_cast<double>(a.c_lo));
+          if (best_f < 0 || f < best_f || (f == best_f && (d < best_d || (d == best_d && L < best)))) {
+            best_f = f;
+            best_d = d;
+            best = L;
+          }
+        }
+        st->lo_star = best;
+      }
+    }
+    __syncthreads();
+    if (a.grid_mode) zero_hist(st);
+    else if (sh_go) select_step(st, 11, false);
+    return;
+  }
+
+  if (stage == kSums) {
+    if (!a.grid_mode) {
+      if (st->n_neg > 0) select_step(st, 11, false);
+      return;
+    }
+    if (tid == 0 && begin_upper(a, st)) {
+      const U128 X{st->tgt_hi, st->tgt_lo};
+      const unsigned long long D = static_cast<unsigned long long>(st->dmul);
+      long long cum = 0;
+      U128 best_f{0, 0};
+      double best_d = 0;
+      float best = 0;
+      bool have = false;
+      for (int j = 0; j < a.n_hcand; ++j) {
+        cum += static_cast<long long>(st->h_w[j]);
+        const U128 f = absdiff128(mul_u64(static_cast<unsigned long long>(cum), D), X);
+        const float H = cand_at(a.hi_grid0, a.step, j);
+        const double d = fabs(static_cast<double>(H) - static_cast<double>(a.c_hi));
+        const bool better = !have || lt128(f, best_f) ||
+                            (!lt128(best_f, f) && (d < best_d || (d == best_d && H < best)));
+        if (better) {
+          best_f = f;
+          best_d = d;
+          best = H;
+          have = true;
+        }
+      }
+      st->hi_star = best;
+    }
+    return;
+  }
+
+  if (stage == kL2) {
+    if (st->n_neg > 0) select_step(st, 10, true);
+    if (tid == 0) reset_neighbours(st);
+    return;
+  }
+
+  if (stage == kLNb) {
+    if (tid == 0) {
+      if (st->n_neg > 0) {
+        // minimisers of |C(L) - k|, C(L) = #{A<0 : r_fp8 <= L}, around u = r_(k)
+        const long long k = static_cast<long long>(st->k_bf16);
+        const float fu = __uint_as_float(st->u_key);
+        const long long w_above = st->p_le - k, w_below = k - st->p_lt;
+        const float z = st->nb_below1 ? __uint_as_float(st->nb_below1 - 1) : -INFINITY;
+        const float w = st->nb_above != kNone ? __uint_as_float(st->nb_above) : INFINITY;
+        float lo, hi;
+        if (w_above < w_below) {
+          lo = fu;
+          hi = next_down(w);
+        } else if (w_below < w_above) {
+          lo = z;
+          hi = next_down(fu);
+        } else {
+          lo = z;
+          hi = next_down(w);
+        }
+        st->lo_star = lower_from_interval(a, st, lo, hi);
+      }
+      st->k_fp8 = 0;
+      st->s_neg_fp = 0;
+      st->below = 0;
+      st->prefix = 0;
+    }
+    __syncthreads();
+    zero_hist(st);
+    return;
+  }
+
+  if (stage == kH0) {
+    if (tid == 0) sh_go = begin_upper(a, st);
+    __syncthreads();
+    if (sh_go) select_step(st, 11, false);
+    return;
+  }
+
+  if (stage == kH1 || stage == kH2) {
+    if (tid == 0) sh_go = st->h_active && st->found;
+    __syncthreads();
+    if (sh_go) select_step(st, stage == kH1 ? 11 : 10, stage == kH2);
+    if (stage == kH2 && tid == 0) {
+      if (!st->found) st->u_key = kNone;
+      reset_neighbours(st);
+    }
+    return;
+  }
+
+  if (stage == kHNb) {
+    if (tid == 0 && st->h_active) {
+      // minimisers of |P(H) D - X|, P(H) = sum_{A>0, r_fp8 < H} q, as a closed
+      // float interval of H, from u and its positive-weight neighbours
+      const U128 X{st->tgt_hi, st->tgt_lo};
+      const unsigned long long D = static_cast<unsigned long long>(st->dmul);
+      const float z = st->nb_below1 ? __uint_as_float(st->nb_below1 - 1) : -INFINITY;
+      const float w = st->nb_above != kNone ? __uint_as_float(st->nb_above) : INFINITY;
+      float lo, hi;
+      if (!st->found) {  // even all of P stays below the target
+        lo = next_up(z);
+        hi = INFINITY;
+      } else {
+        const float fu = __uint_as_float(st->u_key);
+        const U128 above = sub128(mul_u64(static_cast<unsigned long long>(st->p_le), D), X);
+        const U128 below = sub128(X, mul_u64(static_cast<unsigned long long>(st->p_lt), D));
+        if (lt128(above, below)) {
+          lo = next_up(fu);
+          hi = w;
+        } else if (lt128(below, above)) {
+          lo = next_up(z);
+          hi = fu;
+        } else {
+          lo = next_up(z);
+          hi = w;
+        }
+      }
+      st->hi_star = upper_from_interval(a, st, lo, hi);
+    }
+    return;
+  }
+
+  if (stage == kPFin) {
+    if (tid == 0) write_result(a, st);
+  }
+}
+
+}  // namespace
+
+size_t calib_workspace_bytes(int64_t) { return align_up(sizeof(State), 256); }
+
+cudaError_t launch_calibrate(const float* r_fp8, const float* r_bf16, const float* adv,
+                             const uint8_t* mask, const float* coef, int64_t T, float eps_low,
+                             float eps_high, const fp8rl_calib_opts& o, fp8rl_calib_result* result,
+                             void* ws, cudaStream_t s) {
+  Args a{};
+  a.r_fp8 = r_fp8;
+  a.r_bf16 = r_bf16;
+  a.adv = adv;
+  a.mask = mask;
+  a.coef = coef;
+  a.T = T;
+  a.c_lo = 1.0f - eps_low;
+  a.c_hi = 1.0f + eps_high;
+  a.lo_min = static_cast<float>(o.lo_min);
+  a.lo_max = static_cast<float>(o.lo_max);
+  a.hi_min = static_cast<float>(o.hi_min);
+  a.hi_max = static_cast<float>(o.hi_max);
+  a.delta_lo = static_cast<float>(o.delta_lo);
+  a.delta_hi = static_cast<float>(o.delta_hi);
+  a.lo_old = o.lo_old;
+  a.hi_old = o.hi_old;
+  a.grid_mode = o.mode == FP8RL_CALIB_GRID;
+  a.lo_grid0 = o.lo_min;
+  a.hi_grid0 = o.hi_min;
+  a.step = o.step;
+  a.n_lcand = a.grid_mode ? static_cast<int>(std::llround((o.lo_max - o.lo_min) / o.step)) + 1 : 0;
+  a.n_hcand = a.grid_mode ? static_cast<int>(std::llround((o.hi_max - o.hi_min) / o.step)) + 1 : 0;
+  a.st = static_cast<State*>(ws);
+  a.out = result;
+
+  cudaError_t e = cudaMemsetAsync(ws, 0, sizeof(State), s);
+  if (e != cudaSuccess) return e;
+  int64_t want = (T + 1023) / 1024;
+  const int64_t cap = static_cast<int64_t>(sm_count()) * 4;
+  const int grid = static_cast<int>(want < 1 ? 1 : (want > cap ? cap : want));
+  const int stages_exact[] = {kPrep, kSums, kL2, kLNb, kH0, kH1, kH2, kHNb, kPFin};
+  const int stages_grid[] = {kPrep, kSums, kPFin};
+  const int* stages = a.grid_mode ? stages_grid : stages_exact;
+  const int n = a.grid_mode ? 3 : 9;
+  for (int i = 0; i < n; ++i) {
+    pass_kernel<<<grid, 256, 0, s>>>(a, stages[i]);
+    decide_kernel<<<1, 1024, 0, s>>>(a, stages[i]);
+  }
+  return cudaGetLastError();
+}
+
+uint32_t calib_status_take() {
+  uint32_t v = 0, z = 0;
+  if (cudaMemcpyFromSymbol(&v, d_status, sizeof(v)) != cudaSuccess) return 0;
+  cudaMemcpyToSymbol(d_status, &z, sizeof(z));
+  return v;
+}
+
+}  // namespace fp8rl

@@ -1,0 +1,604 @@
+// a3: FP8 lm_head GEMM on the tcgen05 tensor cores with a streaming
+// logsumexp + target-gather epilogue; a4: merge of the per-chunk partials into
+// log-probs and importance ratios (§2.1 ratio, Eq. 3 scaling).
+//
+// z[t][v] = sum_k S_h S_W q_h[t][k] q_W[v][k] is never stored.  Each CTA owns
+// persistent 128 (tokens) x 256 (vocab) output tiles:
+//   warp 0      TMA producer: 128x128 A tile + 256x128 B tile per stage, 128B
+//               swizzle, 4-stage shared-memory ring guarded by mbarriers;
+//   warp 1      MMA issuer: tcgen05.mma kind::f8f6f4 M=128 N=256 K=32, fp32
+//               accumulator in TMEM (two 256-column buffers);
+//   warps 2..9  epilogue: tcgen05.ld of the accumulator, one thread per token
+//               row and 128-column half, scales applied, then the running
+//               (max, sum exp) of its 128 columns and z[t][y_t] if y_t falls in
+//               them.  One (max, sum) pair per token and 128-wide vocabulary
+//               chunk goes to the workspace; nothing of size T x V does.
+// Per-tensor and per-row scales factor out of the K sum, so the accumulator
+// runs over the whole K in TMEM and is scaled once.  Block scales (1x128 for h,
+// 128x128 for W) change every 128-wide K block: the MMA writes each K block's
+// partial product into one of the two TMEM buffers and the epilogue promotes
+// it, acc += S_h[t][kb] S_W[vb][kb] * partial, into registers while the MMA
+// fills the other buffer.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <cmath>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace fp8rl {
+namespace {
+
+__device__ uint32_t d_status;
+
+constexpr int BM = 128;           // tokens per tile (TMEM lanes)
+constexpr int BN = 256;           // vocabulary columns per tile (MMA N)
+constexpr int BK = 128;           // K bytes per stage (one 128B swizzle row)
+constexpr int CHUNK = 128;        // vocabulary columns per LSE partial
+constexpr int STAGES = 4;
+constexpr int EPI_WARPS = 8;
+constexpr int THREADS = 64 + EPI_WARPS * 32;
+constexpr uint32_t A_BYTES = BM * BK;
+constexpr uint32_t B_BYTES = BN * BK;
+constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr uint32_t TMEM_COLS = 2 * BN;
+constexpr size_t SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr uint64_t kDrainNs = 1000000000ull;
+
+enum { kTensor = FP8RL_GRAN_TENSOR, kRow = FP8RL_GRAN_ROWWISE, kBlock = FP8RL_GRAN_BLOCK };
+enum { kEpiLse = 0, kEpiDlogits = 1 };
+
+struct Params {
+  const float* a_scales;
+  const float* b_scales;
+  const int32_t* targets;
+  float2* partials;
+  float* zy;
+  const float* lse;
+  const float* grad;
+  float* out;
+  int M, N, K;
+  int num_m, num_n, num_kb;
+  int n_chunks;
+  uint64_t wait_limit_ns;
+};
+
+__device__ __forceinline__ void flag(uint32_t bits) { atomicOr(&d_status, bits); }
+
+// Running epilogue state of one thread: row `row`, vocabulary columns
+// [col0, col0 + 128) consumed 32 at a time (values already scaled).
+struct EpiState {
+  float m, s, zy;
+  int j;  // target column relative to col0 (outside [0, 128): not here)
+};
+
+template <int EPI>
+__device__ __forceinline__ void epi_begin(const Params& p, EpiState& e, int row, int col0) {
+  e.m = -INFINITY;
+  e.s = 0.f;
+  e.zy = 0.f;
+  e.j = -1;
+  if (row < p.M) {
+    const int y = p.targets[row];
+    if (y >= 0 && y < p.N) e.j = y - col0;
+  }
+}
+
+// Columns [col0 + base, col0 + base + 32).
+template <int EPI>
+__device__ __forceinline__ void epi_consume32(const Params& p, EpiState& e, const float* z, int row,
+                                              int col0, int base) {
+  const int ncol = p.N - (col0 + base);  // valid columns in this piece (may be <= 0 or >= 32)
+  if (ncol <= 0 || row >= p.M) return;
+  if (EPI == kEpiLse) {
+    float cm = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      if (i < ncol) cm = fmaxf(cm, z[i]);
+    const float mn = fmaxf(e.m, cm);
+    const float mb = mn * kLog2e;
+    float acc = 0.f;
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      if (i < ncol) acc += exp2f(fmaf(z[i], kLog2e, -mb));
+    e.s = e.s * exp2f((e.m - mn) * kLog2e) + acc;
+    e.m = mn;
+    const int jj = e.j - base;
+    if (jj >= 0 && jj < 32) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        if (i == jj) e.zy = z[i];
+    }
+  } else {
+    const float l = p.lse[row], g = p.grad[row];
+    float* o = p.out + static_cast<size_t>(row) * p.N + col0 + base;
+    const int jj = e.j - base;
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      if (i < ncol) o[i] = g * ((i == jj ? 1.f : 0.f) - expf(z[i] - l));
+  }
+}
+
+template <int EPI>
+__device__ __forceinline__ void epi_finish(const Params& p, const EpiState& e, int row, int chunk) {
+  if (EPI != kEpiLse || row >= p.M || chunk >= p.n_chunks) return;
+  p.partials[static_cast<size_t>(chunk) * p.M + row] = make_float2(e.m, e.s);
+  if (e.j >= 0 && e.j < CHUNK) p.zy[row] = e.zy;
+}
+
+template <int MODE, int EPI>
+__global__ void __launch_bounds__(THREADS, 1)
+    fp8_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                    const Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* smA = smem;
+  uint8_t* smB = smem + STAGES * A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smB + STAGES * B_BYTES);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + STAGES;
+  uint64_t* acc_full = bars + 2 * STAGES;
+  uint64_t* acc_empty = acc_full + 2;
+  uint64_t* done = acc_empty + 2;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(done + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(smem_u32(&acc_full[b]), 1);
+      mbar_init(smem_u32(&acc_empty[b]), EPI_WARPS);
+    }
+    mbar_init(smem_u32(done), 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_holder), TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+  const int total = p.num_m * p.num_n;
+  const uint64_t lim = p.wait_limit_ns;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t armed = 0, armed_phase = 0;  // bit s: stage s loaded / its parity
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+        const int m0 = (tile % p.num_m) * BM, n0 = (tile / p.num_m) * BN;
+        for (int kb = 0; kb < p.num_kb; ++kb) {
+          if (!mbar_wait(smem_u32(&empty[stage]), phase ^ 1, lim, abort_flag)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(smem_u32(&full[stage]), STAGE_BYTES);
+          tma_load_2d(smem_u32(smA + stage * A_BYTES), &tmA, smem_u32(&full[stage]), kb * BK, m0);
+          tma_load_2d(smem_u32(smB + stage * B_BYTES), &tmB, smem_u32(&full[stage]), kb * BK, n0);
+          armed |= 1u << stage;
+          armed_phase = (armed_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        flag(kErrTimeout);
+      }
+      // no copy may still be in flight when the CTA exits
+      for (int s = 0; s < STAGES; ++s)
+        if (armed & (1u << s)) mbar_wait(smem_u32(&full[s]), (armed_phase >> s) & 1, kDrainNs, nullptr);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      int stage = 0, ab = 0;
+      uint32_t phase = 0, aphase = 0;
+      constexpr uint32_t idesc = idesc_e4m3_f32(BM, BN);
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+        if (MODE != kBlock) {
+          if (!mbar_wait(smem_u32(&acc_empty[ab]), aphase ^ 1, lim, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+        }
+        for (int kb = 0; kb < p.num_kb; ++kb) {
+          if (!mbar_wait(smem_u32(&full[stage]), phase, lim, abort_flag)) {
+            ok = false;
+            break;
+          }
+          if (MODE == kBlock) {
+            if (!mbar_wait(smem_u32(&acc_empty[ab]), aphase ^ 1, lim, abort_flag)) {
+              ok = false;
+              break;
+            }
+          }
+          tc_fence_after();
+          const uint32_t d = tmem_base + static_cast<uint32_t>(ab * BN);
+          const uint64_t adesc = smem_desc_sw128(smem_u32(smA + stage * A_BYTES));
+          const uint64_t bdesc = smem_desc_sw128(smem_u32(smB + stage * B_BYTES));
+#pragma unroll
+          for (int k = 0; k < BK / 32; ++k) {
+            const uint32_t acc = (MODE == kBlock) ? (k > 0) : (kb > 0 || k > 0);
+            // +32 bytes along K inside the swizzled 128-byte row
+            mma_f8f6f4(d, adesc + 2 * k, bdesc + 2 * k, idesc, acc);
+          }
+          mma_commit(smem_u32(&empty[stage]));
+          if (MODE == kBlock) {
+            mma_commit(smem_u32(&acc_full[ab]));
+            ab ^= 1;
+            if (ab == 0) aphase ^= 1;
+          }
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (!ok) break;
+        if (MODE != kBlock) {
+          mma_commit(smem_u32(&acc_full[ab]));
+          ab ^= 1;
+          if (ab == 0) aphase ^= 1;
+        }
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        flag(kErrTimeout);
+      }
+      // every MMA issued above has completed once this commit lands
+      mma_commit(smem_u32(done));
+      mbar_wait(smem_u32(done), 0, kDrainNs, nullptr);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int ew = warp - 2;
+    const int quarter = warp & 3;  // TMEM lanes this warp may access
+    const int half = ew >> 2;      // which 128 columns of the 256-wide tile
+    const int rit = quarter * 32 + lane;
+    const uint32_t t_row = static_cast<uint32_t>(quarter * 32) << 16;
+    int ab = 0;
+    uint32_t aphase = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+      const int m_blk = tile % p.num_m, n_blk = tile / p.num_m;
+      const int row = m_blk * BM + rit;
+      const bool row_ok = row < p.M;
+      const int col0 = n_blk * BN + half * CHUNK;
+      const int chunk = n_blk * 2 + half;
+      EpiState es;
+      epi_begin<EPI>(p, es, row, col0);
+      if (MODE == kBlock) {
+        float z[CHUNK];
+#pragma unroll
+        for (int i = 0; i < CHUNK; ++i) z[i] = 0.f;
+        const bool wb_ok = chunk < p.n_chunks;
+        const float* sa_ptr = p.a_scales + row;                                    // [kb][M]
+        const float* sb_ptr = p.b_scales + static_cast<size_t>(chunk) * p.num_kb;  // [vb][kb]
+        float sa = row_ok ? __ldg(sa_ptr) : 0.f;
+        float sb = wb_ok ? __ldg(sb_ptr) : 0.f;
+        for (int kb = 0; kb < p.num_kb; ++kb) {
+          const float sc = sa * sb;
+          if (kb + 1 < p.num_kb) {
+            sa = row_ok ? __ldg(sa_ptr + static_cast<size_t>(kb + 1) * p.M) : 0.f;
+            sb = wb_ok ? __ldg(sb_ptr + kb + 1) : 0.f;
+          }
+          ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&acc_full[ab]), aphase, lim, abort_flag));
+          if (!ok) break;
+          tc_fence_after();
+          const uint32_t taddr = tmem_base + t_row + static_cast<uint32_t>(ab * BN + half * CHUNK);
+#pragma unroll
+          for (int c = 0; c < CHUNK / 32; ++c) {
+            float v[32];
+            tmem_ld_32x32b_x32(taddr + c * 32, v);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) z[c * 32 + i] = fmaf(v[i], sc, z[c * 32 + i]);
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&acc_empty[ab]));
+          ab ^= 1;
+          if (ab == 0) aphase ^= 1;
+        }
+        if (!ok) break;
+#pragma unroll
+        for (int c = 0; c < CHUNK / 32; ++c) epi_consume32<EPI>(p, es, z + c * 32, row, col0, c * 32);
+      } else {
+        ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&acc_full[ab]), aphase, lim, abort_flag));
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t taddr = tmem_base + t_row + static_cast<uint32_t>(ab * BN + half * CHUNK);
+        const float sa = (MODE == kTensor) ? __ldg(p.a_scales) : (row_ok ? __ldg(p.a_scales + row) : 0.f);
+        const float s0 = (MODE == kTensor) ? sa * __ldg(p.b_scales) : 0.f;
+#pragma unroll 1
+        for (int c = 0; c < CHUNK / 32; ++c) {
+          float v[32];
+          tmem_ld_32x32b_x32(taddr + c * 32, v);
+          if (MODE == kRow) {
+            // lane i fetches the scale of column i of this piece; broadcast by shuffle
+            const int colq = col0 + c * 32 + lane;
+            const float sbl = colq < p.N ? __ldg(p.b_scales + colq) : 0.f;
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] *= sa * __shfl_sync(0xffffffffu, sbl, i);
+          } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] *= s0;
+          }
+          epi_consume32<EPI>(p, es, v, row, col0, c * 32);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&acc_empty[ab]));
+        ab ^= 1;
+        if (ab == 0) aphase ^= 1;
+      }
+      epi_finish<EPI>(p, es, row, chunk);
+    }
+    if (!ok) {
+      *abort_flag = 1;
+      flag(kErrTimeout);
+    }
+    tc_fence_before();
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, TMEM_COLS);
+  }
+}
+
+// ------------------------------------------------------------------ combine
+__global__ void combine_kernel(const float2* __restrict__ partials, const float* __restrict__ zy,
+                               const int32_t* __restrict__ targets,
+                               const float* __restrict__ logp_old, float* __restrict__ logp,
+                               float* __restrict__ lse_out, float* __restrict__ ratio, int64_t M,
+                               int64_t N, int64_t n_chunks) {
+  const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (t >= M) return;
+  float m = -INFINITY, s = 0.f;
+  int64_t c = 0;
+  for (; c + 4 <= n_chunks; c += 4) {
+    float2 q[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) q[u] = __ldg(partials + (c + u) * M + t);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (q[u].x > m) {
+        s = s * exp2f((m - q[u].x) * kLog2e) + q[u].y;
+        m = q[u].x;
+      } else {
+        s += q[u].y * exp2f((q[u].x - m) * kLog2e);
+      }
+    }
+  }
+  for (; c < n_chunks; ++c) {
+    const float2 q = __ldg(partials + c * M + t);
+    if (q.x > m) {
+      s = s * exp2f((m - q.x) * kLog2e) + q.y;
+      m = q.x;
+    } else {
+      s += q.y * exp2f((q.x - m) * kLog2e);
+    }
+  }
+  const float l = m + logf(s);
+  const int32_t y = targets[t];
+  float lp;
+  if (y >= 0 && y < N) {
+    lp = zy[t] - l;
+  } else {
+    lp = NAN;
+    flag(kErrDevice);
+  }
+  logp[t] = lp;
+  if (lse_out) lse_out[t] = l;
+  if (ratio) ratio[t] = expf(lp - logp_old[t]);
+}
+
+__global__ void ratios_kernel(const float* __restrict__ a, const float* __restrict__ b, int64_t T,
+                              float* __restrict__ r) {
+  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < T;
+       t += (int64_t)gridDim.x * blockDim.x)
+    r[t] = expf(a[t] - b[t]);
+}
+
+// Rows selected for dense dlogits are gathered (codes, scales, targets, lse,
+// grad) into a contiguous operand for the same GEMM kernel.
+__global__ void gather_rows_kernel(const uint8_t* __restrict__ h_codes,
+                                   const float* __restrict__ h_scales, int gran, int64_t T,
+                                   int64_t H, const int32_t* __restrict__ targets,
+                                   const float* __restrict__ lse, const float* __restrict__ grad,
+                                   const int64_t* __restrict__ rows, int64_t n_rows,
+                                   uint8_t* __restrict__ g_codes, float* __restrict__ g_scales,
+                                   int32_t* __restrict__ g_targets, float* __restrict__ g_lse,
+                                   float* __restrict__ g_grad) {
+  const int64_t i = blockIdx.x;
+  if (i >= n_rows) return;
+  int64_t t = rows[i];
+  const bool ok = t >= 0 && t < T;
+  if (!ok) {
+    if (threadIdx.x == 0) flag(kErrDevice);
+    t = 0;
+  }
+  const uint4* src = reinterpret_cast<const uint4*>(h_codes + t * H);
+  uint4* dst = reinterpret_cast<uint4*>(g_codes + i * H);
+  for (int64_t v = threadIdx.x; v < H / 16; v += blockDim.x) dst[v] = ok ? src[v] : make_uint4(0, 0, 0, 0);
+  if (threadIdx.x == 0) {
+    g_targets[i] = targets[t];
+    g_lse[i] = lse[t];
+    g_grad[i] = ok ? grad[t] : NAN;
+    if (gran == kTensor) {
+      if (i == 0) g_scales[0] = h_scales[0];
+    } else if (gran == kRow) {
+      g_scales[i] = h_scales[t];
+    }
+  }
+  if (gran == kBlock) {
+    const int64_t nkb = H / 128;
+    for (int64_t kb = threadIdx.x; kb < nkb; kb += blockDim.x) g_scales[kb * n_rows + i] = h_scales[kb * T + t];
+  }
+}
+
+__global__ void wait_selftest_kernel(uint64_t limit_ns) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(smem_u32(&bar), 1);
+    fence_mbar_init();
+    // nothing ever arrives on this barrier: the wait must expire
+    if (!mbar_wait(smem_u32(&bar), 0, limit_ns, nullptr)) flag(kErrTimeout);
+  }
+}
+
+// ------------------------------------------------------------------ host side
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (fn == nullptr) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  }
+  return fn;
+}
+
+// K-major uint8 matrix [rows][K], box (128 K) x box_rows, 128B swizzle, zero
+// fill outside the matrix.
+bool make_tmap(CUtensorMap* tm, const uint8_t* base, int64_t rows, int64_t K, uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (fn == nullptr) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(K)};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(tm, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t*>(base), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+template <int MODE, int EPI>
+cudaError_t launch_mode(const CUtensorMap& ta, const CUtensorMap& tb, const Params& p, int grid,
+                        cudaStream_t s) {
+  auto kern = fp8_gemm_kernel<MODE, EPI>;
+  static int configured_device = -1;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (configured_device != dev) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(SMEM_BYTES));
+    if (e != cudaSuccess) return e;
+    configured_device = dev;
+  }
+  kern<<<grid, THREADS, SMEM_BYTES, s>>>(ta, tb, p);
+  return cudaGetLastError();
+}
+
+template <int EPI>
+cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s) {
+  if (a.M == 0 || a.N == 0) return cudaSuccess;
+  CUtensorMap ta, tb;
+  if (!make_tmap(&ta, a.a_codes, a.M, a.K, BM) || !make_tmap(&tb, a.b_codes, a.N, a.K, BN))
+    return cudaErrorInvalidValue;
+  Params p{};
+  p.a_scales = a.a_scales;
+  p.b_scales = a.b_scales;
+  p.targets = a.targets;
+  p.partials = a.partials;
+  p.zy = a.zy;
+  p.lse = a.lse;
+  p.grad = a.grad;
+  p.out = a.out;
+  p.M = static_cast<int>(a.M);
+  p.N = static_cast<int>(a.N);
+  p.K = static_cast<int>(a.K);
+  p.num_m = static_cast<int>((a.M + BM - 1) / BM);
+  p.num_n = static_cast<int>((a.N + BN - 1) / BN);
+  p.num_kb = static_cast<int>((a.K + BK - 1) / BK);
+  p.n_chunks = static_cast<int>((a.N + CHUNK - 1) / CHUNK);
+  p.wait_limit_ns = wait_limit_ns();
+  const int64_t tiles = static_cast<int64_t>(p.num_m) * p.num_n;
+  const int grid = static_cast<int>(tiles < sm_count() ? tiles : sm_count());
+  switch (a.gran) {
+    case kTensor: return launch_mode<kTensor, EPI>(ta, tb, p, grid, s);
+    case kRow: return launch_mode<kRow, EPI>(ta, tb, p, grid, s);
+    default: return launch_mode<kBlock, EPI>(ta, tb, p, grid, s);
+  }
+}
+
+int blocks_for(int64_t n, int threads) {
+  int64_t b = (n + threads - 1) / threads;
+  return static_cast<int>(b < 1 ? 1 : b);
+}
+
+}  // namespace
+
+cudaError_t launch_gemm_lse(const GemmArgs& a, cudaStream_t s) { return launch_gemm<kEpiLse>(a, s); }
+
+cudaError_t launch_gemm_dlogits(const GemmArgs& a, cudaStream_t s) {
+  return launch_gemm<kEpiDlogits>(a, s);
+}
+
+cudaError_t launch_combine(const float2* partials, const float* zy, const int32_t* targets,
+                           const float* logp_old, float* logp, float* lse, float* ratio,
+                           int64_t M, int64_t N, cudaStream_t s) {
+  if (M == 0) return cudaSuccess;
+  combine_kernel<<<blocks_for(M, 256), 256, 0, s>>>(partials, zy, targets, logp_old, logp, lse,
+                                                    ratio, M, N, (N + CHUNK - 1) / CHUNK);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_ratios(const float* lp_new, const float* lp_old, int64_t T, float* r,
+                          cudaStream_t s) {
+  if (T == 0) return cudaSuccess;
+  int b = blocks_for(T, 256);
+  if (b > sm_count() * 8) b = sm_count() * 8;
+  ratios_kernel<<<b, 256, 0, s>>>(lp_new, lp_old, T, r);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather_rows(const uint8_t* h_codes, const float* h_scales, int gran, int64_t T,
+                               int64_t H, const int32_t* targets, const float* lse,
+                               const float* grad, const int64_t* rows, int64_t n_rows,
+                               uint8_t* g_codes, float* g_scales, int32_t* g_targets,
+                               float* g_lse, float* g_grad, cudaStream_t s) {
+  if (n_rows == 0) return cudaSuccess;
+  gather_rows_kernel<<<static_cast<unsigned>(n_rows), 128, 0, s>>>(
+      h_codes, h_scales, gran, T, H, targets, lse, grad, rows, n_rows, g_codes, g_scales,
+      g_targets, g_lse, g_grad);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_wait_selftest(uint64_t limit_ns, cudaStream_t s) {
+  wait_selftest_kernel<<<1, 32, 0, s>>>(limit_ns);
+  return cudaGetLastError();
+}
+
+uint32_t gemm_status_take() {
+  uint32_t v = 0, z = 0;
+  if (cudaMemcpyFromSymbol(&v, d_status, sizeof(v)) != cudaSuccess) return 0;
+  cudaMemcpyToSymbol(d_status, &z, sizeof(z));
+  return v;
+}
+
+}  // namespace fp8rl

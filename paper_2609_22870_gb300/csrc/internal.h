@@ -1,0 +1,74 @@
+// Host-side interface between the C ABI (api.cu) and the kernel translation
+// units.  Nothing here is exported from libfp8rl.so.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "fp8rl.h"
+
+namespace fp8rl {
+
+// Bounded-wait limit for every in-kernel spin-wait (nanoseconds of GPU time).
+uint64_t wait_limit_ns();
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// ------------------------------------------------------------- quantize.cu
+cudaError_t launch_quantize(const void* x, int64_t rows, int64_t cols, int64_t ld, int gran,
+                            int role, uint8_t* codes, float* scales, void* ws, cudaStream_t s);
+uint32_t quantize_status_take();
+
+// ----------------------------------------------------------------- gemm.cu
+struct GemmArgs {
+  const uint8_t* a_codes;   // [M][K]
+  const float* a_scales;
+  const uint8_t* b_codes;   // [N][K]
+  const float* b_scales;
+  int gran;
+  int64_t M, N, K;
+  const int32_t* targets;   // [M]
+  // LSE epilogue outputs (workspace)
+  float2* partials;         // [ceil(N/128)][M]
+  float* zy;                // [M]
+  // dlogits epilogue
+  const float* lse;         // [M]
+  const float* grad;        // [M]
+  float* out;               // [M][N]
+};
+cudaError_t launch_gemm_lse(const GemmArgs& a, cudaStream_t s);
+cudaError_t launch_gemm_dlogits(const GemmArgs& a, cudaStream_t s);
+cudaError_t launch_combine(const float2* partials, const float* zy, const int32_t* targets,
+                           const float* logp_old, float* logp, float* lse, float* ratio,
+                           int64_t M, int64_t N, cudaStream_t s);
+cudaError_t launch_ratios(const float* lp_new, const float* lp_old, int64_t T, float* r,
+                          cudaStream_t s);
+cudaError_t launch_gather_rows(const uint8_t* h_codes, const float* h_scales, int gran,
+                               int64_t T, int64_t H, const int32_t* targets, const float* lse,
+                               const float* grad, const int64_t* rows, int64_t n_rows,
+                               uint8_t* g_codes, float* g_scales, int32_t* g_targets,
+                               float* g_lse, float* g_grad, cudaStream_t s);
+cudaError_t launch_wait_selftest(uint64_t limit_ns, cudaStream_t s);
+uint32_t gemm_status_take();
+
+// ---------------------------------------------------------------- calib.cu
+size_t calib_workspace_bytes(int64_t T);
+cudaError_t launch_calibrate(const float* r_fp8, const float* r_bf16, const float* adv,
+                             const uint8_t* mask, const float* coef, int64_t T, float eps_low,
+                             float eps_high, const fp8rl_calib_opts& opts,
+                             fp8rl_calib_result* result, void* ws, cudaStream_t s);
+uint32_t calib_status_take();
+
+// ----------------------------------------------------------------- loss.cu
+size_t surrogate_workspace_bytes(int64_t T);
+cudaError_t launch_surrogate(const float* r, const float* adv, const uint8_t* mask,
+                             const float* w, int64_t T, float lo, float hi, const float* bounds,
+                             float* grad, uint8_t* clip_mask, fp8rl_clip_stats* stats, void* ws,
+                             cudaStream_t s);
+uint32_t loss_status_take();
+
+// SM count of the current device (cached per device).
+int sm_count();
+
+}  // namespace fp8rl

@@ -18,5 +18,7 @@ def cuda_lib():
     import torch
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
+    from paper_2609_22870_gb300 import _build
+    _build.build()
     from paper_2609_22870_gb300 import api
     return api

@@ -1,0 +1,134 @@
+"""GPU parity: Calibrated Clipping (a5) bit-exact against the oracle.
+
+Both sides select on the same seeded synthetic ratios.  L*, H*, the smoothed
+bounds, the counts, the fixed-point shift and every exact sum must match to
+the bit; rho is compared to float64 rounding.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import calibrate as OC
+from paper_2609_22870_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+
+def _inputs(T, seed, sigma_fp8=0.05, tie_every=0, zero_adv=0.1, mask_p=0.9, coef_scale=None):
+    r_bf, r_fp, coef = synth.ratio_inputs(T, seed, sigma_fp8=sigma_fp8, tie_every=tie_every)
+    g = torch.Generator().manual_seed(seed + 99)
+    adv = torch.randn(T, generator=g)
+    adv[torch.rand(T, generator=g) < zero_adv] = 0
+    mask = (torch.rand(T, generator=g) < mask_p).to(torch.uint8)
+    if coef_scale is not None:
+        coef = coef / coef.max() * coef_scale
+    return r_fp.float(), r_bf.float(), adv.float(), mask, coef.float()
+
+
+def _run(api, r_fp, r_bf, adv, mask, coef, eps_low, eps_high, **opts):
+    d = [None if t is None else t.cuda() for t in (r_fp, r_bf, adv, mask, coef)]
+    buf = api.calibrate_clip_bounds(*d, eps_low, eps_high, api.calib_opts(**opts) if opts else None)
+    api.check()
+    return api.read_calib_result(buf)
+
+
+def _ref(r_fp, r_bf, adv, mask, coef, eps_low, eps_high, **opts):
+    n = lambda t: None if t is None else t.numpy()  # noqa: E731
+    return OC.calibrate_clip_bounds(n(r_fp), n(r_bf), n(adv), n(mask), n(coef), eps_low, eps_high, opts)
+
+
+def _compare(got, ref):
+    for k in ("lo_star", "hi_star", "lo_new", "hi_new", "c_lo", "c_hi"):
+        assert np.float32(got[k]) == ref[k] or (np.isnan(got[k]) and np.isnan(ref[k])), (k, got[k], ref[k])
+    for k in ("n_neg", "n_pos", "k_bf16", "k_fp8", "flags", "shift", "sum_pos_bf16", "sum_neg_bf16",
+              "sum_neg_fp8", "sum_pos_fp8"):
+        assert got[k] == ref[k], (k, got[k], ref[k])
+    for k in ("rho_bf16", "rho_fp8"):
+        if np.isnan(ref[k]):
+            assert np.isnan(got[k])
+        else:
+            assert abs(got[k] - ref[k]) <= 1e-12 * max(1.0, abs(ref[k])), (k, got[k], ref[k])
+
+
+MODES = [OC.EXACT, OC.GRID]
+
+
+@pytest.mark.parametrize("mode", MODES)
+@pytest.mark.parametrize("T", [1, 2, 17, 1000, 40000])
+@pytest.mark.parametrize("eps", [(0.2, 0.2), (0.2, 0.28)])
+def test_calibrate_parity(cuda_lib, mode, T, eps):
+    args = _inputs(T, T + int(eps[1] * 100))
+    _compare(_run(cuda_lib, *args, *eps, mode=mode), _ref(*args, *eps, mode=mode))
+
+
+@pytest.mark.parametrize("mode", MODES)
+@pytest.mark.parametrize("seed", range(6))
+def test_calibrate_wide_noise_hits_interval_ends(cuda_lib, mode, seed):
+    """Large FP8 noise pushes the unconstrained optimum outside I_L / I_H."""
+    args = _inputs(5000, 300 + seed, sigma_fp8=[0.02, 0.3, 0.6, 1.0, 2.0, 0.1][seed])
+    _compare(_run(cuda_lib, *args, 0.2, 0.2, mode=mode), _ref(*args, 0.2, 0.2, mode=mode))
+
+
+@pytest.mark.parametrize("mode", MODES)
+@pytest.mark.parametrize("tie_every", [2, 7, 1000])
+def test_calibrate_ties(cuda_lib, mode, tie_every):
+    args = _inputs(6000, 41 + tie_every, tie_every=tie_every)
+    _compare(_run(cuda_lib, *args, 0.2, 0.2, mode=mode), _ref(*args, 0.2, 0.2, mode=mode))
+
+
+@pytest.mark.parametrize("mode", MODES)
+def test_calibrate_identity_returns_reference_bounds(cuda_lib, mode):
+    r_fp, r_bf, adv, mask, coef = _inputs(20000, 5)
+    got = _run(cuda_lib, r_bf, r_bf, adv, mask, coef, 0.2, 0.28, mode=mode)
+    c_lo, c_hi = OC.reference_bounds(0.2, 0.28)
+    assert np.float32(got["lo_star"]) == c_lo and np.float32(got["hi_star"]) == c_hi
+
+
+@pytest.mark.parametrize("scale", [1e-30, 1e-6, 1.0, 1e6, 1e30])
+def test_calibrate_coef_scales(cuda_lib, scale):
+    args = _inputs(3000, 8, coef_scale=scale)
+    _compare(_run(cuda_lib, *args, 0.2, 0.2), _ref(*args, 0.2, 0.2))
+
+
+@pytest.mark.parametrize("mode", MODES)
+def test_calibrate_smoothing_and_nullable_inputs(cuda_lib, mode):
+    r_fp, r_bf, adv, mask, coef = _inputs(4000, 12, sigma_fp8=0.1)
+    kw = dict(mode=mode, lo_old=0.6, hi_old=1.8)
+    _compare(_run(cuda_lib, r_fp, r_bf, adv, None, None, 0.2, 0.2, **kw),
+             _ref(r_fp, r_bf, adv, None, None, 0.2, 0.2, **kw))
+
+
+@pytest.mark.parametrize("mode", MODES)
+@pytest.mark.parametrize("case", ["no_neg", "no_pos", "all_masked", "empty", "zero_coef"])
+def test_calibrate_degenerate(cuda_lib, mode, case):
+    r_fp, r_bf, adv, mask, coef = _inputs(500, 13)
+    if case == "no_neg":
+        adv = adv.abs()
+    elif case == "no_pos":
+        adv = -adv.abs()
+    elif case == "all_masked":
+        mask = torch.zeros_like(mask)
+    elif case == "zero_coef":
+        coef = torch.zeros_like(coef)
+    elif case == "empty":
+        r_fp, r_bf, adv, mask, coef = (t[:0] for t in (r_fp, r_bf, adv, mask, coef))
+    _compare(_run(cuda_lib, r_fp, r_bf, adv, mask, coef, 0.2, 0.2, mode=mode),
+             _ref(r_fp, r_bf, adv, mask, coef, 0.2, 0.2, mode=mode))
+
+
+def test_calibrate_grid_custom_interval(cuda_lib):
+    args = _inputs(8000, 14, sigma_fp8=0.08)
+    kw = dict(mode=OC.GRID, lo_min=0.6, lo_max=0.95, hi_min=1.1, hi_max=3.0, step=0.005)
+    _compare(_run(cuda_lib, *args, 0.2, 0.2, **kw), _ref(*args, 0.2, 0.2, **kw))
+
+
+@pytest.mark.parametrize("name", ["grpo_8b", "dapo_32b", "long_8b"])
+def test_calibrate_full_size(cuda_lib, name):
+    """Token counts and group/mask layouts of the full workloads."""
+    w = synth.WORKLOADS[name]
+    adv, mask = synth.rollout(w)
+    r_bf, r_fp, coef = synth.ratio_inputs(w.T, w.seed, sigma_fp8=0.04)
+    for mode in MODES:
+        _compare(_run(cuda_lib, r_fp, r_bf, adv, mask, coef, w.eps_low, w.eps_high, mode=mode),
+                 _ref(r_fp, r_bf, adv, mask, coef, w.eps_low, w.eps_high, mode=mode))

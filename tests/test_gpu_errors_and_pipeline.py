@@ -1,0 +1,141 @@
+"""GPU: error reporting through the C ABI, the bounded-wait timeout path, and the
+whole hot path in one call sequence (properties that hold at any size)."""
+
+import ctypes
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import calibrate as OC
+from oracle import quantize as OQ
+from paper_2609_22870_gb300 import synth
+from tests.gpu_helpers import oracle_logprobs_rows, sample_rows
+
+pytestmark = pytest.mark.gpu
+
+
+def test_host_detected_errors(cuda_lib):
+    api = cuda_lib
+    x = torch.zeros(4, 200, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(api.Fp8rlError) as e:
+        api.quantize(x[:, :192], api.GRAN_BLOCK, api.ROLE_ACT)  # 192 % 128 != 0
+    assert e.value.status == api.ESHAPE
+    st = api.lib.fp8rl_quantize(None, 4, 128, 128, 0, 0, None, None, None, 0, None)
+    assert st == api.EINVAL
+    buf = torch.zeros(4 * 136 + 8, dtype=torch.bfloat16, device="cuda")
+    codes = torch.empty(4 * 128, dtype=torch.uint8, device="cuda")
+    sc = torch.empty(4, dtype=torch.float32, device="cuda")
+    st = api.lib.fp8rl_quantize(ctypes.c_void_p(buf.data_ptr() + 2), 4, 128, 136, 1, 0,
+                                ctypes.c_void_p(codes.data_ptr()), ctypes.c_void_p(sc.data_ptr()),
+                                None, 0, None)
+    assert st == api.EALIGN
+    st = api.lib.fp8rl_quantize(ctypes.c_void_p(buf.data_ptr()), 4, 128, 136, 0, 0,
+                                ctypes.c_void_p(codes.data_ptr()), ctypes.c_void_p(sc.data_ptr()),
+                                None, 0, None)
+    assert st == api.EWORKSPACE
+    api.check()
+
+
+def test_bad_target_flags_device_error_and_nan(cuda_lib):
+    api = cuda_lib
+    h = synth.normal_bf16(130, 128, 1.0, 1, "cuda")
+    W = synth.normal_bf16(300, 128, 0.02, 2, "cuda")
+    y = torch.randint(0, 300, (130,), dtype=torch.int32, device="cuda")
+    y[7] = 300
+    y[9] = -1
+    hc, hs = api.quantize(h, 0)
+    wc, ws = api.quantize(W, 0, api.ROLE_WEIGHT)
+    out = api.token_logprobs(hc, hs, wc, ws, 0, y)
+    assert api.check_status() == api.EDEVICE
+    lp = out["logp"].cpu().numpy()
+    assert np.isnan(lp[7]) and np.isnan(lp[9]) and np.all(np.isfinite(np.delete(lp, [7, 9])))
+    api.check()  # the status word was cleared
+
+
+def test_non_finite_inputs_flag(cuda_lib):
+    api = cuda_lib
+    x = torch.zeros(3, 128, dtype=torch.bfloat16, device="cuda")
+    x[1, 5] = float("inf")
+    api.quantize(x, api.GRAN_BLOCK, api.ROLE_ACT)
+    assert api.check_status() == api.EDEVICE
+    r = torch.ones(10, device="cuda")
+    r[3] = -1.0
+    api.calibrate_clip_bounds(r, torch.ones(10, device="cuda"), -torch.ones(10, device="cuda"), None,
+                              None, 0.2, 0.2)
+    assert api.check_status() == api.EDEVICE
+    api.check()
+
+
+def test_bounded_wait_expires_and_context_survives(cuda_lib):
+    api = cuda_lib
+    api.wait_selftest(2_000_000)  # 2 ms; nothing signals the barrier
+    assert api.check_status() == api.ETIMEOUT
+    x = synth.normal_bf16(8, 128, 1.0, 3, "cuda")
+    codes, scales = api.quantize(x, api.GRAN_ROWWISE)
+    api.check()
+    ref_c, _ = OQ.quantize(x.float().cpu().numpy(), OQ.ROWWISE)
+    assert np.array_equal(codes.cpu().numpy(), ref_c)
+
+
+@pytest.mark.parametrize("name,T,H,V", [("grpo_8b", 1100, 512, 5000), ("dapo_32b", 700, 640, 3000)])
+def test_pipeline_small(cuda_lib, name, T, H, V):
+    """score_calibrate_loss end to end at a size the oracle scores in full."""
+    api = cuda_lib
+    w = synth.scaled(synth.WORKLOADS[name], T=T, H=H, V=V)
+    h, W, y = synth.hidden_states(w, "cuda"), synth.lm_head_weight(w, "cuda"), synth.targets(w, "cuda")
+    adv, mask = synth.rollout(w)
+    ref_lp, _, _ = oracle_logprobs_rows(h, W, w.gran, y, np.arange(w.T))
+    noise = synth.old_policy_noise(w).numpy()
+    logp_old = (ref_lp + noise).astype(np.float32)        # old policy near the BF16 scorer
+    r_bf16 = np.exp(-noise).astype(np.float32)
+    coef = np.exp(logp_old).astype(np.float32)
+    b = api.score_calibrate_loss(h, W, y, torch.from_numpy(logp_old).cuda(), torch.from_numpy(r_bf16).cuda(),
+                                 adv.cuda(), mask.cuda(), torch.from_numpy(coef).cuda(), w.gran,
+                                 w.eps_low, w.eps_high)
+    api.check()
+    assert np.max(np.abs(b.logp.cpu().numpy() - ref_lp)) <= 2e-3
+    res = api.read_calib_result(b.cal_res)
+    st = api.read_clip_stats(b.stats)
+    _pipeline_properties(res, st, b, adv.numpy(), mask.numpy(), r_bf16, w)
+
+
+def _pipeline_properties(res, st, b, adv, mask, r_bf16, w):
+    r = b.ratio.cpu().numpy()
+    neg = (mask != 0) & (adv < 0)
+    pos = (mask != 0) & (adv > 0)
+    c_lo, c_hi = OC.reference_bounds(w.eps_low, w.eps_high)
+    assert res["n_neg"] == neg.sum() and res["n_pos"] == pos.sum()
+    assert res["k_bf16"] == int(np.sum(neg & (r_bf16 <= c_lo)))
+    assert res["k_fp8"] == int(np.sum(neg & (r <= np.float32(res["lo_star"]))))
+    assert 0.5 <= res["lo_star"] <= 0.9 and 1.2 <= res["hi_star"] <= 2.0
+    # new bounds = SmoothUpdate from no previous bound = searched bounds
+    assert res["lo_new"] == res["lo_star"] and res["hi_new"] == res["hi_star"]
+    # the loss used exactly these bounds
+    assert st["lo"] == res["lo_new"] and st["hi"] == res["hi_new"]
+    cm = b.clip_mask.cpu().numpy()
+    assert np.array_equal((cm & 1) != 0, pos & (r >= np.float32(res["hi_new"])))
+    assert np.array_equal((cm & 2) != 0, neg & (r <= np.float32(res["lo_new"])))
+
+
+@pytest.mark.parametrize("name", ["grpo_8b", "dapo_32b", "long_8b"])
+def test_pipeline_full_size(cuda_lib, name):
+    """The whole path at the full configurations: logp on sampled rows against
+    the oracle, every other stage by the properties it must satisfy."""
+    api = cuda_lib
+    w = synth.WORKLOADS[name]
+    h, W, y = synth.hidden_states(w, "cuda"), synth.lm_head_weight(w, "cuda"), synth.targets(w, "cuda")
+    adv, mask = synth.rollout(w)
+    noise = synth.old_policy_noise(w)
+    logp_old = torch.full((w.T,), -float(np.log(w.V))) + noise
+    r_bf16 = torch.exp(-noise)
+    coef = torch.exp(logp_old)
+    b = api.score_calibrate_loss(h, W, y, logp_old.float().cuda(), r_bf16.float().cuda(), adv.cuda(),
+                                 mask.cuda(), coef.float().cuda(), w.gran, w.eps_low, w.eps_high)
+    api.check()
+    rows = sample_rows(w.T, 16, 9)
+    ref_lp, _, _ = oracle_logprobs_rows(h, W, w.gran, y, rows)
+    assert np.max(np.abs(b.logp.cpu().numpy()[rows] - ref_lp)) <= 2e-3
+    res = api.read_calib_result(b.cal_res)
+    st = api.read_clip_stats(b.stats)
+    _pipeline_properties(res, st, b, adv.numpy(), mask.numpy(), r_bf16.float().numpy(), w)

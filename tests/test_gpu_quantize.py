@@ -1,0 +1,96 @@
+"""GPU parity: E4M3 quantisation (Eq. 3) bit-exact against the oracle."""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import quantize as OQ
+from paper_2609_22870_gb300 import synth
+from tests.gpu_helpers import scales_natural
+
+pytestmark = pytest.mark.gpu
+
+CASES = [(OQ.TENSOR, OQ.ACT), (OQ.ROWWISE, OQ.ACT), (OQ.ROWWISE, OQ.WEIGHT),
+         (OQ.BLOCK, OQ.ACT), (OQ.BLOCK, OQ.WEIGHT)]
+
+
+def _input(rows, cols, seed, ld=None):
+    x = synth.normal_bf16(rows, cols, 1.0, seed, "cuda").float()
+    g = torch.Generator(device="cpu").manual_seed(seed)
+    rowscale = torch.exp2(torch.randint(-20, 12, (rows, 1), generator=g).float()).cuda()
+    x = x * rowscale
+    if rows > 3:
+        x[1] = 0.0                      # an all-zero row: S = 1
+        x[2, : min(cols, 200)] = 0.0    # zero blocks
+    x = x.to(torch.bfloat16)
+    if ld is not None and ld > cols:
+        big = torch.zeros(rows, ld, dtype=torch.bfloat16, device="cuda")
+        big[:, :cols] = x
+        x = big[:, :cols]
+    return x
+
+
+@pytest.mark.parametrize("gran,role", CASES)
+@pytest.mark.parametrize("rows,cols,ld", [(1, 128, None), (7, 256, None), (129, 384, 512),
+                                          (300, 512, None), (1000, 4096, None), (257, 5120, None)])
+def test_quantize_bit_exact(cuda_lib, gran, role, rows, cols, ld):
+    x = _input(rows, cols, rows * 31 + cols, ld)
+    codes, scales = cuda_lib.quantize(x, gran, role)
+    cuda_lib.check()
+    ref_c, ref_s = OQ.quantize(x.float().cpu().numpy(), gran, role)
+    assert np.array_equal(codes.cpu().numpy(), ref_c)
+    assert np.array_equal(scales_natural(scales, rows, cols, gran, role), ref_s)
+
+
+@pytest.mark.parametrize("gran", [OQ.ROWWISE])
+def test_quantize_non_block_cols_multiple_of_16(cuda_lib, gran):
+    x = _input(33, 48, 5)
+    codes, scales = cuda_lib.quantize(x, gran, OQ.ACT)
+    cuda_lib.check()
+    ref_c, ref_s = OQ.quantize(x.float().cpu().numpy(), gran, OQ.ACT)
+    assert np.array_equal(codes.cpu().numpy(), ref_c)
+    assert np.array_equal(scales.cpu().numpy()[:33], ref_s)
+
+
+@pytest.mark.parametrize("name", ["grpo_8b", "dapo_32b"])
+@pytest.mark.parametrize("gran", [OQ.TENSOR, OQ.ROWWISE, OQ.BLOCK])
+def test_quantize_full_size_lm_head_sampled(cuda_lib, name, gran):
+    """Full Qwen-sized lm_head W (V = 151936): sampled 128-row strips bit-exact."""
+    w = synth.WORKLOADS[name]
+    W = synth.lm_head_weight(w, "cuda")
+    codes, scales = cuda_lib.quantize(W, gran, OQ.WEIGHT)
+    cuda_lib.check()
+    V, H = W.shape
+    rng = np.random.default_rng(0)
+    strips = sorted(set(rng.choice(V // 128, 6, replace=False).tolist() + [0, (V - 1) // 128]))
+    s_all = scales_natural(scales, V, H, gran, OQ.WEIGHT)
+    if gran == OQ.TENSOR:
+        amax = np.float32(0)
+        for v0 in range(0, V, 8192):
+            amax = max(amax, np.max(np.abs(W[v0:v0 + 8192].float().cpu().numpy())))
+        s_ref = OQ.scale_from_amax(amax).reshape(1)
+        assert np.array_equal(s_all, s_ref)
+    for sb in strips:
+        r0, r1 = sb * 128, min(V, sb * 128 + 128)
+        xs = W[r0:r1].float().cpu().numpy()
+        if gran == OQ.TENSOR:
+            ref_c = OQ._encode_block(xs, s_ref[0])
+        else:
+            ref_c, ref_s = OQ.quantize(xs, gran, OQ.WEIGHT)
+            got_s = s_all[r0:r1] if gran == OQ.ROWWISE else s_all[sb:sb + 1]
+            assert np.array_equal(got_s, ref_s)
+        assert np.array_equal(codes[r0:r1].cpu().numpy(), ref_c), (gran, sb)
+
+
+@pytest.mark.parametrize("name", ["grpo_8b", "long_8b"])
+def test_quantize_full_size_hidden_sampled(cuda_lib, name):
+    w = synth.WORKLOADS[name]
+    h = synth.hidden_states(w, "cuda")
+    codes, scales = cuda_lib.quantize(h, OQ.BLOCK, OQ.ACT)
+    cuda_lib.check()
+    rows = np.array(sorted(set(np.random.default_rng(1).choice(w.T, 200, replace=False).tolist()
+                               + [0, w.T - 1])))
+    ref_c, ref_s = OQ.quantize(h[torch.as_tensor(rows).cuda()].float().cpu().numpy(), OQ.BLOCK, OQ.ACT)
+    s_all = scales_natural(scales, w.T, w.H, OQ.BLOCK, OQ.ACT)
+    assert np.array_equal(codes[torch.as_tensor(rows).cuda()].cpu().numpy(), ref_c)
+    assert np.array_equal(s_all[rows], ref_s)
