@@ -217,7 +217,7 @@ def calibrate_clip_bounds(r_fp8, r_bf16, adv, mask, coef, eps_low, eps_high, opt
     r_fp8 = np.asarray(r_fp8, np.float32)
     r_bf16 = np.asarray(r_bf16, np.float32)
     adv = np.asarray(adv, np.float32)
-    mask = np.asarray(mask) != 0
+    mask = np.ones(r_fp8.size, bool) if mask is None else np.asarray(mask) != 0
     coef = np.ones_like(r_fp8) if coef is None else np.asarray(coef, np.float32)
     for a in (r_fp8, r_bf16, adv, coef):
         if not np.all(np.isfinite(a)):

@@ -28,11 +28,16 @@ CLIP_HI = 1  # bit set in the clip mask: A > 0 and r >= H
 CLIP_LO = 2  # bit set in the clip mask: A < 0 and r <= L
 
 
+def _valid(mask, n):
+    """Valid-token mask; no mask means every token is valid."""
+    return np.ones(n, bool) if mask is None else np.asarray(mask) != 0
+
+
 def clip_mask(r, adv, mask, lo, hi):
     """Per-token clip bits, compared in float32 as the inputs are float32."""
     r = np.asarray(r, np.float32)
     adv = np.asarray(adv, np.float32)
-    valid = np.asarray(mask) != 0
+    valid = _valid(mask, r.size)
     up = valid & (adv > 0) & (r >= np.float32(hi))
     dn = valid & (adv < 0) & (r <= np.float32(lo))
     return (up * CLIP_HI + dn * CLIP_LO).astype(np.uint8)
@@ -42,7 +47,7 @@ def clipped_surrogate(r, adv, mask, w, lo, hi):
     """Token-mean clipped surrogate loss, per-token terms, grad and counts."""
     r32 = np.asarray(r, np.float32)
     a32 = np.asarray(adv, np.float32)
-    valid = np.asarray(mask) != 0
+    valid = _valid(mask, r32.size)
     r64 = r32.astype(np.float64)
     a64 = a32.astype(np.float64)
     w64 = np.ones_like(r64) if w is None else np.asarray(w, np.float32).astype(np.float64)

@@ -78,3 +78,11 @@ def test_gradient_finite_difference(seed):
         e[t] = h
         fd = (loss(logp + e) - loss(logp - e)) / (2 * h)
         assert abs(fd - out["grad"][t]) < 5e-6 * max(1, abs(fd)), t
+
+
+def test_absent_mask_means_all_valid():
+    r = np.array([1.0, 1.5, 0.5], np.float32)
+    a = np.array([1.0, 1.0, -1.0], np.float32)
+    out = S.clipped_surrogate(r, a, None, None, 0.8, 1.2)
+    ref = S.clipped_surrogate(r, a, np.ones(3, np.uint8), None, 0.8, 1.2)
+    assert out["n_valid"] == 3 and out["loss"] == ref["loss"]
