@@ -55,7 +55,7 @@ def workload_desc(w):
 
 # ------------------------------------------------------------------ clocks
 class ClockSampler:
-    """nvidia-smi samples (200 ms) during the timed region."""
+    """nvidia-smi samples (every 100 ms) during the timed region."""
 
     FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -70,7 +70,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "100"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.thread = threading.Thread(target=self._read, daemon=True)
             self.thread.start()
@@ -137,6 +137,17 @@ def bf16_reference_logprobs(h, W, y, chunk=16384):
     return zy - (m + torch.log(s))
 
 
+def select_workload(args):
+    from paper_2609_22870_gb300 import synth
+    w = synth.WORKLOADS[args.workload]
+    if args.gran is not None:
+        import dataclasses
+        w = dataclasses.replace(w, name=f"{w.name}_g{args.gran}", gran=args.gran)
+    if args.tokens:
+        w = synth.scaled(w, T=args.tokens, name=f"{w.name}_T{args.tokens}")
+    return w
+
+
 def kernels_per_step(gran, mode):
     q = 2 if gran == 0 else 1
     calib = 6 if mode == 1 else 18
@@ -149,9 +160,7 @@ def run_ours(args, rank, world, local_rank):
 
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
-    w = synth.WORKLOADS[args.workload]
-    if args.gran is not None:
-        w = synth.granularity_sweep(args.gran) if args.workload == "grpo_8b" else w
+    w = select_workload(args)
     T, H, V, gran = w.T, w.H, w.V, w.gran
     h = synth.hidden_states(w, dev)
     W = synth.lm_head_weight(w, dev)
@@ -371,8 +380,8 @@ def run_reference(args, rank, world):
     from paper_2609_22870_gb300 import synth
     if rank != 0:
         return None
-    w = synth.WORKLOADS[args.workload]
-    per_step = max(2.0, 150.0 / max(1, args.steps + args.warmup))
+    w = select_workload(args)
+    per_step = max(0.1, 120.0 / max(1, args.steps + args.warmup))
     for i in range(args.warmup):
         oracle_step_estimate(w, budget_s=per_step, seed=100 + i)
     vals = []
@@ -397,11 +406,12 @@ def run_reference(args, rank, world):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
-    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="grpo_8b")
-    ap.add_argument("--gran", type=int, default=None, help="override granularity (0/1/2) of grpo_8b")
+    ap.add_argument("--gran", type=int, default=None, help="override the granularity (0 tensor, 1 row, 2 block)")
+    ap.add_argument("--tokens", type=int, default=0, help="score this many tokens instead (a smaller case)")
     ap.add_argument("--calib-mode", type=int, default=0)
     ap.add_argument("--cpu-budget", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -24,10 +24,10 @@ fp8rl_status cuda_fail(cudaError_t e) {
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 bool valid_gran(int g) { return g == FP8RL_GRAN_TENSOR || g == FP8RL_GRAN_ROWWISE || g == FP8RL_GRAN_BLOCK; }
 
-// Workspace layout of fp8rl_token_logprobs: partials [ceil(V/128)][T] float2,
-// then z_y [T] float.
+// Workspace layout of fp8rl_token_logprobs: per-token LSE partials
+// [gemm_partials_per_token(V)][T] float2, then z_y [T] float.
 size_t partials_bytes(int64_t T, int64_t V) {
-  return align_up(static_cast<size_t>((V + 127) / 128) * static_cast<size_t>(T) * sizeof(float2), 256);
+  return align_up(static_cast<size_t>(gemm_partials_per_token(V)) * static_cast<size_t>(T) * sizeof(float2), 256);
 }
 size_t logprob_ws(int64_t T, int64_t V) {
   return partials_bytes(T, V) + align_up(static_cast<size_t>(T) * sizeof(float), 256);

@@ -8,7 +8,12 @@
 //               swizzle, 4-stage shared-memory ring guarded by mbarriers;
 //   warp 1      MMA issuer: tcgen05.mma kind::f8f6f4 M=128 N=256 K=32, fp32
 //               accumulator in TMEM (two 256-column buffers);
-//   warps 2..9  epilogue: tcgen05.ld of the accumulator, one thread per token
+//   warp 2      block scaling only: stages each K block's activation and
+//               weight scales into a shared-memory ring, so the epilogue never
+//               waits on global loads;
+//   warp 3      idle (it completes the first warpgroup, whose register budget
+//               is lowered to 40 so the epilogue can hold 224);
+//   warps 4..11 epilogue: tcgen05.ld of the accumulator, one thread per token
 //               row and 128-column half, scales applied, then the running
 //               (max, sum exp) of its 128 columns and z[t][y_t] if y_t falls in
 //               them.  One (max, sum) pair per token and 128-wide vocabulary
@@ -38,12 +43,18 @@ constexpr int BK = 128;           // K bytes per stage (one 128B swizzle row)
 constexpr int CHUNK = 128;        // vocabulary columns per LSE partial
 constexpr int STAGES = 4;
 constexpr int EPI_WARPS = 8;
-constexpr int THREADS = 64 + EPI_WARPS * 32;
+constexpr int EPI_WARP0 = 4;      // first epilogue warp (start of warpgroup 1)
+constexpr int THREADS = 128 + EPI_WARPS * 32;
+constexpr int CTRL_REGS = 40;     // register budget of warpgroup 0 (producer, MMA)
+constexpr int EPI_REGS = 224;     // register budget of the two epilogue warpgroups
 constexpr uint32_t A_BYTES = BM * BK;
 constexpr uint32_t B_BYTES = BN * BK;
 constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr uint32_t TMEM_COLS = 2 * BN;
-constexpr size_t SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;
+constexpr int SC_SLOTS = 8;                       // scale ring depth (K blocks)
+constexpr uint32_t SC_SLOT_FLOATS = BM + 4;       // 128 activation + 2 weight (+2 pad)
+constexpr uint32_t SC_BYTES = SC_SLOTS * SC_SLOT_FLOATS * 4;
+constexpr size_t SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + SC_BYTES + 512;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr uint64_t kDrainNs = 1000000000ull;
 
@@ -137,12 +148,15 @@ __global__ void __launch_bounds__(THREADS, 1)
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* smA = smem;
   uint8_t* smB = smem + STAGES * A_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smB + STAGES * B_BYTES);
+  float* sc_ring = reinterpret_cast<float*>(smB + STAGES * B_BYTES);  // [SC_SLOTS][132]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smB + STAGES * B_BYTES + SC_BYTES);
   uint64_t* full = bars;
   uint64_t* empty = bars + STAGES;
   uint64_t* acc_full = bars + 2 * STAGES;
   uint64_t* acc_empty = acc_full + 2;
-  uint64_t* done = acc_empty + 2;
+  uint64_t* sc_full = acc_empty + 2;
+  uint64_t* sc_empty = sc_full + SC_SLOTS;
+  uint64_t* done = sc_empty + SC_SLOTS;
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(done + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
@@ -155,6 +169,10 @@ __global__ void __launch_bounds__(THREADS, 1)
     for (int b = 0; b < 2; ++b) {
       mbar_init(smem_u32(&acc_full[b]), 1);
       mbar_init(smem_u32(&acc_empty[b]), EPI_WARPS);
+    }
+    for (int i = 0; i < SC_SLOTS; ++i) {
+      mbar_init(smem_u32(&sc_full[i]), 32);
+      mbar_init(smem_u32(&sc_empty[i]), EPI_WARPS);
     }
     mbar_init(smem_u32(done), 1);
     *abort_flag = 0;
@@ -175,110 +193,145 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int total = p.num_m * p.num_n;
   const uint64_t lim = p.wait_limit_ns;
 
-  if (warp == 0) {
+  if (warp < EPI_WARP0) {
+   warpgroup_reg_dealloc<CTRL_REGS>();
+   if (warp == 0) {
     // ------------------------------------------------------------ producer
-    if (lane == 0) {
-      int stage = 0;
-      uint32_t phase = 0;
-      uint32_t armed = 0, armed_phase = 0;  // bit s: stage s loaded / its parity
-      bool ok = true;
-      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
-        const int m0 = (tile % p.num_m) * BM, n0 = (tile / p.num_m) * BN;
-        for (int kb = 0; kb < p.num_kb; ++kb) {
-          if (!mbar_wait(smem_u32(&empty[stage]), phase ^ 1, lim, abort_flag)) {
-            ok = false;
-            break;
-          }
+    // the whole warp runs the loop (uniform control flow); one elected lane
+    // issues the barrier arrive and the two TMA loads of each stage
+    int stage = 0;
+    uint32_t phase = 0;
+    uint32_t armed = 0, armed_phase = 0;  // bit s: stage s loaded / its parity
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+      const int m0 = (tile % p.num_m) * BM, n0 = (tile / p.num_m) * BN;
+      for (int kb = 0; kb < p.num_kb; ++kb) {
+        ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&empty[stage]), phase ^ 1, lim, abort_flag));
+        if (!ok) break;
+        if (elect_one()) {
           mbar_arrive_expect_tx(smem_u32(&full[stage]), STAGE_BYTES);
           tma_load_2d(smem_u32(smA + stage * A_BYTES), &tmA, smem_u32(&full[stage]), kb * BK, m0);
           tma_load_2d(smem_u32(smB + stage * B_BYTES), &tmB, smem_u32(&full[stage]), kb * BK, n0);
-          armed |= 1u << stage;
-          armed_phase = (armed_phase & ~(1u << stage)) | (phase << stage);
-          if (++stage == STAGES) {
-            stage = 0;
-            phase ^= 1;
-          }
+        }
+        __syncwarp();
+        armed |= 1u << stage;
+        armed_phase = (armed_phase & ~(1u << stage)) | (phase << stage);
+        if (++stage == STAGES) {
+          stage = 0;
+          phase ^= 1;
         }
       }
-      if (!ok) {
-        *abort_flag = 1;
-        flag(kErrTimeout);
-      }
-      // no copy may still be in flight when the CTA exits
-      for (int s = 0; s < STAGES; ++s)
-        if (armed & (1u << s)) mbar_wait(smem_u32(&full[s]), (armed_phase >> s) & 1, kDrainNs, nullptr);
     }
-  } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      int stage = 0, ab = 0;
-      uint32_t phase = 0, aphase = 0;
-      constexpr uint32_t idesc = idesc_e4m3_f32(BM, BN);
-      bool ok = true;
-      for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
-        if (MODE != kBlock) {
-          if (!mbar_wait(smem_u32(&acc_empty[ab]), aphase ^ 1, lim, abort_flag)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-        }
-        for (int kb = 0; kb < p.num_kb; ++kb) {
-          if (!mbar_wait(smem_u32(&full[stage]), phase, lim, abort_flag)) {
-            ok = false;
-            break;
-          }
-          if (MODE == kBlock) {
-            if (!mbar_wait(smem_u32(&acc_empty[ab]), aphase ^ 1, lim, abort_flag)) {
-              ok = false;
-              break;
-            }
-          }
-          tc_fence_after();
-          const uint32_t d = tmem_base + static_cast<uint32_t>(ab * BN);
-          const uint64_t adesc = smem_desc_sw128(smem_u32(smA + stage * A_BYTES));
-          const uint64_t bdesc = smem_desc_sw128(smem_u32(smB + stage * B_BYTES));
-#pragma unroll
-          for (int k = 0; k < BK / 32; ++k) {
-            const uint32_t acc = (MODE == kBlock) ? (k > 0) : (kb > 0 || k > 0);
-            // +32 bytes along K inside the swizzled 128-byte row
-            mma_f8f6f4(d, adesc + 2 * k, bdesc + 2 * k, idesc, acc);
-          }
-          mma_commit(smem_u32(&empty[stage]));
-          if (MODE == kBlock) {
-            mma_commit(smem_u32(&acc_full[ab]));
-            ab ^= 1;
-            if (ab == 0) aphase ^= 1;
-          }
-          if (++stage == STAGES) {
-            stage = 0;
-            phase ^= 1;
-          }
-        }
+    if (!ok && lane == 0) {
+      *abort_flag = 1;
+      flag(kErrTimeout);
+    }
+    // no copy may still be in flight when the CTA exits
+    for (int s = 0; s < STAGES; ++s)
+      if (armed & (1u << s)) mbar_wait(smem_u32(&full[s]), (armed_phase >> s) & 1, kDrainNs, nullptr);
+   } else if (warp == 2 && MODE == kBlock) {
+    // ------------------------------------------------------------ scale loader
+    // per K block: the 128 activation scales S_h[kb][m0 .. m0+127] and the
+    // scales of the two weight blocks the tile spans, into ring slot `slot`
+    int slot = 0;
+    uint32_t sphase = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+      const int m0 = (tile % p.num_m) * BM, n_blk = tile / p.num_m;
+      const int wb0 = 2 * n_blk;
+      for (int kb = 0; kb < p.num_kb; ++kb) {
+        ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&sc_empty[slot]), sphase ^ 1, lim, abort_flag));
         if (!ok) break;
-        if (MODE != kBlock) {
-          mma_commit(smem_u32(&acc_full[ab]));
+        const uint32_t dst = smem_u32(sc_ring + slot * SC_SLOT_FLOATS);
+        const float* src = p.a_scales + static_cast<size_t>(kb) * p.M;
+        // asynchronous 4-byte copies: the warp never waits for the data, the
+        // barrier completes when every lane's copies have landed
+#pragma unroll
+        for (int j = 0; j < BM / 32; ++j) {
+          const int r = m0 + j * 32 + lane;
+          if (r < p.M) cp_async_4(dst + (j * 32 + lane) * 4, src + r);
+        }
+        if (lane < 2 && wb0 + lane < p.n_chunks)
+          cp_async_4(dst + (BM + lane) * 4, p.b_scales + static_cast<size_t>(wb0 + lane) * p.num_kb + kb);
+        cp_async_mbar_arrive(smem_u32(&sc_full[slot]));
+        if (++slot == SC_SLOTS) {
+          slot = 0;
+          sphase ^= 1;
+        }
+      }
+    }
+    if (!ok && lane == 0) {
+      *abort_flag = 1;
+      flag(kErrTimeout);
+    }
+    asm volatile("cp.async.wait_all;" ::: "memory");  // no copy in flight at exit
+   } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    // whole warp converged; elect.sync picks the lane that issues each
+    // tcgen05.mma / tcgen05.commit
+    int stage = 0, ab = 0;
+    uint32_t phase = 0, aphase = 0;
+    constexpr uint32_t idesc = idesc_e4m3_f32(BM, BN);
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+      if (MODE != kBlock) {
+        ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&acc_empty[ab]), aphase ^ 1, lim, abort_flag));
+        if (!ok) break;
+        tc_fence_after();
+      }
+      for (int kb = 0; kb < p.num_kb; ++kb) {
+        ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&full[stage]), phase, lim, abort_flag));
+        if (!ok) break;
+        if (MODE == kBlock) {
+          ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&acc_empty[ab]), aphase ^ 1, lim, abort_flag));
+          if (!ok) break;
+        }
+        tc_fence_after();
+        const uint32_t d = tmem_base + static_cast<uint32_t>(ab * BN);
+        const uint64_t adesc = smem_desc_sw128(smem_u32(smA + stage * A_BYTES));
+        const uint64_t bdesc = smem_desc_sw128(smem_u32(smB + stage * B_BYTES));
+#pragma unroll
+        for (int k = 0; k < BK / 32; ++k) {
+          const uint32_t acc = (MODE == kBlock) ? (k > 0) : (kb > 0 || k > 0);
+          // +32 bytes along K inside the swizzled 128-byte row
+          mma_f8f6f4_elect(d, adesc + 2 * k, bdesc + 2 * k, idesc, acc);
+        }
+        mma_commit_elect(smem_u32(&empty[stage]));
+        if (MODE == kBlock) {
+          mma_commit_elect(smem_u32(&acc_full[ab]));
           ab ^= 1;
           if (ab == 0) aphase ^= 1;
         }
+        if (++stage == STAGES) {
+          stage = 0;
+          phase ^= 1;
+        }
       }
-      if (!ok) {
-        *abort_flag = 1;
-        flag(kErrTimeout);
+      if (!ok) break;
+      if (MODE != kBlock) {
+        mma_commit_elect(smem_u32(&acc_full[ab]));
+        ab ^= 1;
+        if (ab == 0) aphase ^= 1;
       }
-      // every MMA issued above has completed once this commit lands
-      mma_commit(smem_u32(done));
-      mbar_wait(smem_u32(done), 0, kDrainNs, nullptr);
     }
+    if (!ok && lane == 0) {
+      *abort_flag = 1;
+      flag(kErrTimeout);
+    }
+    // every MMA issued above has completed once this commit lands
+    mma_commit_elect(smem_u32(done));
+    mbar_wait(smem_u32(done), 0, kDrainNs, nullptr);
+   }
   } else {
+    warpgroup_reg_alloc<EPI_REGS>();
     // ------------------------------------------------------------ epilogue
-    const int ew = warp - 2;
+    const int ew = warp - EPI_WARP0;
     const int quarter = warp & 3;  // TMEM lanes this warp may access
     const int half = ew >> 2;      // which 128 columns of the 256-wide tile
     const int rit = quarter * 32 + lane;
     const uint32_t t_row = static_cast<uint32_t>(quarter * 32) << 16;
-    int ab = 0;
-    uint32_t aphase = 0;
+    int ab = 0, sslot = 0;
+    uint32_t aphase = 0, sphase = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
       const int m_blk = tile % p.num_m, n_blk = tile / p.num_m;
@@ -289,38 +342,54 @@ __global__ void __launch_bounds__(THREADS, 1)
       EpiState es;
       epi_begin<EPI>(p, es, row, col0);
       if (MODE == kBlock) {
-        float z[CHUNK];
+        float2 z2[CHUNK / 2];
 #pragma unroll
-        for (int i = 0; i < CHUNK; ++i) z[i] = 0.f;
-        const bool wb_ok = chunk < p.n_chunks;
-        const float* sa_ptr = p.a_scales + row;                                    // [kb][M]
-        const float* sb_ptr = p.b_scales + static_cast<size_t>(chunk) * p.num_kb;  // [vb][kb]
-        float sa = row_ok ? __ldg(sa_ptr) : 0.f;
-        float sb = wb_ok ? __ldg(sb_ptr) : 0.f;
+        for (int i = 0; i < CHUNK / 2; ++i) z2[i] = make_float2(0.f, 0.f);
         for (int kb = 0; kb < p.num_kb; ++kb) {
-          const float sc = sa * sb;
-          if (kb + 1 < p.num_kb) {
-            sa = row_ok ? __ldg(sa_ptr + static_cast<size_t>(kb + 1) * p.M) : 0.f;
-            sb = wb_ok ? __ldg(sb_ptr + kb + 1) : 0.f;
+          // this K block's scales from the ring (staged by the loader warp)
+          ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&sc_full[sslot]), sphase, lim, abort_flag));
+          if (!ok) break;
+          const float* scs = sc_ring + sslot * SC_SLOT_FLOATS;
+          const float sc = scs[rit] * scs[BM + half];
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&sc_empty[sslot]));
+          if (++sslot == SC_SLOTS) {
+            sslot = 0;
+            sphase ^= 1;
           }
           ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&acc_full[ab]), aphase, lim, abort_flag));
           if (!ok) break;
           tc_fence_after();
           const uint32_t taddr = tmem_base + t_row + static_cast<uint32_t>(ab * BN + half * CHUNK);
+          const float2 sc2 = make_float2(sc, sc);
+          // four 32-column chunks, double-buffered: the load of chunk c + 1
+          // is in flight while chunk c is promoted; the TMEM buffer goes back
+          // to the MMA as soon as the last chunk has landed in registers
+          uint32_t ra[32], rb[32];
+          tmem_ld_32x32b_x32_issue(taddr, ra);
+          tmem_wait_ld(ra);
 #pragma unroll
           for (int c = 0; c < CHUNK / 32; ++c) {
-            float v[32];
-            tmem_ld_32x32b_x32(taddr + c * 32, v);
+            uint32_t(&cur)[32] = (c & 1) ? rb : ra;
+            uint32_t(&nxt)[32] = (c & 1) ? ra : rb;
+            if (c + 1 < CHUNK / 32) tmem_ld_32x32b_x32_issue(taddr + (c + 1) * 32, nxt);
+            if (c + 1 == CHUNK / 32) {
+              tc_fence_before();
+              __syncwarp();
+              if (lane == 0) mbar_arrive(smem_u32(&acc_empty[ab]));
+            }
 #pragma unroll
-            for (int i = 0; i < 32; ++i) z[c * 32 + i] = fmaf(v[i], sc, z[c * 32 + i]);
+            for (int i = 0; i < 16; ++i) {
+              z2[c * 16 + i].x = fmaf(__uint_as_float(cur[2 * i]), sc, z2[c * 16 + i].x);
+              z2[c * 16 + i].y = fmaf(__uint_as_float(cur[2 * i + 1]), sc, z2[c * 16 + i].y);
+            }
+            if (c + 1 < CHUNK / 32) tmem_wait_ld(nxt);
           }
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(smem_u32(&acc_empty[ab]));
           ab ^= 1;
           if (ab == 0) aphase ^= 1;
         }
         if (!ok) break;
+        const float* z = reinterpret_cast<const float*>(z2);
 #pragma unroll
         for (int c = 0; c < CHUNK / 32; ++c) epi_consume32<EPI>(p, es, z + c * 32, row, col0, c * 32);
       } else {
@@ -505,8 +574,18 @@ cudaError_t launch_mode(const CUtensorMap& ta, const CUtensorMap& tb, const Para
   int dev = 0;
   cudaGetDevice(&dev);
   if (configured_device != dev) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(SMEM_BYTES));
+    // The warpgroups re-split the registers the CTA was launched with
+    // (setmaxnreg): each SM sub-partition holds one control warp and two
+    // epilogue warps, so 3 x (launch registers) must cover 40 + 2 x 224.
+    // Refuse to launch a build where that does not hold (it would wait forever).
+    cudaFuncAttributes attr;
+    cudaError_t e = cudaFuncGetAttributes(&attr, kern);
+    if (e != cudaSuccess) return e;
+    if (attr.numRegs * 3 < CTRL_REGS + 2 * EPI_REGS ||
+        attr.numRegs * THREADS < 128 * CTRL_REGS + EPI_WARPS * 32 * EPI_REGS)
+      return cudaErrorInvalidConfiguration;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(SMEM_BYTES));
     if (e != cudaSuccess) return e;
     configured_device = dev;
   }
@@ -552,6 +631,8 @@ int blocks_for(int64_t n, int threads) {
 }
 
 }  // namespace
+
+int64_t gemm_partials_per_token(int64_t N) { return (N + CHUNK - 1) / CHUNK; }
 
 cudaError_t launch_gemm_lse(const GemmArgs& a, cudaStream_t s) { return launch_gemm<kEpiLse>(a, s); }
 

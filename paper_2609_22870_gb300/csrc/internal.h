@@ -30,13 +30,16 @@ struct GemmArgs {
   int64_t M, N, K;
   const int32_t* targets;   // [M]
   // LSE epilogue outputs (workspace)
-  float2* partials;         // [ceil(N/128)][M]
+  float2* partials;         // [gemm_partials_per_token(N)][M]
   float* zy;                // [M]
   // dlogits epilogue
   const float* lse;         // [M]
   const float* grad;        // [M]
   float* out;               // [M][N]
 };
+// LSE partials the GEMM leaves per token (one per column slot of each
+// 256-wide vocabulary tile).
+int64_t gemm_partials_per_token(int64_t N);
 cudaError_t launch_gemm_lse(const GemmArgs& a, cudaStream_t s);
 cudaError_t launch_gemm_dlogits(const GemmArgs& a, cudaStream_t s);
 cudaError_t launch_combine(const float2* partials, const float* zy, const int32_t* targets,
