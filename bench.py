@@ -35,6 +35,11 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 FP8_OVER_BF16 = 4.5 / 2.25  # nominal dense FP8 / BF16 tensor rates
 GRAN_NAMES = {0: "tensor", 1: "row", 2: "block"}
 
+# DRAM bytes (read + write) per launch of the GEMM kernel on the default
+# workload, from one ncu capture (profiles/fp8_gemm_kernel_block_T2048_full_and_traffic.md);
+# reported only while the kernel source is the one that was measured.
+GEMM_TRAFFIC = {"workload": "grpo_8b", "bytes": 5.56e9, "gemm_cu_sha256_prefix": "5829fd7ed9aae213"}
+
 
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
@@ -43,6 +48,16 @@ def load_peaks():
             d = json.load(f)
         return d, "measured"
     return dict(FALLBACK_PEAKS), "fallback"
+
+
+def measured_gemm_traffic(w):
+    import hashlib
+    src = os.path.join(ROOT, "paper_2609_22870_gb300", "csrc", "gemm.cu")
+    with open(src, "rb") as f:
+        digest = hashlib.sha256(f.read()).hexdigest()[:16]
+    if w.name == GEMM_TRAFFIC["workload"] and digest == GEMM_TRAFFIC["gemm_cu_sha256_prefix"]:
+        return GEMM_TRAFFIC["bytes"]
+    return None
 
 
 def workload_desc(w):
@@ -302,7 +317,7 @@ def run_ours(args, rank, world, local_rank):
                      "achieved": achieved, "peak": fp8_peak, "unit": "TFLOP/s",
                      "frac": achieved / fp8_peak,
                      "peak_source": f"{peak_src} bf16 sustained x {FP8_OVER_BF16:g} (nominal FP8/BF16)",
-                     "traffic": None},
+                     "traffic": measured_gemm_traffic(w), "traffic_unit": "bytes per launch"},
         "stages_ms": {"quantize_h": stage[0], "quantize_w": stage[1], "gemm_lse": stage[2],
                       "combine": stage[3], "calibrate": stage[4], "surrogate": stage[5]},
         "e2e": {"value": world * T / (e2e_ms * 1e-3), "unit": "tokens/s",
