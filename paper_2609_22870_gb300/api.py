@@ -68,6 +68,7 @@ _SIGS = {
     "fp8rl_logit_partials": (_i, [_p, _p, _p, _p, _i, _i64, _i64, _i64, _p, _p, _sz, _p]),
     "fp8rl_combine_logprobs": (_i, [_i64, _i64, _i64, _i, _p, _p, _p, _p, _p, _p, _sz, _p]),
     "fp8rl_importance_ratios": (_i, [_p, _p, _i64, _p, _p]),
+    "fp8rl_token_logprobs_noalloc": (_i, [_p, _p, _p, _p, _i, _i64, _i64, _i64, _p, _p, _p, _p, _p, _p]),
     "fp8rl_default_calib_opts": (None, [ctypes.POINTER(CalibOpts)]),
     "fp8rl_calibrate_workspace_size": (_sz, [_i64]),
     "fp8rl_calibrate_clip_bounds": (_i, [_p, _p, _p, _p, _p, _i64, _f, _f, ctypes.POINTER(CalibOpts),
@@ -200,6 +201,26 @@ def token_logprobs(h_codes, h_scales, w_codes, w_scales, gran, targets, logp_old
                                  T, H, V, _ptr(targets), _ptr(logp_old), _ptr(logp), _ptr(lse),
                                  _ptr(ratio), _ptr(workspace), workspace.numel(), _stream(stream)),
         "fp8rl_token_logprobs")
+    return {"logp": logp, "lse": lse, "ratio": ratio}
+
+
+def token_logprobs_noalloc(h_codes, h_scales, w_codes, w_scales, gran, targets, logp_old=None,
+                           want_lse=True, want_ratio=None, out=None, stream=None):
+    """fp8rl_token_logprobs_noalloc: like token_logprobs, but the scratch is the
+    library's fixed static array, for callers that cannot allocate a workspace
+    (shapes needing more than FP8RL_NOALLOC_SCRATCH_BYTES are refused)."""
+    T, H, V = _gemm_args(h_codes, h_scales, w_codes, w_scales, targets)
+    dev = h_codes.device
+    want_ratio = logp_old is not None if want_ratio is None else want_ratio
+    _dev(logp_old, torch.float32, "logp_old", T)
+    o = out or {}
+    logp = o.get("logp", torch.empty(T, dtype=torch.float32, device=dev))
+    lse = o.get("lse", torch.empty(T, dtype=torch.float32, device=dev)) if want_lse else None
+    ratio = o.get("ratio", torch.empty(T, dtype=torch.float32, device=dev)) if want_ratio else None
+    _ok(lib.fp8rl_token_logprobs_noalloc(_ptr(h_codes), _ptr(h_scales), _ptr(w_codes), _ptr(w_scales),
+                                         gran, T, H, V, _ptr(targets), _ptr(logp_old), _ptr(logp),
+                                         _ptr(lse), _ptr(ratio), _stream(stream)),
+        "fp8rl_token_logprobs_noalloc")
     return {"logp": logp, "lse": lse, "ratio": ratio}
 
 

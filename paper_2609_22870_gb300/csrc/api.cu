@@ -46,6 +46,8 @@ fp8rl_status check_gemm_shape(const uint8_t* hc, const float* hs, const uint8_t*
 
 uint64_t wait_limit_ns() { return g_wait_ns.load(std::memory_order_relaxed); }
 
+void record_cuda_error(cudaError_t e) { cuda_fail(e); }
+
 int sm_count() {
   static int cached[64] = {0};
   int dev = 0;

@@ -74,4 +74,7 @@ uint32_t loss_status_take();
 // SM count of the current device (cached per device).
 int sm_count();
 
+// Records `e` as the text fp8rl_last_cuda_error() returns on this thread.
+void record_cuda_error(cudaError_t e);
+
 }  // namespace fp8rl
