@@ -418,6 +418,80 @@ def run_reference(args, rank, world):
             "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
+def run_kernel_rooflines(args, local_rank):
+    """HBM-bound kernels at stress sizes: bytes are the algorithmic bytes of
+    one call (every input read once, every output written once), time is the
+    CUDA-event average over repeated calls on inputs larger than L2."""
+    import torch
+    from paper_2609_22870_gb300 import api, synth
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    peaks, src = load_peaks()
+    hbm = peaks["hbm_gbs"]
+    out = []
+
+    def timed(fn, reps):
+        fn()
+        torch.cuda.synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(reps):
+            fn()
+        b.record()
+        torch.cuda.synchronize()
+        api.check()
+        return a.elapsed_time(b) / reps
+
+    def line(kernel, shape, nbytes, ms):
+        gbs = nbytes / (ms * 1e-3) / 1e9
+        out.append({"kernel": kernel, "shape": shape, "bytes": nbytes, "ms": ms, "GB/s": gbs,
+                    "peak_GB/s": hbm, "frac": gbs / hbm, "peak_source": src})
+
+    # a1/a2 quantise at the long workload's h (T 131072 x 4096) and the lm_head W
+    T, H, V = 131072, 4096, 151936
+    h = synth.normal_bf16(T, H, 1.0, 7, dev)
+    for gran, name in ((2, "block 1x128"), (1, "row"), (0, "tensor")):
+        codes = torch.empty(T, H, dtype=torch.uint8, device=dev)
+        sc = torch.empty(max(1, api.scales_count(T, H, gran, 0)), dtype=torch.float32, device=dev)
+        ws = torch.empty(256, dtype=torch.uint8, device=dev)
+        ms = timed(lambda: api.quantize(h, gran, 0, codes, sc, ws), 10)
+        line(f"quantize h ({name})", [T, H], T * H * 3 + sc.numel() * 4, ms)
+    del h, codes
+    W = synth.normal_bf16(V, H, 0.02, 8, dev)
+    for gran, name in ((2, "block 128x128"), (1, "row")):
+        codes = torch.empty(V, H, dtype=torch.uint8, device=dev)
+        sc = torch.empty(max(1, api.scales_count(V, H, gran, 1)), dtype=torch.float32, device=dev)
+        ms = timed(lambda: api.quantize(W, gran, 1, codes, sc), 10)
+        line(f"quantize W ({name})", [V, H], V * H * 3 + sc.numel() * 4, ms)
+    del W, codes
+
+    # a5/a6 at T = 2^27 synthetic ratios
+    T = 1 << 27
+    g = torch.Generator(device=dev)
+    g.manual_seed(9)
+    r_bf = torch.exp(torch.randn(T, generator=g, device=dev) * 0.05)
+    r_fp = r_bf * torch.exp(torch.randn(T, generator=g, device=dev) * 0.05)
+    adv = torch.randn(T, generator=g, device=dev)
+    coef = torch.exp(torch.randn(T, generator=g, device=dev) * 2 - 11)
+    mask = (torch.rand(T, generator=g, device=dev) < 0.9).to(torch.uint8)
+    res = torch.zeros(128, dtype=torch.uint8, device=dev)
+    cws = torch.empty(api.calibrate_workspace_size(T), dtype=torch.uint8, device=dev)
+    for mode, name in ((0, "exact"), (1, "grid")):
+        opts = api.calib_opts(mode=mode)
+        ms = timed(lambda: api.calibrate_clip_bounds(r_fp, r_bf, adv, mask, coef, 0.2, 0.2, opts, res, cws), 5)
+        line(f"calibrate ({name})", [T], T * 17, ms)
+    grad = torch.empty(T, device=dev)
+    cm = torch.empty(T, dtype=torch.uint8, device=dev)
+    st = torch.zeros(128, dtype=torch.uint8, device=dev)
+    sws = torch.empty(api.surrogate_workspace_size(T), dtype=torch.uint8, device=dev)
+    ms = timed(lambda: api.clipped_surrogate(r_fp, adv, mask, None, 0.8, 1.2, None, stats=st, workspace=sws,
+                                             out={"grad": grad, "clip_mask": cm}), 10)
+    line("clipped surrogate", [T], T * (4 + 4 + 1 + 4 + 1), ms)
+    return out
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -430,12 +504,18 @@ def main():
     ap.add_argument("--calib-mode", type=int, default=0)
     ap.add_argument("--cpu-budget", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--kernels", action="store_true",
+                    help="print HBM rooflines of the memory-bound kernels at stress sizes instead")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.kernels:
+        for item in run_kernel_rooflines(args, local_rank):
+            print(json.dumps(item), flush=True)
+        return
     if args.impl == "reference":
         line = run_reference(args, rank, world)
     else:

@@ -48,6 +48,19 @@ uint64_t wait_limit_ns() { return g_wait_ns.load(std::memory_order_relaxed); }
 
 void record_cuda_error(cudaError_t e) { cuda_fail(e); }
 
+void* tensormap_encoder() {
+  static void* fn = nullptr;
+  if (fn == nullptr) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = ptr;
+  }
+  return fn;
+}
+
 int sm_count() {
   static int cached[64] = {0};
   int dev = 0;

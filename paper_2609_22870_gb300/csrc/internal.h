@@ -77,4 +77,8 @@ int sm_count();
 // Records `e` as the text fp8rl_last_cuda_error() returns on this thread.
 void record_cuda_error(cudaError_t e);
 
+// The driver's cuTensorMapEncodeTiled (PFN_cuTensorMapEncodeTiled_v12000), or
+// null when the driver does not provide it.
+void* tensormap_encoder();
+
 }  // namespace fp8rl

@@ -4,6 +4,7 @@ import numpy as np
 import pytest
 import torch
 
+from oracle import e4m3
 from oracle import quantize as OQ
 from paper_2609_22870_gb300 import synth
 from tests.gpu_helpers import scales_natural
@@ -94,3 +95,47 @@ def test_quantize_full_size_hidden_sampled(cuda_lib, name):
     s_all = scales_natural(scales, w.T, w.H, OQ.BLOCK, OQ.ACT)
     assert np.array_equal(codes[torch.as_tensor(rows).cuda()].cpu().numpy(), ref_c)
     assert np.array_equal(s_all[rows], ref_s)
+
+
+def _adversarial_bits(seed):
+    """One 128-element row per positive finite bf16 amax (bit patterns
+    0x0001 .. 0x7F7F, so every block scale S a bf16 block can have, from the
+    subnormal range to 3.39e38 / 448), the other elements placed on bf16
+    values next to E4M3 rounding midpoints times S, where the quotient's last
+    bits decide the code, plus signed zeros."""
+    rng = np.random.default_rng(seed)
+    a_bits = np.arange(1, 0x7F80, dtype=np.uint32)
+    n = a_bits.size
+    amax = (a_bits << 16).view(np.float32)
+    s = OQ.scale_from_amax(amax).astype(np.float64)
+    vals = np.sort(np.unique(np.abs(e4m3.decode(np.arange(0, 0x7F, dtype=np.uint8)).astype(np.float64))))
+    mids = (vals[:-1] + vals[1:]) / 2
+    target = mids[rng.integers(0, mids.size, size=(n, 127))] * s[:, None]
+    t = target.astype(np.float32).view(np.uint32)
+    rb = (t + 0x7FFF + ((t >> 16) & 1)) >> 16                  # nearest bf16
+    rb = rb.astype(np.int64) + rng.integers(-1, 2, size=rb.shape)  # and its neighbours
+    rb = np.clip(rb, 0, a_bits[:, None].astype(np.int64))
+    sign = rng.integers(0, 2, size=(n, 128)).astype(np.int64) << 15
+    bits = np.empty((n, 128), dtype=np.int64)
+    bits[:, 0] = a_bits
+    bits[:, 1:] = rb
+    bits |= sign
+    bits[::3, 127] = 0x8000                                     # -0
+    bits[1::3, 127] = 0x0000                                    # +0
+    return bits.astype(np.uint16).view(np.int16)
+
+
+@pytest.mark.parametrize("gran,role", CASES)
+def test_quantize_every_bf16_scale_near_midpoints(cuda_lib, gran, role):
+    """The division-free quotient against fl32(x / S) at every block scale
+    and at the inputs most sensitive to its last bit."""
+    bits = _adversarial_bits(7)
+    x = torch.from_numpy(bits).view(torch.bfloat16).cuda()
+    rows, cols = x.shape
+    codes, scales = cuda_lib.quantize(x, gran, role)
+    cuda_lib.check()
+    ref_c, ref_s = OQ.quantize(x.float().cpu().numpy(), gran, role)
+    assert np.array_equal(scales_natural(scales, rows, cols, gran, role), ref_s)
+    got = codes.cpu().numpy()
+    bad = np.argwhere(got != ref_c)
+    assert bad.size == 0, (bad[:5], got[tuple(bad[0])], ref_c[tuple(bad[0])])
