@@ -277,8 +277,9 @@ typedef struct fp8rl_clip_stats {
 size_t fp8rl_surrogate_workspace_size(int64_t T);
 
 /* l_t = -w_t min(r_t A_t, clip(r_t, L, H) A_t) (Eq. 1 with the TIS weight of
- * Eq. 4 and calibrated bounds), loss = sum_valid l_t / n_valid (token mean,
- * float64 accumulation, deterministic for a given T).
+ * Eq. 4 and calibrated bounds), loss = sum_valid l_t / n_valid (token mean;
+ * float32 terms summed with compensation per thread, float64 across threads
+ * in a fixed order: deterministic for a given T on a given device).
  *   r, adv       float [T];  mask uint8 [T] or NULL;  w_tis float [T] or NULL (1)
  *   lo, hi       bounds by value, used when `bounds` is NULL
  *   bounds       DEVICE float[2] {L, H} or NULL (e.g. a fp8rl_calib_result*)

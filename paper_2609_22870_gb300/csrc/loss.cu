@@ -1,15 +1,20 @@
 // a6/a7: clipped surrogate with TIS weights (Eq. 1, Eq. 4), token-mean
 // aggregation, clip counts by advantage sign and dloss/dlogp.
 //
-//   l_t = -w_t min(r_t A_t, clip(r_t, L, H) A_t)        (float64)
+//   l_t = -w_t min(r_t A_t, clip(r_t, L, H) A_t) = -w_t A_t m_t,
+//         m_t = min(r_t, H) when A_t >= 0, max(r_t, L) when A_t < 0
 //   loss = sum_valid l_t / n_valid
 //   clipped (gradient zeroed, §2.1): A > 0 and r >= H, or A < 0 and r <= L
 //   g_t = dloss/dlogp_t = -w_t A_t r_t / n_valid on unclipped valid tokens
 //
-// Two grid-stride passes: the valid-token count (g needs it), then the fused
-// per-token pass writing g and the clip mask.  Block partials are reduced in
-// a fixed order by the last block, so the float64 loss is bit-reproducible for
-// a given T.
+// Two grid-stride passes: the valid-token count (g needs it; skipped without
+// a mask), then the fused per-token pass writing g and the clip mask, four
+// tokens per thread and step with 16-byte loads when the arrays allow.  Terms
+// are float32 (two roundings of the exact product); each thread sums its
+// terms with an error-free two-sum compensation (Knuth), so its partial is
+// the float32 sum to within one rounding; partials meet in float64 through a
+// fixed-order reduction by the last block, so the loss is bit-reproducible for
+// a given T and launch.
 #include "common.cuh"
 #include "internal.h"
 
@@ -19,6 +24,7 @@ namespace {
 __device__ uint32_t d_status;
 
 constexpr int kThreads = 256;
+constexpr int kCtasPerSm = 8;
 
 struct Partial {
   double loss;
@@ -34,76 +40,122 @@ struct Work {
 };
 
 int grid_of(int64_t T) {
-  int64_t want = (T + kThreads * 4 - 1) / (kThreads * 4);
-  const int64_t cap = static_cast<int64_t>(sm_count()) * 4;
+  const int64_t want = (T + kThreads * 16 - 1) / (kThreads * 16);
+  const int64_t cap = static_cast<int64_t>(sm_count()) * kCtasPerSm;
   return static_cast<int>(want < 1 ? 1 : (want > cap ? cap : want));
+}
+
+// Number of non-zero bytes of a word.
+__device__ __forceinline__ uint32_t nonzero_bytes(uint32_t w) {
+  return __popc((((w & 0x7F7F7F7Fu) + 0x7F7F7F7Fu) | w) & 0x80808080u);
 }
 
 __global__ void __launch_bounds__(kThreads) count_valid_kernel(const uint8_t* __restrict__ mask,
                                                                int64_t T, Work* w) {
-  unsigned long long n = 0;
-  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < T;
-       t += (int64_t)gridDim.x * blockDim.x)
-    n += mask ? (mask[t] != 0) : 1;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) n += __shfl_xor_sync(0xffffffffu, n, o);
-  if ((threadIdx.x & 31) == 0 && n) atomicAdd(&w->n_valid, n);
+  const int64_t tid = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  uint32_t n = 0;
+  const bool vec = (reinterpret_cast<uintptr_t>(mask) & 15) == 0;
+  const int64_t T16 = vec ? T / 16 : 0;
+  for (int64_t i = tid; i < T16; i += stride) {
+    const uint4 v = __ldg(reinterpret_cast<const uint4*>(mask) + i);
+    n += nonzero_bytes(v.x) + nonzero_bytes(v.y) + nonzero_bytes(v.z) + nonzero_bytes(v.w);
+  }
+  for (int64_t t = T16 * 16 + tid; t < T; t += stride) n += mask[t] != 0;
+  const uint32_t s = __reduce_add_sync(0xffffffffu, n);
+  if ((threadIdx.x & 31) == 0 && s) atomicAdd(&w->n_valid, static_cast<unsigned long long>(s));
 }
 
-template <typename T>
-__device__ __forceinline__ T block_sum(T v, T* sh) {
+// Fixed-order sum over the block; thread 0 gets the result.
+template <typename V>
+__device__ __forceinline__ V block_sum(V v, V* sh) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   if (lane == 0) sh[wid] = v;
   __syncthreads();
-  T r = 0;
+  V r = 0;
   if (threadIdx.x == 0)
-    for (int i = 0; i < kThreads / 32; ++i) r += sh[i];  // fixed order
+    for (int i = 0; i < kThreads / 32; ++i) r += sh[i];
   __syncthreads();
   return r;
+}
+
+struct Acc {
+  float s = 0.f, c = 0.f;  // compensated float32 sum: value s + c
+  uint32_t n_pos = 0, n_neg = 0, c_pos = 0, c_neg = 0;
+  // Knuth's two-sum: s + x = t + e exactly.
+  __device__ __forceinline__ void add(float x) {
+    const float t = s + x;
+    const float z = t - s;
+    c += (s - (t - z)) + (x - z);
+    s = t;
+  }
+};
+
+struct Bounds {
+  float lo, hi, inv_n;
+};
+
+// One token: its term, its gradient and clip-mask byte; counts into `a`.
+__device__ __forceinline__ float token(float rt, float at, bool valid, float wt, const Bounds& b,
+                                       Acc& a, float& g, uint32_t& cm) {
+  const bool up = valid && at > 0.f && rt >= b.hi;
+  const bool dn = valid && at < 0.f && rt <= b.lo;
+  const float m = at >= 0.f ? fminf(rt, b.hi) : fmaxf(rt, b.lo);
+  a.n_pos += valid && at > 0.f;
+  a.n_neg += valid && at < 0.f;
+  a.c_pos += up;
+  a.c_neg += dn;
+  g = (valid && !(up || dn)) ? -(wt * at) * rt * b.inv_n : 0.f;
+  cm = (up ? FP8RL_CLIP_HI : 0u) | (dn ? FP8RL_CLIP_LO : 0u);
+  return valid ? -(wt * (at * m)) : 0.f;
 }
 
 __global__ void __launch_bounds__(kThreads) surrogate_kernel(
     const float* __restrict__ r, const float* __restrict__ adv, const uint8_t* __restrict__ mask,
     const float* __restrict__ wts, int64_t T, float lo_arg, float hi_arg,
     const float* __restrict__ bounds, float* __restrict__ grad, uint8_t* __restrict__ clip_mask,
-    fp8rl_clip_stats* __restrict__ stats, Work* w) {
+    fp8rl_clip_stats* __restrict__ stats, Work* w, bool vec) {
   __shared__ double sh_d[kThreads / 32];
   __shared__ unsigned long long sh_u[kThreads / 32];
   __shared__ bool last;
-  const float lo = bounds ? bounds[0] : lo_arg;
-  const float hi = bounds ? bounds[1] : hi_arg;
-  const unsigned long long n_valid = w->n_valid;
-  const float inv_n = n_valid ? 1.0f / static_cast<float>(n_valid) : 0.f;
-  double loss = 0.0;
-  unsigned long long n_pos = 0, n_neg = 0, c_pos = 0, c_neg = 0;
-  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < T;
-       t += (int64_t)gridDim.x * blockDim.x) {
-    const bool valid = mask ? mask[t] != 0 : true;
-    const float rt = r[t], at = adv[t];
-    const float wt = wts ? wts[t] : 1.f;
-    const bool up = valid && at > 0.f && rt >= hi;
-    const bool dn = valid && at < 0.f && rt <= lo;
-    float g = 0.f;
-    if (valid) {
-      const double rd = rt, ad = at;
-      const double cl = fmin(fmax(rd, static_cast<double>(lo)), static_cast<double>(hi));
-      loss += -static_cast<double>(wt) * fmin(rd * ad, cl * ad);
-      n_pos += at > 0.f;
-      n_neg += at < 0.f;
-      c_pos += up;
-      c_neg += dn;
-      if (!(up || dn)) g = -(wt * at) * rt * inv_n;
-    }
-    if (grad) grad[t] = g;
-    if (clip_mask) clip_mask[t] = static_cast<uint8_t>((up ? FP8RL_CLIP_HI : 0) | (dn ? FP8RL_CLIP_LO : 0));
+  Bounds b;
+  b.lo = bounds ? bounds[0] : lo_arg;
+  b.hi = bounds ? bounds[1] : hi_arg;
+  const unsigned long long n_valid = mask ? w->n_valid : static_cast<unsigned long long>(T);
+  b.inv_n = n_valid ? 1.0f / static_cast<float>(n_valid) : 0.f;
+  Acc a;
+  const int64_t tid = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const int64_t T4 = vec ? T / 4 : 0;
+  for (int64_t i = tid; i < T4; i += stride) {
+    const float4 rv = __ldg(reinterpret_cast<const float4*>(r) + i);
+    const float4 av = __ldg(reinterpret_cast<const float4*>(adv) + i);
+    const float4 wv = wts ? __ldg(reinterpret_cast<const float4*>(wts) + i) : make_float4(1.f, 1.f, 1.f, 1.f);
+    const uint32_t mv = mask ? __ldg(reinterpret_cast<const uint32_t*>(mask) + i) : 0x01010101u;
+    float4 gv;
+    uint32_t c0, c1, c2, c3;
+    const float l0 = token(rv.x, av.x, (mv & 0xFFu) != 0, wv.x, b, a, gv.x, c0);
+    const float l1 = token(rv.y, av.y, (mv & 0xFF00u) != 0, wv.y, b, a, gv.y, c1);
+    const float l2 = token(rv.z, av.z, (mv & 0xFF0000u) != 0, wv.z, b, a, gv.z, c2);
+    const float l3 = token(rv.w, av.w, (mv & 0xFF000000u) != 0, wv.w, b, a, gv.w, c3);
+    a.add((l0 + l1) + (l2 + l3));
+    if (grad) reinterpret_cast<float4*>(grad)[i] = gv;
+    if (clip_mask) reinterpret_cast<uint32_t*>(clip_mask)[i] = c0 | (c1 << 8) | (c2 << 16) | (c3 << 24);
   }
-  loss = block_sum(loss, sh_d);
-  n_pos = block_sum(n_pos, sh_u);
-  n_neg = block_sum(n_neg, sh_u);
-  c_pos = block_sum(c_pos, sh_u);
-  c_neg = block_sum(c_neg, sh_u);
+  for (int64_t t = T4 * 4 + tid; t < T; t += stride) {
+    float g;
+    uint32_t cm;
+    a.add(token(r[t], adv[t], mask ? mask[t] != 0 : true, wts ? wts[t] : 1.f, b, a, g, cm));
+    if (grad) grad[t] = g;
+    if (clip_mask) clip_mask[t] = static_cast<uint8_t>(cm);
+  }
+  const double loss = block_sum(static_cast<double>(a.s) + static_cast<double>(a.c), sh_d);
+  const unsigned long long n_pos = block_sum<unsigned long long>(a.n_pos, sh_u);
+  const unsigned long long n_neg = block_sum<unsigned long long>(a.n_neg, sh_u);
+  const unsigned long long c_pos = block_sum<unsigned long long>(a.c_pos, sh_u);
+  const unsigned long long c_neg = block_sum<unsigned long long>(a.c_neg, sh_u);
   if (threadIdx.x == 0) {
     Partial& p = w->part[blockIdx.x];
     p.loss = loss;
@@ -115,18 +167,26 @@ __global__ void __launch_bounds__(kThreads) surrogate_kernel(
     last = atomicAdd(&w->ticket, 1u) == gridDim.x - 1;
   }
   __syncthreads();
-  if (last && threadIdx.x == 0) {
-    __threadfence();
-    double L = 0.0;
-    unsigned long long np = 0, nn = 0, cp = 0, cn = 0;
-    for (unsigned b = 0; b < gridDim.x; ++b) {  // fixed order
-      const volatile Partial& p = w->part[b];
-      L += p.loss;
-      np += p.n_pos;
-      nn += p.n_neg;
-      cp += p.c_pos;
-      cn += p.c_neg;
-    }
+  if (!last) return;
+  // The last block reduces the partials: thread i takes partials i, i + 256,
+  // ... in order, then the fixed-order block sum.
+  __threadfence();
+  double L = 0.0;
+  unsigned long long np = 0, nn = 0, cp = 0, cn = 0;
+  for (unsigned k = threadIdx.x; k < gridDim.x; k += kThreads) {
+    const volatile Partial& p = w->part[k];
+    L += p.loss;
+    np += p.n_pos;
+    nn += p.n_neg;
+    cp += p.c_pos;
+    cn += p.c_neg;
+  }
+  L = block_sum(L, sh_d);
+  np = block_sum(np, sh_u);
+  nn = block_sum(nn, sh_u);
+  cp = block_sum(cp, sh_u);
+  cn = block_sum(cn, sh_u);
+  if (threadIdx.x == 0) {
     fp8rl_clip_stats s;
     s.loss_sum = L;
     s.loss = n_valid ? L / static_cast<double>(n_valid) : 0.0;
@@ -135,13 +195,15 @@ __global__ void __launch_bounds__(kThreads) surrogate_kernel(
     s.n_neg = static_cast<int64_t>(nn);
     s.clipped_pos = static_cast<int64_t>(cp);
     s.clipped_neg = static_cast<int64_t>(cn);
-    s.lo = lo;
-    s.hi = hi;
+    s.lo = b.lo;
+    s.hi = b.hi;
     s.flags = n_valid ? 0 : 1;
     s.reserved = 0;
     *stats = s;
   }
 }
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
 
 }  // namespace
 
@@ -157,9 +219,11 @@ cudaError_t launch_surrogate(const float* r, const float* adv, const uint8_t* ma
   cudaError_t e = cudaMemsetAsync(work, 0, sizeof(Work), s);
   if (e != cudaSuccess) return e;
   const int grid = grid_of(T);
-  count_valid_kernel<<<grid, kThreads, 0, s>>>(mask, T, work);
+  if (mask) count_valid_kernel<<<grid, kThreads, 0, s>>>(mask, T, work);
+  const bool vec = aligned(r, 16) && aligned(adv, 16) && aligned(w, 16) && aligned(grad, 16) &&
+                   aligned(mask, 4) && aligned(clip_mask, 4);
   surrogate_kernel<<<grid, kThreads, 0, s>>>(r, adv, mask, w, T, lo, hi, bounds, grad, clip_mask,
-                                              stats, work);
+                                              stats, work, vec);
   return cudaGetLastError();
 }
 
