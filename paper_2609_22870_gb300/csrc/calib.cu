@@ -48,7 +48,7 @@ enum Stage : int {
 struct State {
   // accumulated by passes (zeroed before the first pass)
   unsigned long long n_neg, n_pos, k_bf16, k_fp8;
-  unsigned long long emax_bits;
+  unsigned long long emax_bits;  // frexp exponent of max|e| plus kEBias (0 = no term)
   unsigned long long s_pos_bf, s_neg_bf, s_neg_fp, s_pos_fp;  // int64 two's complement
   unsigned int bad;
   unsigned int nb_below1;  // 1 + max{key < u} (0 = none)
@@ -96,10 +96,94 @@ __device__ __forceinline__ void flag(uint32_t bits) { atomicOr(&d_status, bits);
 
 __device__ __forceinline__ unsigned key_of(float r) { return __float_as_uint(r) & 0x7FFFFFFFu; }
 
-// q_t = RNE(((coef r) A) 2^s) -- float64 product, exact scaling, RNE to int64.
+// ---- Eq. 5 terms in integer arithmetic (no float64 instruction per token).
+// e = fl64(fl64(c r) a): c r is exact in float64 (48-bit significand); the
+// product with a has up to 72 bits and the float64 multiply rounds it to 53,
+// to nearest, ties to even.  Both roundings (to 53 bits, then to an integer
+// at scale 2^s) are carried out on the exact integer significands.
+constexpr int kEBias = 2048;  // exponents of max|e| are stored biased (0 = no term)
+
+// |x| = m 2^e with an integer significand m < 2^24.
+__device__ __forceinline__ void split(float x, unsigned& m, int& e) {
+  const unsigned b = __float_as_uint(x) & 0x7FFFFFFFu;
+  const unsigned ex = b >> 23, fx = b & 0x7FFFFFu;
+  if (ex == 0) {
+    m = fx;
+    e = -149;
+  } else {
+    m = fx | 0x800000u;
+    e = static_cast<int>(ex) - 150;
+  }
+}
+
+// |fl64(fl64(c r) a)| = m 2^e with m < 2^53 (m = 0 for a zero product).
+__device__ __forceinline__ void term53(float c, float r, float a, unsigned long long& m53, int& e53) {
+  unsigned mc, mr, ma;
+  int ec, er, ea;
+  split(c, mc, ec);
+  split(r, mr, er);
+  split(a, ma, ea);
+  const unsigned long long p = static_cast<unsigned long long>(mc) * mr;  // < 2^48
+  const unsigned long long lo = p * ma;
+  const unsigned long long hi = __umul64hi(p, static_cast<unsigned long long>(ma));  // < 2^8
+  int e = ec + er + ea;
+  if ((lo | hi) == 0) {
+    m53 = 0;
+    e53 = 0;
+    return;
+  }
+  const int len = hi ? 128 - __clzll(static_cast<long long>(hi)) : 64 - __clzll(static_cast<long long>(lo));
+  if (len <= 53) {
+    m53 = lo;
+    e53 = e;
+    return;
+  }
+  const int d = len - 53;  // 1 .. 19
+  unsigned long long m = (hi << (64 - d)) | (lo >> d);
+  const unsigned long long rem = lo & ((1ull << d) - 1);
+  const unsigned long long half = 1ull << (d - 1);
+  if (rem > half || (rem == half && (m & 1))) ++m;
+  e += d;
+  if (m >> 53) {
+    m >>= 1;
+    ++e;
+  }
+  m53 = m;
+  e53 = e;
+}
+
+// frexp exponent E of |fl64(fl64(c r) a)| (value in [2^(E-1), 2^E)) plus
+// kEBias; 0 for a zero product.
+__device__ __forceinline__ unsigned term_exponent(float c, float r, float a) {
+  unsigned long long m;
+  int e;
+  term53(c, r, a, m, e);
+  if (m == 0) return 0;
+  return static_cast<unsigned>(64 - __clzll(static_cast<long long>(m)) + e + kEBias);
+}
+
+// q_t = RNE(fl64(fl64(c r) a) 2^s) as int64.
 __device__ __forceinline__ long long fixed_term(float c, float r, float a, int s) {
-  const double e = (static_cast<double>(c) * static_cast<double>(r)) * static_cast<double>(a);
-  return __double2ll_rn(ldexp(e, s));
+  unsigned long long m;
+  int e;
+  term53(c, r, a, m, e);
+  if (m == 0) return 0;
+  const int t = e + s;
+  unsigned long long q;
+  if (t >= 0) {
+    q = m << (t < 63 ? t : 63);
+  } else {
+    const int d = -t;
+    if (d > 54) {
+      q = 0;
+    } else {
+      q = m >> d;
+      const unsigned long long rem = m & ((1ull << d) - 1);
+      const unsigned long long half = 1ull << (d - 1);
+      if (rem > half || (rem == half && (q & 1))) ++q;
+    }
+  }
+  return a < 0.f ? -static_cast<long long>(q) : static_cast<long long>(q);
 }
 
 __device__ __forceinline__ bool digit_match(unsigned key, int digit, unsigned prefix) {
@@ -119,13 +203,13 @@ __device__ __forceinline__ float cand_at(double x0, double step, int i) {
   return static_cast<float>(x0 + static_cast<double>(i) * step);
 }
 
-// First candidate index i with r <= cand(i) (strict=false) or r < cand(i)
+// First candidate index i with r <= cand[i] (strict=false) or r < cand[i]
 // (strict=true); n if none.  Candidates ascend.
-__device__ __forceinline__ int first_cand(double x0, double step, int n, float r, bool strict) {
+__device__ __forceinline__ int first_cand(const float* cand, int n, float r, bool strict) {
   int lo = 0, hi = n;
   while (lo < hi) {
     const int mid = (lo + hi) >> 1;
-    const float c = cand_at(x0, step, mid);
+    const float c = cand[mid];
     const bool ok = strict ? (r < c) : (r <= c);
     if (ok) hi = mid; else lo = mid + 1;
   }
@@ -143,6 +227,7 @@ __device__ __forceinline__ T warp_sum(T v) {
 __global__ void __launch_bounds__(256) pass_kernel(Args a, int stage) {
   __shared__ unsigned long long sh_cnt[kBuckets];
   __shared__ long long sh_w[kBuckets];
+  __shared__ float sh_cand[kBuckets];  // GRID: the stage's candidate thresholds
   State* st = a.st;
   if ((stage == kH1 || stage == kH2 || stage == kHNb) && !st->h_active) return;
   const bool grid_mode = a.grid_mode != 0;
@@ -153,6 +238,11 @@ __global__ void __launch_bounds__(256) pass_kernel(Args a, int stage) {
     for (int i = threadIdx.x; i < kBuckets; i += blockDim.x) {
       sh_cnt[i] = 0;
       sh_w[i] = 0;
+      if (grid_mode) {
+        const bool lower = stage == kPrep;
+        const int n = lower ? a.n_lcand : a.n_hcand;
+        sh_cand[i] = i < n ? cand_at(lower ? a.lo_grid0 : a.hi_grid0, a.step, i) : 0.f;
+      }
     }
     __syncthreads();
   }
@@ -167,7 +257,7 @@ __global__ void __launch_bounds__(256) pass_kernel(Args a, int stage) {
 
   unsigned long long n_neg = 0, n_pos = 0, k_bf = 0, k_fp = 0;
   long long s_pos_bf = 0, s_neg_bf = 0, s_neg_fp = 0, s_pos_fp = 0;
-  double emax = 0.0;
+  unsigned emax = 0;
   unsigned bad = 0;
   unsigned nb_below1 = 0, nb_above = kNone, nb_m = kNone, nb_M1 = 0;
 
@@ -188,14 +278,10 @@ __global__ void __launch_bounds__(256) pass_kernel(Args a, int stage) {
         if (rb <= a.c_lo) ++k_bf;
       }
       if (pos) ++n_pos;
-      if (neg || pos) {
-        const double eb = (static_cast<double>(c) * rb) * static_cast<double>(A);
-        const double ef = (static_cast<double>(c) * rf) * static_cast<double>(A);
-        emax = fmax(emax, fmax(fabs(eb), fabs(ef)));
-      }
+      if (neg || pos) emax = max(emax, max(term_exponent(c, rb, A), term_exponent(c, rf, A)));
       if (neg) {
         if (grid_mode) {
-          atomicAdd(&sh_cnt[first_cand(a.lo_grid0, a.step, a.n_lcand, rf, false)], 1ull);
+          atomicAdd(&sh_cnt[first_cand(sh_cand, a.n_lcand, rf, false)], 1ull);
         } else {
           const unsigned d = digit_of(key_of(rf), 0);
           atomicAdd(&sh_cnt[d], 1ull);
@@ -216,7 +302,7 @@ __global__ void __launch_bounds__(256) pass_kernel(Args a, int stage) {
         if (neg && rf > lo_star) s_neg_fp += qf;
         if (neg && rf <= lo_star) ++k_fp;
         if (pos) {
-          const int j = first_cand(a.hi_grid0, a.step, a.n_hcand, rf, true);
+          const int j = first_cand(sh_cand, a.n_hcand, rf, true);
           atomicAdd(reinterpret_cast<unsigned long long*>(&sh_w[j]),
                     static_cast<unsigned long long>(qf));
           atomicAdd(&sh_cnt[j], 1ull);
@@ -284,8 +370,7 @@ __global__ void __launch_bounds__(256) pass_kernel(Args a, int stage) {
   s_neg_bf = warp_sum(s_neg_bf);
   s_neg_fp = warp_sum(s_neg_fp);
   s_pos_fp = warp_sum(s_pos_fp);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) emax = fmax(emax, __shfl_xor_sync(0xffffffffu, emax, o));
+  emax = __reduce_max_sync(0xffffffffu, emax);
   bad = __reduce_or_sync(0xffffffffu, bad);
   nb_below1 = __reduce_max_sync(0xffffffffu, nb_below1);
   nb_above = __reduce_min_sync(0xffffffffu, nb_above);
@@ -300,7 +385,7 @@ __global__ void __launch_bounds__(256) pass_kernel(Args a, int stage) {
     if (s_neg_bf) atomicAdd(&st->s_neg_bf, static_cast<unsigned long long>(s_neg_bf));
     if (s_neg_fp) atomicAdd(&st->s_neg_fp, static_cast<unsigned long long>(s_neg_fp));
     if (s_pos_fp) atomicAdd(&st->s_pos_fp, static_cast<unsigned long long>(s_pos_fp));
-    if (emax > 0.0) atomicMax(&st->emax_bits, static_cast<unsigned long long>(__double_as_longlong(emax)));
+    if (emax) atomicMax(&st->emax_bits, static_cast<unsigned long long>(emax));
     if (bad) {
       atomicOr(&st->bad, 1u);
       flag(kErrDevice);
@@ -519,12 +604,10 @@ __global__ void __launch_bounds__(1024) decide_kernel(Args a, int stage) {
   if (stage == kPrep) {
     if (tid == 0) {
       // fixed-point shift s = 62 - E - B: max|e| < 2^E, 2^B >= signed tokens
-      const double emax = __longlong_as_double(static_cast<long long>(st->emax_bits));
       const unsigned long long nt = st->n_neg + st->n_pos;
       int s = 0;
-      if (nt > 0 && emax > 0.0) {
-        int E;
-        frexp(emax, &E);
+      if (nt > 0 && st->emax_bits > 0) {
+        const int E = static_cast<int>(st->emax_bits) - kEBias;
         const int B = nt > 1 ? 64 - __clzll(static_cast<long long>(nt - 1)) : 0;
         s = 62 - E - B;
       }
