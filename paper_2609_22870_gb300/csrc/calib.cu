@@ -68,6 +68,7 @@ struct State {
   float lo_star, hi_star;
   int flags;
   int h_active;  // stage 2 runs (not degenerate)
+  int p_known;   // P(H*) = s_pos_fp already known: the last pass is skipped
   int pad1;
   // histograms
   unsigned long long h_cnt[kBuckets];
@@ -198,6 +199,32 @@ __device__ __forceinline__ unsigned digit_of(unsigned key, int digit) {
   return key & 0x3FFu;
 }
 
+// frexp exponent of fl32(fl32(|c r|) |a|) plus kEBias, or -1 when that
+// product or c r is not a normal float32 (zero, subnormal, overflow).  For a normal
+// product the exact |fl64(fl64(c r) a)| lies within a factor 1 +- 2^-22 of
+// it, so its exponent differs by at most one.
+__device__ __forceinline__ int approx_exponent(float c, float r, float a) {
+  const float cr = fabsf(c * r);
+  const unsigned ecr = __float_as_uint(cr) >> 23;
+  if (ecr == 0 || ecr >= 255) return -1;  // c r itself must be normal
+  const float p = cr * fabsf(a);
+  const unsigned ex = __float_as_uint(p) >> 23;
+  if (ex == 0 || ex >= 255) return -1;
+  return static_cast<int>(ex) - 126 + kEBias;
+}
+
+// q = RNE(fl64(fl64(c r) a) 2^s) != 0, decided from the float32 product when
+// it is clearly above 1/2 or below 1/4 after scaling, exactly otherwise.
+__device__ __forceinline__ bool fixed_nonzero(float c, float r, float a, int s) {
+  const int ea = approx_exponent(c, r, a);
+  if (ea >= 0) {
+    const int e = ea - kEBias + s;  // product 2^s in [2^(e-1), 2^e)
+    if (e - 1 >= 1) return true;    // >= 2
+    if (e <= -2) return false;      // < 1/4
+  }
+  return fixed_term(c, r, a, s) != 0;
+}
+
 // Candidate i of an Algorithm 1 grid, fl32(x0 + i * step) in float64.
 __device__ __forceinline__ float cand_at(double x0, double step, int i) {
   return static_cast<float>(x0 + static_cast<double>(i) * step);
@@ -224,20 +251,180 @@ __device__ __forceinline__ T warp_sum(T v) {
 }
 
 // ------------------------------------------------------------------ passes
+// Scalar results a thread accumulates over its tokens.
+struct PassAcc {
+  unsigned long long n_neg, n_pos, k_bf, k_fp;
+  long long s_pos_bf, s_neg_bf, s_neg_fp, s_pos_fp;
+  unsigned emax, bad, nb_below1, nb_above, nb_m, nb_M1;
+};
+
+// Constants of one pass.
+struct PassCtx {
+  int stage, digit, shift;
+  bool grid_mode;
+  float lo_star, hi_star;
+  unsigned prefix, u, key_lm, key_lM, key_hm, key_hM;
+};
+
+// One token of a pass: updates the thread's scalars and returns the
+// histogram bin the token adds `w` to (-1: none).
+__device__ __forceinline__ int pass_token(const Args& a, const PassCtx& x, const float* sh_cand,
+                                          bool valid, float A, float rf, float rb, float c,
+                                          PassAcc& acc, long long& w) {
+  w = 0;
+  const bool neg = valid && A < 0.f, pos = valid && A > 0.f;
+  if (x.stage == kPrep) {
+    if (!(isfinite(A) && isfinite(rf) && isfinite(rb) && isfinite(c)) || rf < 0.f || rb < 0.f ||
+        c < 0.f)
+      acc.bad = 1;
+    if (neg) {
+      ++acc.n_neg;
+      if (rb <= a.c_lo) ++acc.k_bf;
+    }
+    if (pos) ++acc.n_pos;
+    if (neg || pos) {
+      // the exact exponent only where it can raise the running maximum
+      const int eb = approx_exponent(c, rb, A), ef = approx_exponent(c, rf, A);
+      if (eb < 0 || eb + 1 > static_cast<int>(acc.emax)) acc.emax = max(acc.emax, term_exponent(c, rb, A));
+      if (ef < 0 || ef + 1 > static_cast<int>(acc.emax)) acc.emax = max(acc.emax, term_exponent(c, rf, A));
+    }
+    if (!neg) return -1;
+    w = 1;
+    return x.grid_mode ? first_cand(sh_cand, a.n_lcand, rf, false) : static_cast<int>(digit_of(key_of(rf), 0));
+  }
+  if (x.stage == kSums) {
+    if (!(neg || pos)) return -1;
+    const long long qb = fixed_term(c, rb, A, x.shift);
+    if (pos && rb < a.c_hi) acc.s_pos_bf += qb;
+    if (neg && rb > a.c_lo) acc.s_neg_bf += qb;
+    if (x.grid_mode) {
+      const long long qf = fixed_term(c, rf, A, x.shift);
+      if (neg && rf > x.lo_star) acc.s_neg_fp += qf;
+      if (neg && rf <= x.lo_star) ++acc.k_fp;
+      if (!pos) return -1;
+      w = qf;
+      return first_cand(sh_cand, a.n_hcand, rf, true);
+    }
+    if (!neg) return -1;
+    const unsigned key = key_of(rf);
+    if (!digit_match(key, 1, x.prefix)) return -1;
+    w = 1;
+    return static_cast<int>(digit_of(key, 1));
+  }
+  if (x.stage == kL2 || x.stage == kLNb) {
+    if (!neg) return -1;
+    const unsigned key = key_of(rf);
+    if (x.stage == kL2) {
+      if (!digit_match(key, 2, x.prefix)) return -1;
+      w = 1;
+      return static_cast<int>(digit_of(key, 2));
+    }
+    if (key < x.u) acc.nb_below1 = max(acc.nb_below1, key + 1);
+    if (key > x.u) acc.nb_above = min(acc.nb_above, key);
+    if (key > x.key_lm) acc.nb_m = min(acc.nb_m, key);
+    if (key <= x.key_lM) acc.nb_M1 = max(acc.nb_M1, key + 1);
+    return -1;
+  }
+  // H stages: Pos set, weights q_fp8.  kH0 needs q_fp8 for both signs: one
+  // evaluation for every signed token keeps the warp on one path.
+  if (x.stage == kH0) {
+    if (!(neg || pos)) return -1;
+    const long long qf = fixed_term(c, rf, A, x.shift);
+    if (neg) {
+      if (rf > x.lo_star) acc.s_neg_fp += qf;
+      else ++acc.k_fp;
+      return -1;
+    }
+    w = qf;
+    return static_cast<int>(digit_of(key_of(rf), 0));
+  }
+  if (!pos) return -1;
+  const unsigned key = key_of(rf);
+  if (x.stage == kPFin) {
+    if (rf < x.hi_star) acc.s_pos_fp += fixed_term(c, rf, A, x.shift);
+    return -1;
+  }
+  if (x.stage == kHNb) {
+    if (fixed_nonzero(c, rf, A, x.shift)) {
+      if (key < x.u) acc.nb_below1 = max(acc.nb_below1, key + 1);
+      if (key > x.u) acc.nb_above = min(acc.nb_above, key);
+      if (key >= x.key_hm) acc.nb_m = min(acc.nb_m, key);
+      if (key < x.key_hM) acc.nb_M1 = max(acc.nb_M1, key + 1);
+    }
+    return -1;
+  }
+  if (!digit_match(key, x.digit, x.prefix)) return -1;
+  w = fixed_term(c, rf, A, x.shift);
+  return static_cast<int>(digit_of(key, x.digit));
+}
+
+// Block histogram in shared memory with native 32-bit atomics only: counts
+// as 32-bit words, 64-bit weights as low and high words, the carry out of the
+// low word taken from the value the atomic returns (exact modulo 2^64).
+struct ShHist {
+  unsigned cnt[kBuckets];
+  unsigned wlo[kBuckets];
+  unsigned whi[kBuckets];
+};
+
+__device__ __forceinline__ void sh_add(ShHist& h, int d, unsigned n, unsigned long long w) {
+  atomicAdd(&h.cnt[d], n);
+  const unsigned lo = static_cast<unsigned>(w), hi = static_cast<unsigned>(w >> 32);
+  const unsigned old = lo ? atomicAdd(&h.wlo[d], lo) : 0u;
+  const unsigned carry = (old + lo < old) ? 1u : 0u;
+  if (hi + carry) atomicAdd(&h.whi[d], hi + carry);
+}
+
+// Adds every lane's (bin d, weight w >= 0) to the block histogram with one
+// update per distinct bin of the warp: ratios crowd into few bins of a
+// leading digit.  Weights are summed in three 21-bit slices by 32-bit warp
+// reductions (32 slices cannot overflow).  Called by all 32 lanes together;
+// d < 0 adds nothing.
+template <bool COUNTS>
+__device__ __forceinline__ void hist_add_warp(ShHist& sh, int d, long long w) {
+  const int lane = threadIdx.x & 31;
+  unsigned pending = __ballot_sync(0xffffffffu, d >= 0);
+  while (pending) {
+    const int leader = __ffs(pending) - 1;
+    const int dl = __shfl_sync(0xffffffffu, d, leader);
+    const bool mine = d == dl;
+    const unsigned grp = __ballot_sync(0xffffffffu, mine);
+    unsigned long long sum = __popc(grp);
+    if (!COUNTS) {
+      const unsigned long long v = mine ? static_cast<unsigned long long>(w) : 0ull;
+      const unsigned s0 = __reduce_add_sync(0xffffffffu, static_cast<unsigned>(v & 0x1FFFFFu));
+      const unsigned s1 = __reduce_add_sync(0xffffffffu, static_cast<unsigned>((v >> 21) & 0x1FFFFFu));
+      const unsigned s2 = __reduce_add_sync(0xffffffffu, static_cast<unsigned>(v >> 42));
+      sum = static_cast<unsigned long long>(s0) + (static_cast<unsigned long long>(s1) << 21) +
+            (static_cast<unsigned long long>(s2) << 42);
+    }
+    if (lane == leader) sh_add(sh, dl, __popc(grp), sum);
+    pending &= ~grp;
+  }
+}
+
+// Per-lane update, for digits whose bins are spread out.
+__device__ __forceinline__ void hist_add_lane(ShHist& sh, int d, long long w) {
+  if (d >= 0) sh_add(sh, d, 1u, static_cast<unsigned long long>(w));
+}
+
+// Passes read G tokens per lane and step: 16-byte loads when G = 4.
+template <int G>
 __global__ void __launch_bounds__(256) pass_kernel(Args a, int stage) {
-  __shared__ unsigned long long sh_cnt[kBuckets];
-  __shared__ long long sh_w[kBuckets];
+  __shared__ ShHist sh;
   __shared__ float sh_cand[kBuckets];  // GRID: the stage's candidate thresholds
   State* st = a.st;
   if ((stage == kH1 || stage == kH2 || stage == kHNb) && !st->h_active) return;
+  if (stage == kPFin && st->p_known) return;
   const bool grid_mode = a.grid_mode != 0;
   const bool want_hist = grid_mode ? (stage == kPrep || stage == kSums)
                                    : (stage == kPrep || stage == kSums || stage == kL2 ||
                                       stage == kH0 || stage == kH1 || stage == kH2);
   if (want_hist) {
     for (int i = threadIdx.x; i < kBuckets; i += blockDim.x) {
-      sh_cnt[i] = 0;
-      sh_w[i] = 0;
+      sh.cnt[i] = 0;
+      sh.wlo[i] = 0;
+      sh.whi[i] = 0;
       if (grid_mode) {
         const bool lower = stage == kPrep;
         const int n = lower ? a.n_lcand : a.n_hcand;
@@ -255,113 +442,104 @@ __global__ void __launch_bounds__(256) pass_kernel(Args a, int stage) {
   const unsigned key_lm = key_of(a.lo_min), key_lM = key_of(a.lo_max);
   const unsigned key_hm = key_of(a.hi_min), key_hM = key_of(a.hi_max);
 
-  unsigned long long n_neg = 0, n_pos = 0, k_bf = 0, k_fp = 0;
-  long long s_pos_bf = 0, s_neg_bf = 0, s_neg_fp = 0, s_pos_fp = 0;
-  unsigned emax = 0;
-  unsigned bad = 0;
-  unsigned nb_below1 = 0, nb_above = kNone, nb_m = kNone, nb_M1 = 0;
-
-  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < a.T;
-       t += (int64_t)gridDim.x * blockDim.x) {
-    const bool valid = a.mask ? a.mask[t] != 0 : true;
-    const float A = a.adv[t];
-    const float rf = a.r_fp8[t];
-    const bool neg = valid && A < 0.f, pos = valid && A > 0.f;
-    if (stage == kPrep) {
-      const float rb = a.r_bf16[t];
-      const float c = a.coef ? a.coef[t] : 1.f;
-      if (!(isfinite(A) && isfinite(rf) && isfinite(rb) && isfinite(c)) || rf < 0.f || rb < 0.f ||
-          c < 0.f)
-        bad = 1;
-      if (neg) {
-        ++n_neg;
-        if (rb <= a.c_lo) ++k_bf;
-      }
-      if (pos) ++n_pos;
-      if (neg || pos) emax = max(emax, max(term_exponent(c, rb, A), term_exponent(c, rf, A)));
-      if (neg) {
-        if (grid_mode) {
-          atomicAdd(&sh_cnt[first_cand(sh_cand, a.n_lcand, rf, false)], 1ull);
-        } else {
-          const unsigned d = digit_of(key_of(rf), 0);
-          atomicAdd(&sh_cnt[d], 1ull);
-          atomicAdd(reinterpret_cast<unsigned long long*>(&sh_w[d]), 1ull);
-        }
-      }
-      continue;
+  PassCtx x;
+  x.stage = stage;
+  x.digit = digit;
+  x.shift = shift;
+  x.grid_mode = grid_mode;
+  x.lo_star = lo_star;
+  x.hi_star = hi_star;
+  x.prefix = prefix;
+  x.u = u;
+  x.key_lm = key_lm;
+  x.key_lM = key_lM;
+  x.key_hm = key_hm;
+  x.key_hM = key_hM;
+  PassAcc acc{0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, kNone, kNone, 0};
+  // histogram update: 0 none, 1 warp-aggregated counts, 2 warp-aggregated
+  // weights (leading digit, grid candidates), 3 per lane (later digits)
+  int hist_mode = 0;
+  if (want_hist) {
+    if (stage == kPrep) hist_mode = 1;
+    else if (stage == kH0 || (grid_mode && stage == kSums)) hist_mode = 2;
+    else hist_mode = 3;
+  }
+  const bool need_rb = stage == kPrep || stage == kSums;
+  const bool need_c = a.coef != nullptr && !(stage == kL2 || stage == kLNb);
+  const int lane = threadIdx.x & 31;
+  const int64_t ng = a.T / G;
+  const int64_t warp_id = (blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x) >> 5;
+  const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+  // warp-uniform steps: every lane runs every step (the histogram update is
+  // a warp collective); lanes past the end see invalid zero tokens
+  for (int64_t base = warp_id * 32; base < ng; base += nwarps * 32) {
+    const int64_t g = base + lane;
+    const bool in = g < ng;
+    float rf[G], A[G], rb[G], c[G];
+    bool valid[G];
+#pragma unroll
+    for (int j = 0; j < G; ++j) {
+      rf[j] = 0.f;
+      A[j] = 0.f;
+      rb[j] = 0.f;
+      c[j] = 1.f;
+      valid[j] = false;
     }
-    if (stage == kSums) {
-      if (!(neg || pos)) continue;
-      const float rb = a.r_bf16[t];
-      const float c = a.coef ? a.coef[t] : 1.f;
-      const long long qb = fixed_term(c, rb, A, shift);
-      if (pos && rb < a.c_hi) s_pos_bf += qb;
-      if (neg && rb > a.c_lo) s_neg_bf += qb;
-      if (grid_mode) {
-        const long long qf = fixed_term(c, rf, A, shift);
-        if (neg && rf > lo_star) s_neg_fp += qf;
-        if (neg && rf <= lo_star) ++k_fp;
-        if (pos) {
-          const int j = first_cand(sh_cand, a.n_hcand, rf, true);
-          atomicAdd(reinterpret_cast<unsigned long long*>(&sh_w[j]),
-                    static_cast<unsigned long long>(qf));
-          atomicAdd(&sh_cnt[j], 1ull);
+    if (in) {
+      if (G == 4) {
+        const float4 vf = __ldg(reinterpret_cast<const float4*>(a.r_fp8) + g);
+        const float4 va = __ldg(reinterpret_cast<const float4*>(a.adv) + g);
+        rf[0] = vf.x; rf[1] = vf.y; rf[2] = vf.z; rf[3] = vf.w;
+        A[0] = va.x; A[1] = va.y; A[2] = va.z; A[3] = va.w;
+        if (need_rb) {
+          const float4 vb = __ldg(reinterpret_cast<const float4*>(a.r_bf16) + g);
+          rb[0] = vb.x; rb[1] = vb.y; rb[2] = vb.z; rb[3] = vb.w;
         }
-      } else if (neg) {
-        const unsigned key = key_of(rf);
-        if (digit_match(key, 1, prefix)) {
-          const unsigned d = digit_of(key, 1);
-          atomicAdd(&sh_cnt[d], 1ull);
-          atomicAdd(reinterpret_cast<unsigned long long*>(&sh_w[d]), 1ull);
+        if (need_c) {
+          const float4 vc = __ldg(reinterpret_cast<const float4*>(a.coef) + g);
+          c[0] = vc.x; c[1] = vc.y; c[2] = vc.z; c[3] = vc.w;
         }
-      }
-      continue;
-    }
-    if (stage == kL2 || stage == kLNb) {
-      if (!neg) continue;
-      const unsigned key = key_of(rf);
-      if (stage == kL2) {
-        if (digit_match(key, 2, prefix)) {
-          const unsigned d = digit_of(key, 2);
-          atomicAdd(&sh_cnt[d], 1ull);
-          atomicAdd(reinterpret_cast<unsigned long long*>(&sh_w[d]), 1ull);
-        }
+        const uint32_t m = a.mask ? __ldg(reinterpret_cast<const uint32_t*>(a.mask) + g) : 0x01010101u;
+#pragma unroll
+        for (int j = 0; j < G; ++j) valid[j] = ((m >> (8 * j)) & 0xFFu) != 0;
       } else {
-        if (key < u) nb_below1 = max(nb_below1, key + 1);
-        if (key > u) nb_above = min(nb_above, key);
-        if (key > key_lm) nb_m = min(nb_m, key);
-        if (key <= key_lM) nb_M1 = max(nb_M1, key + 1);
+        rf[0] = a.r_fp8[g];
+        A[0] = a.adv[g];
+        if (need_rb) rb[0] = a.r_bf16[g];
+        if (need_c) c[0] = a.coef[g];
+        valid[0] = a.mask ? a.mask[g] != 0 : true;
       }
-      continue;
     }
-    // H stages: Pos set, weights q_fp8
-    if (stage == kH0 && neg) {
-      const float c = a.coef ? a.coef[t] : 1.f;
-      if (rf > lo_star) s_neg_fp += fixed_term(c, rf, A, shift);
-      else ++k_fp;
-    }
-    if (!pos) continue;
-    const float c = a.coef ? a.coef[t] : 1.f;
-    const long long qf = fixed_term(c, rf, A, shift);
-    const unsigned key = key_of(rf);
-    if (stage == kPFin) {
-      if (rf < hi_star) s_pos_fp += qf;
-    } else if (stage == kHNb) {
-      if (qf > 0) {
-        if (key < u) nb_below1 = max(nb_below1, key + 1);
-        if (key > u) nb_above = min(nb_above, key);
-        if (key >= key_hm) nb_m = min(nb_m, key);
-        if (key < key_hM) nb_M1 = max(nb_M1, key + 1);
-      }
-    } else if (digit_match(key, digit, prefix)) {
-      const unsigned d = digit_of(key, digit);
-      atomicAdd(&sh_cnt[d], 1ull);
-      atomicAdd(reinterpret_cast<unsigned long long*>(&sh_w[d]), static_cast<unsigned long long>(qf));
+#pragma unroll
+    for (int j = 0; j < G; ++j) {
+      long long w;
+      const int d = pass_token(a, x, sh_cand, valid[j], A[j], rf[j], rb[j], c[j], acc, w);
+      if (hist_mode == 1) hist_add_warp<true>(sh, d, w);
+      else if (hist_mode == 2) hist_add_warp<false>(sh, d, w);
+      else if (hist_mode == 3) hist_add_lane(sh, d, w);
     }
   }
+  if (G > 1 && blockIdx.x == 0 && threadIdx.x < 32) {  // the last T mod 4 tokens
+    const int64_t t = ng * G + lane;
+    const bool in = t < a.T;
+    const float rf = in ? a.r_fp8[t] : 0.f;
+    const float A = in ? a.adv[t] : 0.f;
+    const float rb = in && need_rb ? a.r_bf16[t] : 0.f;
+    const float c = in && need_c ? a.coef[t] : 1.f;
+    const bool valid = in && (a.mask ? a.mask[t] != 0 : true);
+    long long w;
+    const int d = pass_token(a, x, sh_cand, valid, A, rf, rb, c, acc, w);
+    if (hist_mode == 1) hist_add_warp<true>(sh, d, w);
+    else if (hist_mode == 2) hist_add_warp<false>(sh, d, w);
+    else if (hist_mode == 3) hist_add_lane(sh, d, w);
+  }
+  unsigned long long n_neg = acc.n_neg, n_pos = acc.n_pos, k_bf = acc.k_bf, k_fp = acc.k_fp;
+  long long s_pos_bf = acc.s_pos_bf, s_neg_bf = acc.s_neg_bf, s_neg_fp = acc.s_neg_fp,
+            s_pos_fp = acc.s_pos_fp;
+  unsigned emax = acc.emax, bad = acc.bad;
+  unsigned nb_below1 = acc.nb_below1, nb_above = acc.nb_above, nb_m = acc.nb_m, nb_M1 = acc.nb_M1;
 
   // ---- flush: warp-aggregated scalars, then the block histogram
-  const int lane = threadIdx.x & 31;
   n_neg = warp_sum(n_neg);
   n_pos = warp_sum(n_pos);
   k_bf = warp_sum(k_bf);
@@ -398,9 +576,9 @@ __global__ void __launch_bounds__(256) pass_kernel(Args a, int stage) {
   if (want_hist) {
     __syncthreads();
     for (int i = threadIdx.x; i < kBuckets; i += blockDim.x) {
-      if (sh_cnt[i]) {
-        atomicAdd(&st->h_cnt[i], sh_cnt[i]);
-        atomicAdd(&st->h_w[i], static_cast<unsigned long long>(sh_w[i]));
+      if (sh.cnt[i]) {
+        atomicAdd(&st->h_cnt[i], static_cast<unsigned long long>(sh.cnt[i]));
+        atomicAdd(&st->h_w[i], (static_cast<unsigned long long>(sh.whi[i]) << 32) | sh.wlo[i]);
       }
     }
   }
@@ -767,6 +945,17 @@ __global__ void __launch_bounds__(1024) decide_kernel(Args a, int stage) {
         }
       }
       st->hi_star = upper_from_interval(a, st, lo, hi);
+      if (st->found) {
+        // H* inside (z, u] or (u, w]: P(H*) is the select's p_lt or p_le
+        const float H = st->hi_star, fu = __uint_as_float(st->u_key);
+        if (H > fu && H <= w) {
+          st->s_pos_fp = static_cast<unsigned long long>(st->p_le);
+          st->p_known = 1;
+        } else if (H <= fu && H > z) {
+          st->s_pos_fp = static_cast<unsigned long long>(st->p_lt);
+          st->p_known = 1;
+        }
+      }
     }
     return;
   }
@@ -812,7 +1001,9 @@ cudaError_t launch_calibrate(const float* r_fp8, const float* r_bf16, const floa
 
   cudaError_t e = cudaMemsetAsync(ws, 0, sizeof(State), s);
   if (e != cudaSuccess) return e;
-  int64_t want = (T + 1023) / 1024;
+  auto al = [](const void* p, uintptr_t n) { return (reinterpret_cast<uintptr_t>(p) & (n - 1)) == 0; };
+  const bool vec = al(r_fp8, 16) && al(r_bf16, 16) && al(adv, 16) && al(coef, 16) && al(mask, 4);
+  int64_t want = (T + 4095) / 4096;
   const int64_t cap = static_cast<int64_t>(sm_count()) * 4;
   const int grid = static_cast<int>(want < 1 ? 1 : (want > cap ? cap : want));
   const int stages_exact[] = {kPrep, kSums, kL2, kLNb, kH0, kH1, kH2, kHNb, kPFin};
@@ -820,7 +1011,8 @@ cudaError_t launch_calibrate(const float* r_fp8, const float* r_bf16, const floa
   const int* stages = a.grid_mode ? stages_grid : stages_exact;
   const int n = a.grid_mode ? 3 : 9;
   for (int i = 0; i < n; ++i) {
-    pass_kernel<<<grid, 256, 0, s>>>(a, stages[i]);
+    if (vec) pass_kernel<4><<<grid, 256, 0, s>>>(a, stages[i]);
+    else pass_kernel<1><<<grid, 256, 0, s>>>(a, stages[i]);
     decide_kernel<<<1, 1024, 0, s>>>(a, stages[i]);
   }
   return cudaGetLastError();

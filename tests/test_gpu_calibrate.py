@@ -132,3 +132,16 @@ def test_calibrate_full_size(cuda_lib, name):
     for mode in MODES:
         _compare(_run(cuda_lib, r_fp, r_bf, adv, mask, coef, w.eps_low, w.eps_high, mode=mode),
                  _ref(r_fp, r_bf, adv, mask, coef, w.eps_low, w.eps_high, mode=mode))
+
+
+@pytest.mark.parametrize("mode", MODES)
+def test_calibrate_unaligned_inputs(cuda_lib, mode):
+    """Inputs that start 4 bytes (1 byte for the mask) past an allocation
+    boundary take the scalar-load passes; same result as the oracle."""
+    T = 3001
+    args = _inputs(T + 1, 77)
+    d = [None if t is None else t.cuda()[1:] for t in args]
+    buf = cuda_lib.calibrate_clip_bounds(*d, 0.2, 0.28, cuda_lib.calib_opts(mode=mode))
+    cuda_lib.check()
+    host = [None if t is None else t[1:] for t in args]
+    _compare(cuda_lib.read_calib_result(buf), _ref(*host, 0.2, 0.28, mode=mode))
