@@ -436,53 +436,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
 }
 
-// ------------------------------------------------------------------ combine
-__global__ void combine_kernel(const float2* __restrict__ partials, const float* __restrict__ zy,
-                               const int32_t* __restrict__ targets,
-                               const float* __restrict__ logp_old, float* __restrict__ logp,
-                               float* __restrict__ lse_out, float* __restrict__ ratio, int64_t M,
-                               int64_t N, int64_t n_chunks) {
-  const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (t >= M) return;
-  float m = -INFINITY, s = 0.f;
-  int64_t c = 0;
-  for (; c + 4 <= n_chunks; c += 4) {
-    float2 q[4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) q[u] = __ldg(partials + (c + u) * M + t);
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      if (q[u].x > m) {
-        s = s * exp2f((m - q[u].x) * kLog2e) + q[u].y;
-        m = q[u].x;
-      } else {
-        s += q[u].y * exp2f((q[u].x - m) * kLog2e);
-      }
-    }
-  }
-  for (; c < n_chunks; ++c) {
-    const float2 q = __ldg(partials + c * M + t);
-    if (q.x > m) {
-      s = s * exp2f((m - q.x) * kLog2e) + q.y;
-      m = q.x;
-    } else {
-      s += q.y * exp2f((q.x - m) * kLog2e);
-    }
-  }
-  const float l = m + logf(s);
-  const int32_t y = targets[t];
-  float lp;
-  if (y >= 0 && y < N) {
-    lp = zy[t] - l;
-  } else {
-    lp = NAN;
-    flag(kErrDevice);
-  }
-  logp[t] = lp;
-  if (lse_out) lse_out[t] = l;
-  if (ratio) ratio[t] = expf(lp - logp_old[t]);
-}
-
+// ------------------------------------------------------------------ ratios
 __global__ void ratios_kernel(const float* __restrict__ a, const float* __restrict__ b, int64_t T,
                               float* __restrict__ r) {
   for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < T;
@@ -638,15 +592,6 @@ cudaError_t launch_gemm_lse(const GemmArgs& a, cudaStream_t s) { return launch_g
 
 cudaError_t launch_gemm_dlogits(const GemmArgs& a, cudaStream_t s) {
   return launch_gemm<kEpiDlogits>(a, s);
-}
-
-cudaError_t launch_combine(const float2* partials, const float* zy, const int32_t* targets,
-                           const float* logp_old, float* logp, float* lse, float* ratio,
-                           int64_t M, int64_t N, cudaStream_t s) {
-  if (M == 0) return cudaSuccess;
-  combine_kernel<<<blocks_for(M, 256), 256, 0, s>>>(partials, zy, targets, logp_old, logp, lse,
-                                                    ratio, M, N, (N + CHUNK - 1) / CHUNK);
-  return cudaGetLastError();
 }
 
 cudaError_t launch_ratios(const float* lp_new, const float* lp_old, int64_t T, float* r,

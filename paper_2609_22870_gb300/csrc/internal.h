@@ -54,6 +54,7 @@ cudaError_t launch_gather_rows(const uint8_t* h_codes, const float* h_scales, in
                                float* g_lse, float* g_grad, cudaStream_t s);
 cudaError_t launch_wait_selftest(uint64_t limit_ns, cudaStream_t s);
 uint32_t gemm_status_take();
+uint32_t combine_status_take();
 
 // ---------------------------------------------------------------- calib.cu
 size_t calib_workspace_bytes(int64_t T);
