@@ -176,6 +176,27 @@ fp8rl_status fp8rl_token_logprobs_noalloc(const uint8_t* h_codes, const float* h
                                           const int32_t* targets, const float* logp_old,
                                           float* logp, float* lse, float* ratio, void* stream);
 
+/* The BF16 shadow pass of §4 / Algorithm 1: the reference ratios r_BF16 that
+ * Calibrated Clipping matches come from forward passes in BF16.  This scores
+ * the sampled tokens from the unquantised operands,
+ *   z[t][v] = sum_k h[t][k] W[v][k]   (BF16 x BF16 products, fp32 accumulation
+ *                                       on the tensor cores)
+ * with the same streaming logsumexp + target gather as fp8rl_token_logprobs
+ * (z is never stored), then logp, lse and ratio exactly as there.
+ *   h   bf16 [T][ld_h] row-major (first H of each row used), 16-byte aligned
+ *   W   bf16 [V][ld_w] row-major (the lm_head weight), 16-byte aligned
+ *   ld_h, ld_w  row strides in elements, multiples of 8, >= H
+ *   targets, logp_old, logp, lse, ratio  as for fp8rl_token_logprobs
+ * Requires T >= 1, V >= 1, H >= 64 and H % 64 == 0.  The workspace (sized by
+ * fp8rl_bf16_token_logprobs_workspace_size) holds the per-chunk partials. */
+size_t fp8rl_bf16_token_logprobs_workspace_size(int64_t T, int64_t H, int64_t V);
+
+fp8rl_status fp8rl_bf16_token_logprobs(const void* h, int64_t ld_h, const void* W, int64_t ld_w,
+                                       int64_t T, int64_t H, int64_t V,
+                                       const int32_t* targets, const float* logp_old,
+                                       float* logp, float* lse, float* ratio,
+                                       void* workspace, size_t workspace_bytes, void* stream);
+
 /* r_t = exp(logp_new_t - logp_old_t) (§2.1), float [T]. */
 fp8rl_status fp8rl_importance_ratios(const float* logp_new, const float* logp_old,
                                      int64_t T, float* ratio, void* stream);

@@ -19,6 +19,14 @@ the same granularity.
 
 dLoss/dlogits follows from the chain rule through log-softmax:
   dL/dz[t, v] = g_t * (1{v == y_t} - exp(z[t, v] - lse_t)),  g_t = dL/dlogp_t.
+
+The BF16 shadow pass (§4, Algorithm 1: the reference ratios r_BF16 come from
+forward passes in BF16, recomputed every few steps) scores the same tokens
+from the unquantised BF16 operands:
+
+  z[t, v]   = sum_k  h[t, k] * W[v, k]                        (bf16 values)
+
+again in float64, followed by the same log-softmax and gather.
 """
 
 import numpy as np
@@ -50,6 +58,24 @@ def log_softmax_gather(z, targets):
 def token_logprobs(h_codes, h_scales, w_codes, w_scales, gran, targets, rows=None):
     """Per-token log-prob (and lse) of the target under the FP8 lm_head."""
     z = logits(h_codes, h_scales, w_codes, w_scales, gran, rows)
+    y = np.asarray(targets)
+    if rows is not None:
+        y = y[np.asarray(rows)]
+    return log_softmax_gather(z, y)
+
+
+def bf16_logits(h, W, rows=None):
+    """z = h @ W^T in float64 from the bf16-valued operands (the BF16 shadow
+    pass of §4; no quantisation)."""
+    h = np.asarray(h, dtype=np.float64)
+    if rows is not None:
+        h = h[np.asarray(rows)]
+    return h @ np.asarray(W, dtype=np.float64).T
+
+
+def bf16_token_logprobs(h, W, targets, rows=None):
+    """Per-token (logp, lse) of the target under the BF16 lm_head (§4 reference pass)."""
+    z = bf16_logits(h, W, rows)
     y = np.asarray(targets)
     if rows is not None:
         y = y[np.asarray(rows)]

@@ -68,6 +68,9 @@ _SIGS = {
     "fp8rl_logit_partials": (_i, [_p, _p, _p, _p, _i, _i64, _i64, _i64, _p, _p, _sz, _p]),
     "fp8rl_combine_logprobs": (_i, [_i64, _i64, _i64, _i, _p, _p, _p, _p, _p, _p, _sz, _p]),
     "fp8rl_importance_ratios": (_i, [_p, _p, _i64, _p, _p]),
+    "fp8rl_bf16_token_logprobs_workspace_size": (_sz, [_i64, _i64, _i64]),
+    "fp8rl_bf16_token_logprobs": (_i, [_p, _i64, _p, _i64, _i64, _i64, _i64, _p, _p, _p, _p, _p, _p,
+                                       _sz, _p]),
     "fp8rl_token_logprobs_noalloc": (_i, [_p, _p, _p, _p, _i, _i64, _i64, _i64, _p, _p, _p, _p, _p, _p]),
     "fp8rl_default_calib_opts": (None, [ctypes.POINTER(CalibOpts)]),
     "fp8rl_calibrate_workspace_size": (_sz, [_i64]),
@@ -238,6 +241,38 @@ def combine_logprobs(T, H, V, gran, targets, workspace, logp_old=None, logp=None
     _ok(lib.fp8rl_combine_logprobs(T, H, V, gran, _ptr(targets), _ptr(logp_old), _ptr(logp),
                                    _ptr(lse), _ptr(ratio), _ptr(workspace), workspace.numel(),
                                    _stream(stream)), "fp8rl_combine_logprobs")
+
+
+def bf16_token_logprobs_workspace_size(T, H, V):
+    return int(lib.fp8rl_bf16_token_logprobs_workspace_size(T, H, V))
+
+
+def bf16_token_logprobs(h, W, targets, logp_old=None, want_lse=True, want_ratio=None,
+                        workspace=None, out=None, stream=None):
+    """fp8rl_bf16_token_logprobs: the BF16 shadow pass (unquantised bf16 h, W)
+    -> dict(logp, lse, ratio) of float32 [T] tensors."""
+    for name, x in (("h", h), ("W", W)):
+        if x.dim() != 2 or x.dtype != torch.bfloat16 or not x.is_cuda or x.stride(1) != 1:
+            raise ValueError(f"{name}: expected a 2-D CUDA bf16 tensor with unit column stride")
+    T, H = h.shape
+    V = W.shape[0]
+    if W.shape[1] != H:
+        raise ValueError("h and W disagree on the hidden size")
+    _dev(targets, torch.int32, "targets", T)
+    _dev(logp_old, torch.float32, "logp_old", T)
+    dev = h.device
+    want_ratio = logp_old is not None if want_ratio is None else want_ratio
+    o = out or {}
+    logp = o.get("logp", torch.empty(T, dtype=torch.float32, device=dev))
+    lse = o.get("lse", torch.empty(T, dtype=torch.float32, device=dev)) if want_lse else None
+    ratio = o.get("ratio", torch.empty(T, dtype=torch.float32, device=dev)) if want_ratio else None
+    if workspace is None:
+        workspace = _workspace(bf16_token_logprobs_workspace_size(T, H, V), dev)
+    _ok(lib.fp8rl_bf16_token_logprobs(_ptr(h), h.stride(0), _ptr(W), W.stride(0), T, H, V,
+                                      _ptr(targets), _ptr(logp_old), _ptr(logp), _ptr(lse),
+                                      _ptr(ratio), _ptr(workspace), workspace.numel(),
+                                      _stream(stream)), "fp8rl_bf16_token_logprobs")
+    return {"logp": logp, "lse": lse, "ratio": ratio}
 
 
 def importance_ratios(logp_new, logp_old, out=None, stream=None):

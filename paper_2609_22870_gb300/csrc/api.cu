@@ -201,6 +201,40 @@ fp8rl_status fp8rl_token_logprobs(const uint8_t* hc, const float* hs, const uint
   return fp8rl_combine_logprobs(T, H, V, g, targets, logp_old, logp, lse, ratio, ws, ws_bytes, stream);
 }
 
+// ------------------------------------------------------------------ BF16 shadow pass
+size_t fp8rl_bf16_token_logprobs_workspace_size(int64_t T, int64_t, int64_t V) {
+  if (T < 0 || V < 0) return 0;
+  return logprob_ws(T, V);
+}
+
+fp8rl_status fp8rl_bf16_token_logprobs(const void* h, int64_t ld_h, const void* w, int64_t ld_w,
+                                       int64_t T, int64_t H, int64_t V, const int32_t* targets,
+                                       const float* logp_old, float* logp, float* lse, float* ratio,
+                                       void* ws, size_t ws_bytes, void* stream) {
+  if (!h || !w || !targets || !logp || (ratio && !logp_old)) return FP8RL_EINVAL;
+  if (T < 1 || V < 1 || H < 64 || H % 64 != 0 || ld_h < H || ld_w < H) return FP8RL_ESHAPE;
+  if (T > 0x7FFFFFFF || V > 0x7FFFFFFF || H > 0x7FFFFFFF) return FP8RL_ESHAPE;
+  if (!aligned16(h) || !aligned16(w) || ld_h % 8 != 0 || ld_w % 8 != 0) return FP8RL_EALIGN;
+  if (!ws || ws_bytes < logprob_ws(T, V)) return FP8RL_EWORKSPACE;
+  GemmArgs a{};
+  a.a_codes = h;
+  a.b_codes = w;
+  a.gran = kGemmBf16;
+  a.M = T;
+  a.N = V;
+  a.K = H;
+  a.lda = ld_h;
+  a.ldb = ld_w;
+  a.targets = targets;
+  a.partials = static_cast<float2*>(ws);
+  a.zy = reinterpret_cast<float*>(static_cast<char*>(ws) + partials_bytes(T, V));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = launch_gemm_lse(a, s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  e = launch_combine(a.partials, a.zy, targets, logp_old, logp, lse, ratio, T, V, s);
+  return e == cudaSuccess ? FP8RL_OK : cuda_fail(e);
+}
+
 fp8rl_status fp8rl_importance_ratios(const float* lp_new, const float* lp_old, int64_t T,
                                      float* ratio, void* stream) {
   if (!lp_new || !lp_old || !ratio) return FP8RL_EINVAL;

@@ -19,7 +19,10 @@
 //               them.  One (max, sum) pair per token and 128-wide vocabulary
 //               chunk goes to the workspace; nothing of size T x V does.
 // Per-tensor and per-row scales factor out of the K sum, so the accumulator
-// runs over the whole K in TMEM and is scaled once.  Block scales (1x128 for h,
+// runs over the whole K in TMEM and is scaled once.  The BF16 shadow pass of §4
+// (reference log-probs from the unquantised operands) runs the same kernel with
+// tcgen05.mma kind::f16 on bf16 tiles (64 elements = 128 bytes per row and
+// stage, so the shared-memory layout is the FP8 one) and no scales.  Block scales (1x128 for h,
 // 128x128 for W) change every 128-wide K block: the MMA writes each K block's
 // partial product into one of the two TMEM buffers and the epilogue promotes
 // it, acc += S_h[t][kb] S_W[vb][kb] * partial, into registers while the MMA
@@ -58,7 +61,8 @@ constexpr size_t SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + SC_BYTES + 512;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr uint64_t kDrainNs = 1000000000ull;
 
-enum { kTensor = FP8RL_GRAN_TENSOR, kRow = FP8RL_GRAN_ROWWISE, kBlock = FP8RL_GRAN_BLOCK };
+enum { kTensor = FP8RL_GRAN_TENSOR, kRow = FP8RL_GRAN_ROWWISE, kBlock = FP8RL_GRAN_BLOCK, kBf16 = 3 };
+static_assert(kBf16 == kGemmBf16, "BF16 mode id shared with the host interface");
 enum { kEpiLse = 0, kEpiDlogits = 1 };
 
 struct Params {
@@ -210,8 +214,10 @@ __global__ void __launch_bounds__(THREADS, 1)
         if (!ok) break;
         if (elect_one()) {
           mbar_arrive_expect_tx(smem_u32(&full[stage]), STAGE_BYTES);
-          tma_load_2d(smem_u32(smA + stage * A_BYTES), &tmA, smem_u32(&full[stage]), kb * BK, m0);
-          tma_load_2d(smem_u32(smB + stage * B_BYTES), &tmB, smem_u32(&full[stage]), kb * BK, n0);
+          // K coordinate in elements: 128 E4M3 or 64 BF16 per 128-byte row
+          const int kx = kb * ((MODE == kBf16) ? BK / 2 : BK);
+          tma_load_2d(smem_u32(smA + stage * A_BYTES), &tmA, smem_u32(&full[stage]), kx, m0);
+          tma_load_2d(smem_u32(smB + stage * B_BYTES), &tmB, smem_u32(&full[stage]), kx, n0);
         }
         __syncwarp();
         armed |= 1u << stage;
@@ -271,7 +277,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     // tcgen05.mma / tcgen05.commit
     int stage = 0, ab = 0;
     uint32_t phase = 0, aphase = 0;
-    constexpr uint32_t idesc = idesc_e4m3_f32(BM, BN);
+    constexpr uint32_t idesc = (MODE == kBf16) ? idesc_bf16_f32(BM, BN) : idesc_e4m3_f32(BM, BN);
     bool ok = true;
     for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
       if (MODE != kBlock) {
@@ -293,8 +299,9 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
         for (int k = 0; k < BK / 32; ++k) {
           const uint32_t acc = (MODE == kBlock) ? (k > 0) : (kb > 0 || k > 0);
-          // +32 bytes along K inside the swizzled 128-byte row
-          mma_f8f6f4_elect(d, adesc + 2 * k, bdesc + 2 * k, idesc, acc);
+          // +32 bytes along K inside the swizzled 128-byte row (32 FP8 or 16 BF16 elements)
+          if (MODE == kBf16) mma_bf16_elect(d, adesc + 2 * k, bdesc + 2 * k, idesc, acc);
+          else mma_f8f6f4_elect(d, adesc + 2 * k, bdesc + 2 * k, idesc, acc);
         }
         mma_commit_elect(smem_u32(&empty[stage]));
         if (MODE == kBlock) {
@@ -397,7 +404,9 @@ __global__ void __launch_bounds__(THREADS, 1)
         if (!ok) break;
         tc_fence_after();
         const uint32_t taddr = tmem_base + t_row + static_cast<uint32_t>(ab * BN + half * CHUNK);
-        const float sa = (MODE == kTensor) ? __ldg(p.a_scales) : (row_ok ? __ldg(p.a_scales + row) : 0.f);
+        const float sa = (MODE == kBf16) ? 1.f
+                         : (MODE == kTensor) ? __ldg(p.a_scales)
+                                             : (row_ok ? __ldg(p.a_scales + row) : 0.f);
         const float s0 = (MODE == kTensor) ? sa * __ldg(p.b_scales) : 0.f;
 #pragma unroll 1
         for (int c = 0; c < CHUNK / 32; ++c) {
@@ -409,7 +418,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             const float sbl = colq < p.N ? __ldg(p.b_scales + colq) : 0.f;
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] *= sa * __shfl_sync(0xffffffffu, sbl, i);
-          } else {
+          } else if (MODE == kTensor) {
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] *= s0;
           }
@@ -505,18 +514,22 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-// K-major uint8 matrix [rows][K], box (128 K) x box_rows, 128B swizzle, zero
-// fill outside the matrix.
-bool make_tmap(CUtensorMap* tm, const uint8_t* base, int64_t rows, int64_t K, uint32_t box_rows) {
+// K-major matrix [rows][K] with row stride `ld` elements, box of 128 bytes
+// along K x box_rows, 128B swizzle, zero fill outside the matrix: uint8 E4M3
+// codes (128 elements per box row) or bf16 values (64 elements).
+bool make_tmap(CUtensorMap* tm, const void* base, int64_t rows, int64_t K, int64_t ld,
+               uint32_t box_rows, bool bf16) {
   auto fn = encode_fn();
   if (fn == nullptr) return false;
+  const int esize = bf16 ? 2 : 1;
   cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(rows)};
-  cuuint64_t strides[1] = {static_cast<cuuint64_t>(K)};
-  cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), box_rows};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld * esize)};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(BK / esize), box_rows};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = fn(tm, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t*>(base), dims, strides,
-                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  CUresult r = fn(tm, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_UINT8, 2,
+                  const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
 
@@ -550,8 +563,10 @@ cudaError_t launch_mode(const CUtensorMap& ta, const CUtensorMap& tb, const Para
 template <int EPI>
 cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s) {
   if (a.M == 0 || a.N == 0) return cudaSuccess;
+  const bool bf16 = a.gran == kBf16;
   CUtensorMap ta, tb;
-  if (!make_tmap(&ta, a.a_codes, a.M, a.K, BM) || !make_tmap(&tb, a.b_codes, a.N, a.K, BN))
+  if (!make_tmap(&ta, a.a_codes, a.M, a.K, a.lda ? a.lda : a.K, BM, bf16) ||
+      !make_tmap(&tb, a.b_codes, a.N, a.K, a.ldb ? a.ldb : a.K, BN, bf16))
     return cudaErrorInvalidValue;
   Params p{};
   p.a_scales = a.a_scales;
@@ -567,7 +582,8 @@ cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s) {
   p.K = static_cast<int>(a.K);
   p.num_m = static_cast<int>((a.M + BM - 1) / BM);
   p.num_n = static_cast<int>((a.N + BN - 1) / BN);
-  p.num_kb = static_cast<int>((a.K + BK - 1) / BK);
+  const int64_t bk_elems = bf16 ? BK / 2 : BK;  // K elements per 128-byte stage row
+  p.num_kb = static_cast<int>((a.K + bk_elems - 1) / bk_elems);
   p.n_chunks = static_cast<int>((a.N + CHUNK - 1) / CHUNK);
   p.wait_limit_ns = wait_limit_ns();
   const int64_t tiles = static_cast<int64_t>(p.num_m) * p.num_n;
@@ -575,6 +591,7 @@ cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s) {
   switch (a.gran) {
     case kTensor: return launch_mode<kTensor, EPI>(ta, tb, p, grid, s);
     case kRow: return launch_mode<kRow, EPI>(ta, tb, p, grid, s);
+    case kBf16: return launch_mode<kBf16, EPI>(ta, tb, p, grid, s);
     default: return launch_mode<kBlock, EPI>(ta, tb, p, grid, s);
   }
 }

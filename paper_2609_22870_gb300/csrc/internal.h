@@ -22,12 +22,13 @@ uint32_t quantize_status_take();
 
 // ----------------------------------------------------------------- gemm.cu
 struct GemmArgs {
-  const uint8_t* a_codes;   // [M][K]
+  const void* a_codes;      // [M][K] E4M3 codes, or bf16 values when gran == kGemmBf16
   const float* a_scales;
-  const uint8_t* b_codes;   // [N][K]
+  const void* b_codes;      // [N][K]
   const float* b_scales;
-  int gran;
+  int gran;                 // fp8rl_gran, or kGemmBf16 (BF16 shadow pass, no scales)
   int64_t M, N, K;
+  int64_t lda, ldb;         // row strides in elements (0 = K)
   const int32_t* targets;   // [M]
   // LSE epilogue outputs (workspace)
   float2* partials;         // [gemm_partials_per_token(N)][M]
@@ -37,6 +38,8 @@ struct GemmArgs {
   const float* grad;        // [M]
   float* out;               // [M][N]
 };
+constexpr int kGemmBf16 = 3;
+
 // LSE partials the GEMM leaves per token (one per column slot of each
 // 256-wide vocabulary tile).
 int64_t gemm_partials_per_token(int64_t N);

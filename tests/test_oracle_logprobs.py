@@ -4,6 +4,10 @@ Closed forms (W = 0, V = 1), one-hot weight rows (catches a transposed or
 mis-indexed operand), scale-exchange invariance between the two operands'
 block scales (catches a dropped or misplaced scale), SciPy's log_softmax, the
 normalisation of the softmax, and a finite-difference check of dlogits.
+
+The BF16 shadow-pass scorer (§4) is pinned by its closed forms, one-hot rows,
+and by agreement with the (separately pinned) FP8 path on operands that E4M3
+represents exactly with scale 1, where quantisation changes nothing.
 """
 
 import numpy as np
@@ -119,3 +123,58 @@ def test_dlogits_finite_difference():
 def test_ratio_identity():
     lp = np.random.default_rng(6).standard_normal(10)
     assert np.all(L.importance_ratios(lp, lp) == 1.0)
+
+
+def _bf16_values(rng, shape, std):
+    """Random float32 values that are exactly representable in bf16."""
+    x = (rng.standard_normal(shape) * std).astype(np.float32)
+    return (x.view(np.uint32) & np.uint32(0xFFFF0000)).view(np.float32)
+
+
+def test_bf16_zero_weight_and_single_word():
+    rng = np.random.default_rng(10)
+    h = _bf16_values(rng, (6, 64), 1.0)
+    lp, lse = L.bf16_token_logprobs(h, np.zeros((29, 64), np.float32), rng.integers(0, 29, 6))
+    assert np.allclose(lp, -np.log(29), rtol=0, atol=1e-14)
+    assert np.allclose(lse, np.log(29), rtol=0, atol=1e-14)
+    lp1, _ = L.bf16_token_logprobs(h, _bf16_values(rng, (1, 64), 0.02), np.zeros(6, np.int64))
+    assert np.all(lp1 == 0.0)
+
+
+def test_bf16_one_hot_rows_pick_hidden_entries():
+    rng = np.random.default_rng(11)
+    T, H, V = 5, 96, 13
+    h = _bf16_values(rng, (T, H), 1.0)
+    cols = rng.integers(0, H, V)
+    W = np.zeros((V, H), np.float32)
+    W[np.arange(V), cols] = 1.0
+    assert np.array_equal(L.bf16_logits(h, W), h[:, cols].astype(np.float64))
+    rows = np.array([4, 1])
+    assert np.array_equal(L.bf16_logits(h, W, rows), h[rows][:, cols].astype(np.float64))
+
+
+def test_bf16_path_equals_fp8_path_on_exact_e4m3_operands():
+    # every finite E4M3 value is a bf16 value; with one entry of +-448 per
+    # tensor the per-tensor scale is exactly 1 and the codes decode to the
+    # inputs, so both scorers see identical operands
+    rng = np.random.default_rng(12)
+    T, H, V = 7, 128, 50
+    finite = np.array([c for c in range(256) if c not in (0x7F, 0xFF)], np.uint8)
+    vals = e4m3.decode(finite).astype(np.float32)
+    h = rng.choice(vals, size=(T, H)).astype(np.float32)
+    W = rng.choice(vals, size=(V, H)).astype(np.float32)
+    h[0, 0] = 448.0
+    W[3, 5] = -448.0
+    hq, hs = Q.quantize(h, Q.TENSOR, Q.ACT)
+    wq, ws = Q.quantize(W, Q.TENSOR, Q.WEIGHT)
+    assert hs[0] == 1.0 and ws[0] == 1.0
+    y = rng.integers(0, V, T)
+    lp8, lse8 = L.token_logprobs(hq, hs, wq, ws, Q.TENSOR, y)
+    lpb, lseb = L.bf16_token_logprobs(h, W, y)
+    assert np.array_equal(lp8, lpb) and np.array_equal(lse8, lseb)
+    # and a perturbation that E4M3 cannot represent separates them
+    h2 = h.copy()
+    h2[1, 1] = np.float32(1.0078125)  # 1 + 2^-7: bf16-exact, not E4M3-exact
+    hq2, hs2 = Q.quantize(h2, Q.TENSOR, Q.ACT)
+    assert not np.array_equal(L.token_logprobs(hq2, hs2, wq, ws, Q.TENSOR, y)[0],
+                              L.bf16_token_logprobs(h2, W, y)[0])
