@@ -26,6 +26,8 @@ calibrate   Calibrated Clipping: lower-bound alignment, upper-bound
             rebalancing, SmoothUpdate (§4, Eq. 5, Algorithm 1).
 surrogate   clipped PPO surrogate with TIS weights, token-mean
             aggregation, clip fractions and dLoss/dlogp (Eq. 1, Eq. 4).
+diagnostics over-clipping counts, clip fractions and probability / ratio
+            NMAE against BF16 references (§3); TIS weights (§2.3).
 """
 
-from . import e4m3, quantize, logprobs, calibrate, surrogate  # noqa: F401
+from . import e4m3, quantize, logprobs, calibrate, surrogate, diagnostics  # noqa: F401
