@@ -271,6 +271,13 @@ def run_ours(args, rank, world, local_rank):
     api.check()
     res = api.read_calib_result(b.cal_res)
     st = api.read_clip_stats(b.stats)
+    # §3 diagnosis of this batch against the BF16 shadow pass (untimed)
+    api.quantize(h, gran, api.ROLE_ACT, b.h_codes, b.h_scales, b.q_ws)
+    api.token_logprobs(b.h_codes, b.h_scales, b.w_codes, b.w_scales, gran, y, logp_old,
+                       workspace=b.lp_ws, out={"logp": b.logp, "lse": b.lse, "ratio": b.ratio})
+    diag = api.read_clip_diag(api.clip_diagnostics(b.ratio, r_bf16, adv_d, mask_d, b.logp, logp_bf16,
+                                                   w.eps_low, w.eps_high))
+    api.check()
 
     ms = elapsed_ms / args.steps
     if world > 1:
@@ -325,6 +332,9 @@ def run_ours(args, rank, world, local_rank):
         "clocks": clk,
         "result": {"lo": res["lo_new"], "hi": res["hi_new"], "loss": st["loss"],
                    "clip_frac_pos": st["clip_frac_pos"], "clip_frac_neg": st["clip_frac_neg"]},
+        "diagnostics": {k: diag[k] for k in ("over_clipped_lo", "over_clipped_hi", "clipped_lo_fp8",
+                                             "clipped_hi_fp8", "clipped_lo_bf16", "clipped_hi_bf16",
+                                             "nmae_prob", "nmae_ratio")},
     }
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = oracle_step_estimate(w, budget_s=args.cpu_budget)

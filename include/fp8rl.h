@@ -332,6 +332,58 @@ fp8rl_status fp8rl_dlogits_rows(const uint8_t* h_codes, const float* h_scales,
                                 void* stream);
 
 /* ---------------------------------------------------------------------- */
+/* §3 diagnostics against BF16 references; TIS weights (§2.3)               */
+/* ---------------------------------------------------------------------- */
+
+/* Device-resident result of fp8rl_clip_diagnostics (counts over valid tokens). */
+typedef struct fp8rl_clip_diag {
+  int64_t n_valid, n_pos, n_neg;    /* mask = 1; and A > 0, A < 0 among them      */
+  int64_t clipped_lo_fp8;           /* A < 0 and r_fp8  <= c_lo                  */
+  int64_t clipped_hi_fp8;           /* A > 0 and r_fp8  >= c_hi                  */
+  int64_t clipped_lo_bf16;          /* A < 0 and r_bf16 <= c_lo                  */
+  int64_t clipped_hi_bf16;          /* A > 0 and r_bf16 >= c_hi                  */
+  int64_t over_clipped_lo;          /* A < 0, r_bf16 > c_lo and r_fp8 <= c_lo     */
+  int64_t over_clipped_hi;          /* A > 0, r_bf16 < c_hi and r_fp8 >= c_hi     */
+  double abs_err_prob, sum_prob_bf16;   /* sum |p_fp8 - p_bf16|, sum p_bf16, p = exp(logp) */
+  double abs_err_ratio, sum_ratio_bf16; /* sum |r_fp8 - r_bf16|, sum |r_bf16|             */
+  double nmae_prob, nmae_ratio;     /* the quotients of the two pairs (NaN if 0/0) */
+  float c_lo, c_hi;                 /* fl32(1 - eps_low), fl32(1 + eps_high)      */
+  int32_t flags;                    /* FP8RL_DIAG_FLAG_* bits                     */
+  int32_t reserved;
+} fp8rl_clip_diag;
+
+#define FP8RL_DIAG_FLAG_NO_VALID 1  /* no valid token                          */
+#define FP8RL_DIAG_FLAG_NO_PROB 2   /* logp_fp8 / logp_bf16 not given: no prob NMAE */
+
+size_t fp8rl_clip_diagnostics_workspace_size(int64_t T);
+
+/* The diagnosis of §3 ("The Cause"): how often FP8 noise pushes tokens over
+ * the trust-region bounds that their BF16 references stay inside
+ * (over-clipping, lower: A < 0, r_BF16 > 1 - eps, r_FP8 <= 1 - eps; upper:
+ * A > 0, r_BF16 < 1 + eps, r_FP8 >= 1 + eps), the PPO clip counts of both
+ * ratio sets at the same bounds (clipped at equality, §2.1), and the
+ * normalised mean absolute error sum |x - x_ref| / sum |x_ref| of the
+ * probabilities exp(logp) and of the ratios.  One pass; counts exact, sums
+ * compensated float32 per thread and float64 across threads in a fixed
+ * order.
+ *   logp_fp8, logp_bf16  float [T] or both NULL (no probability NMAE)
+ *   r_fp8, r_bf16, adv   float [T];  mask uint8 [T] or NULL (all valid)
+ *   out                  DEVICE pointer to one fp8rl_clip_diag */
+fp8rl_status fp8rl_clip_diagnostics(const float* logp_fp8, const float* logp_bf16,
+                                    const float* r_fp8, const float* r_bf16, const float* adv,
+                                    const uint8_t* mask, int64_t T, float eps_low,
+                                    float eps_high, fp8rl_clip_diag* out,
+                                    void* workspace, size_t workspace_bytes, void* stream);
+
+/* The truncated importance-sampling weight of J_TIS (§2.3), which corrects
+ * for the sampler (FP8 rollout) differing from the learner's old policy:
+ *   w_t = min(exp(logp_old_t - logp_sampler_t), C)       (C = 2 typically)
+ * float [T] in, float [T] out (feeds fp8rl_clipped_surrogate's w_tis).
+ * C must be finite and > 0. */
+fp8rl_status fp8rl_tis_weights(const float* logp_old, const float* logp_sampler, int64_t T,
+                               float C, float* w_tis, void* stream);
+
+/* ---------------------------------------------------------------------- */
 /* Bounded waits                                                            */
 /* ---------------------------------------------------------------------- */
 

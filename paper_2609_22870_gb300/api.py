@@ -54,6 +54,18 @@ class ClipStats(ctypes.Structure):
                 ("flags", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
 
+class ClipDiag(ctypes.Structure):
+    _fields_ = [("n_valid", ctypes.c_int64), ("n_pos", ctypes.c_int64), ("n_neg", ctypes.c_int64),
+                ("clipped_lo_fp8", ctypes.c_int64), ("clipped_hi_fp8", ctypes.c_int64),
+                ("clipped_lo_bf16", ctypes.c_int64), ("clipped_hi_bf16", ctypes.c_int64),
+                ("over_clipped_lo", ctypes.c_int64), ("over_clipped_hi", ctypes.c_int64),
+                ("abs_err_prob", ctypes.c_double), ("sum_prob_bf16", ctypes.c_double),
+                ("abs_err_ratio", ctypes.c_double), ("sum_ratio_bf16", ctypes.c_double),
+                ("nmae_prob", ctypes.c_double), ("nmae_ratio", ctypes.c_double),
+                ("c_lo", ctypes.c_float), ("c_hi", ctypes.c_float),
+                ("flags", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
 _p, _i64, _u64, _f, _i, _sz = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_uint64, ctypes.c_float,
                                ctypes.c_int, ctypes.c_size_t)
 _SIGS = {
@@ -81,6 +93,9 @@ _SIGS = {
     "fp8rl_dlogits_workspace_size": (_sz, [_i64, _i64, _i64, _i]),
     "fp8rl_dlogits_rows": (_i, [_p, _p, _p, _p, _i, _i64, _i64, _i64, _p, _p, _p, _p, _i64, _p, _p,
                                 _sz, _p]),
+    "fp8rl_clip_diagnostics_workspace_size": (_sz, [_i64]),
+    "fp8rl_clip_diagnostics": (_i, [_p, _p, _p, _p, _p, _p, _i64, _f, _f, _p, _p, _sz, _p]),
+    "fp8rl_tis_weights": (_i, [_p, _p, _i64, _f, _p, _p]),
     "fp8rl_set_wait_limit_ns": (None, [_u64]),
     "fp8rl_wait_selftest": (_i, [_u64, _p]),
 }
@@ -373,6 +388,44 @@ def read_clip_stats(buf):
     d["clip_frac_neg"] = d["clipped_neg"] / d["n_neg"] if d["n_neg"] else 0.0
     d["clip_frac"] = (d["clipped_pos"] + d["clipped_neg"]) / d["n_valid"] if d["n_valid"] else 0.0
     return d
+
+
+# ------------------------------------------------------------------ diagnostics
+def clip_diagnostics(r_fp8, r_bf16, adv, mask=None, logp_fp8=None, logp_bf16=None, eps_low=0.2,
+                     eps_high=0.2, out=None, workspace=None, stream=None):
+    """fp8rl_clip_diagnostics (§3): over-clipping, clip counts and NMAE against
+    BF16 references -> device buffer holding one fp8rl_clip_diag."""
+    T = r_fp8.numel()
+    for name, t in (("r_fp8", r_fp8), ("r_bf16", r_bf16), ("adv", adv), ("logp_fp8", logp_fp8),
+                    ("logp_bf16", logp_bf16)):
+        _dev(t, torch.float32, name, T)
+    _dev(mask, torch.uint8, "mask", T)
+    dev = r_fp8.device
+    out = torch.zeros(ctypes.sizeof(ClipDiag), dtype=torch.uint8, device=dev) if out is None else out
+    if workspace is None:
+        workspace = _workspace(lib.fp8rl_clip_diagnostics_workspace_size(T), dev)
+    _ok(lib.fp8rl_clip_diagnostics(_ptr(logp_fp8), _ptr(logp_bf16), _ptr(r_fp8), _ptr(r_bf16), _ptr(adv),
+                                   _ptr(mask), T, eps_low, eps_high, _ptr(out), _ptr(workspace),
+                                   workspace.numel(), _stream(stream)), "fp8rl_clip_diagnostics")
+    return out
+
+
+def read_clip_diag(buf):
+    raw = bytes(buf.cpu().numpy().tobytes())
+    d = ClipDiag.from_buffer_copy(raw[: ctypes.sizeof(ClipDiag)])
+    return {name: getattr(d, name) for name, _ in ClipDiag._fields_}
+
+
+def tis_weights(logp_old, logp_sampler, C=2.0, out=None, stream=None):
+    """fp8rl_tis_weights (§2.3): w = min(exp(logp_old - logp_sampler), C)."""
+    T = logp_old.numel()
+    _dev(logp_old, torch.float32, "logp_old", T)
+    _dev(logp_sampler, torch.float32, "logp_sampler", T)
+    out = torch.empty(T, dtype=torch.float32, device=logp_old.device) if out is None else out
+    _dev(out, torch.float32, "out", T)
+    _ok(lib.fp8rl_tis_weights(_ptr(logp_old), _ptr(logp_sampler), T, C, _ptr(out), _stream(stream)),
+        "fp8rl_tis_weights")
+    return out
 
 
 # ------------------------------------------------------------------ dlogits

@@ -304,6 +304,32 @@ fp8rl_status fp8rl_clipped_surrogate(const float* r, const float* adv, const uin
   return e == cudaSuccess ? FP8RL_OK : cuda_fail(e);
 }
 
+// ------------------------------------------------------------------ diagnostics
+size_t fp8rl_clip_diagnostics_workspace_size(int64_t T) { return T < 0 ? 0 : diag_workspace_bytes(T); }
+
+fp8rl_status fp8rl_clip_diagnostics(const float* lp8, const float* lpb, const float* r8,
+                                    const float* rb, const float* adv, const uint8_t* mask,
+                                    int64_t T, float eps_low, float eps_high, fp8rl_clip_diag* out,
+                                    void* ws, size_t ws_bytes, void* stream) {
+  if (!out || (T > 0 && (!r8 || !rb || !adv)) || ((lp8 == nullptr) != (lpb == nullptr)))
+    return FP8RL_EINVAL;
+  if (!std::isfinite(eps_low) || !std::isfinite(eps_high)) return FP8RL_EINVAL;
+  if (T < 0) return FP8RL_ESHAPE;
+  if (!ws || ws_bytes < diag_workspace_bytes(T)) return FP8RL_EWORKSPACE;
+  cudaError_t e = launch_clip_diag(lp8, lpb, r8, rb, adv, mask, T, 1.0f - eps_low, 1.0f + eps_high,
+                                   out, ws, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? FP8RL_OK : cuda_fail(e);
+}
+
+fp8rl_status fp8rl_tis_weights(const float* lp_old, const float* lp_samp, int64_t T, float C,
+                               float* w, void* stream) {
+  if (T > 0 && (!lp_old || !lp_samp || !w)) return FP8RL_EINVAL;
+  if (!std::isfinite(C) || !(C > 0.f)) return FP8RL_EINVAL;
+  if (T < 0) return FP8RL_ESHAPE;
+  cudaError_t e = launch_tis(lp_old, lp_samp, T, C, w, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? FP8RL_OK : cuda_fail(e);
+}
+
 // ------------------------------------------------------------------ dlogits
 // Workspace: gathered codes [n][H], scales, targets, lse, grad.
 static size_t dl_codes_bytes(int64_t n, int64_t H) { return align_up(static_cast<size_t>(n * H), 256); }

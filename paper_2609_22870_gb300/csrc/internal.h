@@ -75,6 +75,14 @@ cudaError_t launch_surrogate(const float* r, const float* adv, const uint8_t* ma
                              cudaStream_t s);
 uint32_t loss_status_take();
 
+// ----------------------------------------------------------------- diag.cu
+size_t diag_workspace_bytes(int64_t T);
+cudaError_t launch_clip_diag(const float* lp8, const float* lpb, const float* r8, const float* rb,
+                             const float* adv, const uint8_t* mask, int64_t T, float c_lo,
+                             float c_hi, fp8rl_clip_diag* out, void* ws, cudaStream_t s);
+cudaError_t launch_tis(const float* lp_old, const float* lp_samp, int64_t T, float C, float* w,
+                       cudaStream_t s);
+
 // SM count of the current device (cached per device).
 int sm_count();
 
