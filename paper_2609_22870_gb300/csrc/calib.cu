@@ -30,6 +30,10 @@ namespace {
 __device__ uint32_t d_status;
 
 constexpr int kBuckets = 2048;
+constexpr int kCoopThreads = 512;         // block of the one-launch (cooperative) kernel
+constexpr int64_t kCoopMaxT = 1 << 18;    // tokens up to which one launch does it all
+constexpr int kCoopTokensPerBlock = 2048; // its grid: ceil(T / 2048) blocks, at most 128
+constexpr int kCoopMaxBlocks = 128;
 
 constexpr unsigned kNone = 0xFFFFFFFFu;
 
@@ -51,6 +55,7 @@ struct State {
   unsigned long long emax_bits;  // frexp exponent of max|e| plus kEBias (0 = no term)
   unsigned long long s_pos_bf, s_neg_bf, s_neg_fp, s_pos_fp;  // int64 two's complement
   unsigned int bad;
+  unsigned int bar_count, bar_gen;  // grid barrier of the one-launch kernel
   unsigned int nb_below1;  // 1 + max{key < u} (0 = none)
   unsigned int nb_above;   // min{key > u}     (kNone = none)
   unsigned int nb_mpiece;  // L: min{key > key(lo_min)}   H: min{key >= key(hi_min), q > 0}
@@ -361,7 +366,7 @@ __device__ __forceinline__ int pass_token(const Args& a, const PassCtx& x, const
 // Block histogram in shared memory with native 32-bit atomics only: counts
 // as 32-bit words, 64-bit weights as low and high words, the carry out of the
 // low word taken from the value the atomic returns (exact modulo 2^64).
-struct ShHist {
+struct __align__(16) ShHist {
   unsigned cnt[kBuckets];
   unsigned wlo[kBuckets];
   unsigned whi[kBuckets];
@@ -408,11 +413,11 @@ __device__ __forceinline__ void hist_add_lane(ShHist& sh, int d, long long w) {
   if (d >= 0) sh_add(sh, d, 1u, static_cast<unsigned long long>(w));
 }
 
-// Passes read G tokens per lane and step: 16-byte loads when G = 4.
+// One pass over the tokens by the whole grid (or by one block in the fused
+// small-T kernel).  Passes read G tokens per lane and step: 16-byte loads when
+// G = 4.  sh_cand holds the stage's grid candidates in GRID mode.
 template <int G>
-__global__ void __launch_bounds__(256) pass_kernel(Args a, int stage) {
-  __shared__ ShHist sh;
-  __shared__ float sh_cand[kBuckets];  // GRID: the stage's candidate thresholds
+__device__ void pass_body(const Args& a, int stage, ShHist& sh, float* sh_cand) {
   State* st = a.st;
   if ((stage == kH1 || stage == kH2 || stage == kHNb) && !st->h_active) return;
   if (stage == kPFin && st->p_known) return;
@@ -584,6 +589,13 @@ __global__ void __launch_bounds__(256) pass_kernel(Args a, int stage) {
   }
 }
 
+template <int G>
+__global__ void __launch_bounds__(256) pass_kernel(Args a, int stage) {
+  __shared__ ShHist sh;
+  __shared__ float sh_cand[kBuckets];
+  pass_body<G>(a, stage, sh, sh_cand);
+}
+
 // ------------------------------------------------------------------ 128-bit
 struct U128 {
   unsigned long long hi, lo;
@@ -614,16 +626,16 @@ __device__ __forceinline__ float smooth(float b_old, float b_star, float delta) 
   return __fadd_rn(b_old, d);
 }
 
-// One step of the weighted radix select, by the whole block: smallest bucket
-// b with cnt[b] > 0 and (below + sum_{b' <= b} w[b']) * D >= X.
-__device__ void select_step(State* st, int bits, bool last) {
-  __shared__ long long sh_incl[kBuckets];
+// One step of the weighted radix select, by the whole block (512 or 1024
+// threads): smallest bucket b with cnt[b] > 0 and
+// (below + sum_{b' <= b} w[b']) * D >= X.  sh_incl: kBuckets of shared scratch.
+__device__ void select_step(State* st, int bits, bool last, long long* sh_incl) {
   __shared__ long long warp_tot[32];
   __shared__ int sh_best;
   const int nb = 1 << bits;
   const int tid = threadIdx.x;
-  const int per = kBuckets / blockDim.x;  // 2 buckets per thread
-  long long local[2] = {0, 0};
+  const int per = kBuckets / blockDim.x;  // 2 or 4 buckets per thread
+  long long local[4] = {0, 0, 0, 0};
   long long run = 0;
   for (int j = 0; j < per; ++j) {
     const int b = tid * per + j;
@@ -774,7 +786,7 @@ __device__ float upper_from_interval(const Args& a, const State* st, float lo, f
   return clampf(a.c_hi, fmaxf(b, a.hi_min), a.hi_max);
 }
 
-__global__ void __launch_bounds__(1024) decide_kernel(Args a, int stage) {
+__device__ void decide_body(const Args& a, int stage, long long* scratch) {
   State* st = a.st;
   const int tid = threadIdx.x;
   __shared__ int sh_go;
@@ -825,13 +837,13 @@ __global__ void __launch_bounds__(1024) decide_kernel(Args a, int stage) {
     }
     __syncthreads();
     if (a.grid_mode) zero_hist(st);
-    else if (sh_go) select_step(st, 11, false);
+    else if (sh_go) select_step(st, 11, false, scratch);
     return;
   }
 
   if (stage == kSums) {
     if (!a.grid_mode) {
-      if (st->n_neg > 0) select_step(st, 11, false);
+      if (st->n_neg > 0) select_step(st, 11, false, scratch);
       return;
     }
     if (tid == 0 && begin_upper(a, st)) {
@@ -862,7 +874,7 @@ __global__ void __launch_bounds__(1024) decide_kernel(Args a, int stage) {
   }
 
   if (stage == kL2) {
-    if (st->n_neg > 0) select_step(st, 10, true);
+    if (st->n_neg > 0) select_step(st, 10, true, scratch);
     if (tid == 0) reset_neighbours(st);
     return;
   }
@@ -902,14 +914,14 @@ __global__ void __launch_bounds__(1024) decide_kernel(Args a, int stage) {
   if (stage == kH0) {
     if (tid == 0) sh_go = begin_upper(a, st);
     __syncthreads();
-    if (sh_go) select_step(st, 11, false);
+    if (sh_go) select_step(st, 11, false, scratch);
     return;
   }
 
   if (stage == kH1 || stage == kH2) {
     if (tid == 0) sh_go = st->h_active && st->found;
     __syncthreads();
-    if (sh_go) select_step(st, stage == kH1 ? 11 : 10, stage == kH2);
+    if (sh_go) select_step(st, stage == kH1 ? 11 : 10, stage == kH2, scratch);
     if (stage == kH2 && tid == 0) {
       if (!st->found) st->u_key = kNone;
       reset_neighbours(st);
@@ -965,6 +977,69 @@ __global__ void __launch_bounds__(1024) decide_kernel(Args a, int stage) {
   }
 }
 
+__global__ void __launch_bounds__(1024) decide_kernel(Args a, int stage) {
+  __shared__ long long sh_incl[kBuckets];
+  decide_body(a, stage, sh_incl);
+}
+
+struct StageList {
+  int n;
+  int s[9];
+};
+
+
+// Grid-wide barrier of the one-launch kernel (all blocks co-resident: it is
+// launched cooperatively).  Thread 0 of each block arrives on a counter; the
+// last arrival opens the next generation.  The wait is bounded by the
+// library's wait limit; false means it expired (the status word says so).
+__device__ bool grid_barrier(State* st, uint64_t limit_ns, volatile int* sh_ok) {
+  __syncthreads();
+  if (gridDim.x == 1) return true;  // one block: the block barrier is the grid barrier
+  if (threadIdx.x == 0) {
+    bool ok = true;
+    volatile unsigned* gen_p = &st->bar_gen;
+    const unsigned gen = *gen_p;
+    __threadfence();
+    if (atomicAdd(&st->bar_count, 1u) == gridDim.x - 1) {
+      st->bar_count = 0;
+      __threadfence();
+      atomicAdd(&st->bar_gen, 1u);
+    } else {
+      const uint64_t t0 = globaltimer_ns();
+      while (*gen_p == gen) {
+        if (globaltimer_ns() - t0 > limit_ns) {
+          ok = false;
+          flag(kErrTimeout);
+          break;
+        }
+        __nanosleep(64);
+      }
+    }
+    __threadfence();
+    *sh_ok = ok;
+  }
+  __syncthreads();
+  return *sh_ok != 0;
+}
+
+// Small and mid-size T: every pass and decision in one cooperative launch, so
+// one launch replaces the 2 x 9 (or 2 x 3) launches of the grid path.  All
+// blocks run each pass over their share of the tokens; block 0 then takes the
+// decision while the others wait at the grid barrier.  The decide steps reuse
+// the pass histogram's shared memory as scan scratch.
+template <int G>
+__global__ void __launch_bounds__(kCoopThreads) coop_kernel(Args a, StageList list, uint64_t limit_ns) {
+  __shared__ ShHist sh;
+  __shared__ float sh_cand[kBuckets];
+  __shared__ int sh_ok;
+  for (int i = 0; i < list.n; ++i) {
+    pass_body<G>(a, list.s[i], sh, sh_cand);
+    if (!grid_barrier(a.st, limit_ns, &sh_ok)) return;
+    if (blockIdx.x == 0) decide_body(a, list.s[i], reinterpret_cast<long long*>(&sh));
+    if (!grid_barrier(a.st, limit_ns, &sh_ok)) return;
+  }
+}
+
 }  // namespace
 
 size_t calib_workspace_bytes(int64_t) { return align_up(sizeof(State), 256); }
@@ -1010,6 +1085,19 @@ cudaError_t launch_calibrate(const float* r_fp8, const float* r_bf16, const floa
   const int stages_grid[] = {kPrep, kSums, kPFin};
   const int* stages = a.grid_mode ? stages_grid : stages_exact;
   const int n = a.grid_mode ? 3 : 9;
+  if (T <= kCoopMaxT) {
+    StageList list{};
+    list.n = n;
+    for (int i = 0; i < n; ++i) list.s[i] = stages[i];
+    int64_t nb = (T + kCoopTokensPerBlock - 1) / kCoopTokensPerBlock;
+    nb = nb < 1 ? 1 : (nb > kCoopMaxBlocks ? kCoopMaxBlocks : nb);
+    if (nb > sm_count()) nb = sm_count();
+    uint64_t limit = wait_limit_ns();
+    void* args[] = {&a, &list, &limit};
+    const void* fn = vec ? reinterpret_cast<const void*>(&coop_kernel<4>)
+                         : reinterpret_cast<const void*>(&coop_kernel<1>);
+    return cudaLaunchCooperativeKernel(fn, dim3(static_cast<unsigned>(nb)), dim3(kCoopThreads), args, 0, s);
+  }
   for (int i = 0; i < n; ++i) {
     if (vec) pass_kernel<4><<<grid, 256, 0, s>>>(a, stages[i]);
     else pass_kernel<1><<<grid, 256, 0, s>>>(a, stages[i]);

@@ -55,7 +55,7 @@ MODES = [OC.EXACT, OC.GRID]
 
 
 @pytest.mark.parametrize("mode", MODES)
-@pytest.mark.parametrize("T", [1, 2, 17, 1000, 40000])
+@pytest.mark.parametrize("T", [1, 2, 17, 1000, 40000, 65537, 200000, 262145])
 @pytest.mark.parametrize("eps", [(0.2, 0.2), (0.2, 0.28)])
 def test_calibrate_parity(cuda_lib, mode, T, eps):
     args = _inputs(T, T + int(eps[1] * 100))
