@@ -1,6 +1,6 @@
 // a3: FP8 lm_head GEMM on the tcgen05 tensor cores with a streaming
-// logsumexp + target-gather epilogue; a4: merge of the per-chunk partials into
-// log-probs and importance ratios (§2.1 ratio, Eq. 3 scaling).
+// logsumexp + target-gather epilogue (§2.1 ratio, Eq. 3 scaling); the merge of
+// the per-chunk partials into log-probs and ratios (a4) is in combine.cu.
 //
 // z[t][v] = sum_k S_h S_W q_h[t][k] q_W[v][k] is never stored.  Each CTA owns
 // persistent 128 (tokens) x 256 (vocab) output tiles:
@@ -12,7 +12,7 @@
 //               weight scales into a shared-memory ring, so the epilogue never
 //               waits on global loads;
 //   warp 3      idle (it completes the first warpgroup, whose register budget
-//               is lowered to 40 so the epilogue can hold 224);
+//               is lowered to 56 so the epilogue can hold 224);
 //   warps 4..11 epilogue: tcgen05.ld of the accumulator, one thread per token
 //               row and 128-column half, scales applied, then the running
 //               (max, sum exp) of its 128 columns and z[t][y_t] if y_t falls in
@@ -48,7 +48,7 @@ constexpr int STAGES = 4;
 constexpr int EPI_WARPS = 8;
 constexpr int EPI_WARP0 = 4;      // first epilogue warp (start of warpgroup 1)
 constexpr int THREADS = 128 + EPI_WARPS * 32;
-constexpr int CTRL_REGS = 40;     // register budget of warpgroup 0 (producer, MMA)
+constexpr int CTRL_REGS = 56;     // register budget of warpgroup 0 (producer, MMA)
 constexpr int EPI_REGS = 224;     // register budget of the two epilogue warpgroups
 constexpr uint32_t A_BYTES = BM * BK;
 constexpr uint32_t B_BYTES = BN * BK;
@@ -81,6 +81,20 @@ struct Params {
 };
 
 __device__ __forceinline__ void flag(uint32_t bits) { atomicOr(&d_status, bits); }
+
+// Tile order: bands of kBandM token blocks, and within a band the token block
+// varies fastest.  The 152 tiles in flight then share one or two vocabulary
+// tiles and a band of h codes small enough to stay in L2, so the lm_head codes
+// are read once per band and h codes about once.
+constexpr int kBandM = 64;
+__device__ __forceinline__ void tile_coords(int tile, const Params& p, int& m_blk, int& n_blk) {
+  const int band = tile / (kBandM * p.num_n);
+  const int m_base = band * kBandM;
+  const int band_m = min(kBandM, p.num_m - m_base);
+  const int local = tile - band * kBandM * p.num_n;
+  m_blk = m_base + local % band_m;
+  n_blk = local / band_m;
+}
 
 // Running epilogue state of one thread: row `row`, vocabulary columns
 // [col0, col0 + 128) consumed 32 at a time (values already scaled).
@@ -208,7 +222,9 @@ __global__ void __launch_bounds__(THREADS, 1)
     uint32_t armed = 0, armed_phase = 0;  // bit s: stage s loaded / its parity
     bool ok = true;
     for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
-      const int m0 = (tile % p.num_m) * BM, n0 = (tile / p.num_m) * BN;
+      int m_blk, n_blk;
+      tile_coords(tile, p, m_blk, n_blk);
+      const int m0 = m_blk * BM, n0 = n_blk * BN;
       for (int kb = 0; kb < p.num_kb; ++kb) {
         ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&empty[stage]), phase ^ 1, lim, abort_flag));
         if (!ok) break;
@@ -243,7 +259,9 @@ __global__ void __launch_bounds__(THREADS, 1)
     uint32_t sphase = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
-      const int m0 = (tile % p.num_m) * BM, n_blk = tile / p.num_m;
+      int m_blk, n_blk;
+      tile_coords(tile, p, m_blk, n_blk);
+      const int m0 = m_blk * BM;
       const int wb0 = 2 * n_blk;
       for (int kb = 0; kb < p.num_kb; ++kb) {
         ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&sc_empty[slot]), sphase ^ 1, lim, abort_flag));
@@ -341,7 +359,8 @@ __global__ void __launch_bounds__(THREADS, 1)
     uint32_t aphase = 0, sphase = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
-      const int m_blk = tile % p.num_m, n_blk = tile / p.num_m;
+      int m_blk, n_blk;
+      tile_coords(tile, p, m_blk, n_blk);
       const int row = m_blk * BM + rit;
       const bool row_ok = row < p.M;
       const int col0 = n_blk * BN + half * CHUNK;
@@ -543,7 +562,7 @@ cudaError_t launch_mode(const CUtensorMap& ta, const CUtensorMap& tb, const Para
   if (configured_device != dev) {
     // The warpgroups re-split the registers the CTA was launched with
     // (setmaxnreg): each SM sub-partition holds one control warp and two
-    // epilogue warps, so 3 x (launch registers) must cover 40 + 2 x 224.
+    // epilogue warps, so 3 x (launch registers) must cover 56 + 2 x 224.
     // Refuse to launch a build where that does not hold (it would wait forever).
     cudaFuncAttributes attr;
     cudaError_t e = cudaFuncGetAttributes(&attr, kern);
