@@ -41,6 +41,24 @@ GRAN_NAMES = {0: "tensor", 1: "row", 2: "block"}
 GEMM_TRAFFIC = {"workload": "grpo_8b", "bytes": 5.56e9, "gemm_cu_sha256_prefix": "5829fd7ed9aae213"}
 
 
+def max_over_ranks(values, world, device="cpu"):
+    """Per-rank timings -> their maxima over all ranks: a job of N replicas is as
+    slow as its slowest rank.  One process per GPU, NCCL on the GPU machine; the same
+    code runs over gloo on CPU in the tests."""
+    if world <= 1:
+        return [float(v) for v in values]
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(x) for x in t.cpu()]
+
+
+def whole_job_rate(units_per_rank, world, ms):
+    """Units processed by all ranks per second, from the max-over-ranks time."""
+    return world * units_per_rank / (ms * 1e-3)
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -216,6 +234,8 @@ def run_ours(args, rank, world, local_rank):
         per_step_events.append(list(ev))
     t1.record(stream)
     torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
     stage = np.zeros(6)
     for evs in per_step_events:
         stage += [evs[i].elapsed_time(evs[i + 1]) for i in range(6)]
@@ -260,6 +280,8 @@ def run_ours(args, rank, world, local_rank):
     for _ in range(max(1, args.warmup)):
         e2e_step()
     torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
@@ -267,6 +289,8 @@ def run_ours(args, rank, world, local_rank):
         e2e_step()
     e1.record(stream)
     torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
     e2e_ms = e0.elapsed_time(e1) / args.steps
     api.check()
     res = api.read_calib_result(b.cal_res)
@@ -280,10 +304,7 @@ def run_ours(args, rank, world, local_rank):
     api.check()
 
     ms = elapsed_ms / args.steps
-    if world > 1:
-        t = torch.tensor([ms, e2e_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms, e2e_ms = float(t[0]), float(t[1])
+    ms, e2e_ms = max_over_ranks([ms, e2e_ms], world, dev)
     if rank != 0:
         return None
     stage /= args.steps
@@ -294,7 +315,7 @@ def run_ours(args, rank, world, local_rank):
     achieved = flops / (gemm_ms * 1e-3) / 1e12
     line = {
         "metric": METRIC,
-        "value": world * T / (ms * 1e-3),
+        "value": whole_job_rate(T, world, ms),
         "unit": "tokens/s",
         "n_gpus": world,
         "steps": args.steps,
@@ -324,7 +345,7 @@ def run_ours(args, rank, world, local_rank):
                         "ms_per_step_amortised_1_in_20": ms + shadow_ms / 20,
                         "note": "BF16 reference scoring of the same tokens (Algorithm 1 needs r_BF16); "
                                 "the paper recomputes it every 20 steps"},
-        "e2e": {"value": world * T / (e2e_ms * 1e-3), "unit": "tokens/s",
+        "e2e": {"value": whole_job_rate(T, world, e2e_ms), "unit": "tokens/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "note": "h, targets, logp_old, r_bf16, adv, mask, coef copied in; stats, bounds, "
                         "dloss/dlogp read back; lm_head W is resident model state"},
