@@ -8,9 +8,10 @@
 //               swizzle, 4-stage shared-memory ring guarded by mbarriers;
 //   warp 1      MMA issuer: tcgen05.mma kind::f8f6f4 M=128 N=256 K=32, fp32
 //               accumulator in TMEM (two 256-column buffers);
-//   warp 2      block scaling only: stages each K block's activation and
-//               weight scales into a shared-memory ring, so the epilogue never
-//               waits on global loads;
+//   warp 2      block scaling only: stages the activation and weight scales
+//               of four K blocks per slot into a shared-memory ring, so the
+//               epilogue never waits on global loads and meets one barrier per
+//               four K blocks;
 //   warp 3      idle (it completes the first warpgroup, whose register budget
 //               is lowered to 56 so the epilogue can hold 224);
 //   warps 4..11 epilogue: tcgen05.ld of the accumulator, one thread per token
@@ -25,8 +26,8 @@
 // stage, so the shared-memory layout is the FP8 one) and no scales.  Block scales (1x128 for h,
 // 128x128 for W) change every 128-wide K block: the MMA writes each K block's
 // partial product into one of the two TMEM buffers and the epilogue promotes
-// it, acc += S_h[t][kb] S_W[vb][kb] * partial, into registers while the MMA
-// fills the other buffer.
+// it, acc += S_h[t][kb] S_W[vb][kb] * partial, into registers (packed f32x2
+// FMAs) while the MMA fills the other buffer.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -54,8 +55,10 @@ constexpr uint32_t A_BYTES = BM * BK;
 constexpr uint32_t B_BYTES = BN * BK;
 constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr uint32_t TMEM_COLS = 2 * BN;
-constexpr int SC_SLOTS = 8;                       // scale ring depth (K blocks)
-constexpr uint32_t SC_SLOT_FLOATS = BM + 4;       // 128 activation + 2 weight (+2 pad)
+constexpr int SC_SLOTS = 4;                       // scale ring depth (slots)
+constexpr int SC_KB = 4;                          // K blocks per slot
+constexpr uint32_t SC_KB_FLOATS = BM + 4;         // 128 activation + 2 weight (+2 pad)
+constexpr uint32_t SC_SLOT_FLOATS = SC_KB * SC_KB_FLOATS;
 constexpr uint32_t SC_BYTES = SC_SLOTS * SC_SLOT_FLOATS * 4;
 constexpr size_t SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + SC_BYTES + 512;
 constexpr float kLog2e = 1.4426950408889634f;
@@ -263,20 +266,24 @@ __global__ void __launch_bounds__(THREADS, 1)
       tile_coords(tile, p, m_blk, n_blk);
       const int m0 = m_blk * BM;
       const int wb0 = 2 * n_blk;
-      for (int kb = 0; kb < p.num_kb; ++kb) {
+      for (int kg = 0; kg < p.num_kb; kg += SC_KB) {
         ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&sc_empty[slot]), sphase ^ 1, lim, abort_flag));
         if (!ok) break;
-        const uint32_t dst = smem_u32(sc_ring + slot * SC_SLOT_FLOATS);
-        const float* src = p.a_scales + static_cast<size_t>(kb) * p.M;
-        // asynchronous 4-byte copies: the warp never waits for the data, the
-        // barrier completes when every lane's copies have landed
+        const int nkb = min(SC_KB, p.num_kb - kg);
+        for (int q = 0; q < nkb; ++q) {
+          const int kb = kg + q;
+          const uint32_t dst = smem_u32(sc_ring + slot * SC_SLOT_FLOATS + q * SC_KB_FLOATS);
+          const float* src = p.a_scales + static_cast<size_t>(kb) * p.M;
+          // asynchronous 4-byte copies: the warp never waits for the data, the
+          // barrier completes when every lane's copies have landed
 #pragma unroll
-        for (int j = 0; j < BM / 32; ++j) {
-          const int r = m0 + j * 32 + lane;
-          if (r < p.M) cp_async_4(dst + (j * 32 + lane) * 4, src + r);
+          for (int j = 0; j < BM / 32; ++j) {
+            const int r = m0 + j * 32 + lane;
+            if (r < p.M) cp_async_4(dst + (j * 32 + lane) * 4, src + r);
+          }
+          if (lane < 2 && wb0 + lane < p.n_chunks)
+            cp_async_4(dst + (BM + lane) * 4, p.b_scales + static_cast<size_t>(wb0 + lane) * p.num_kb + kb);
         }
-        if (lane < 2 && wb0 + lane < p.n_chunks)
-          cp_async_4(dst + (BM + lane) * 4, p.b_scales + static_cast<size_t>(wb0 + lane) * p.num_kb + kb);
         cp_async_mbar_arrive(smem_u32(&sc_full[slot]));
         if (++slot == SC_SLOTS) {
           slot = 0;
@@ -372,16 +379,22 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
         for (int i = 0; i < CHUNK / 2; ++i) z2[i] = make_float2(0.f, 0.f);
         for (int kb = 0; kb < p.num_kb; ++kb) {
-          // this K block's scales from the ring (staged by the loader warp)
-          ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&sc_full[sslot]), sphase, lim, abort_flag));
-          if (!ok) break;
-          const float* scs = sc_ring + sslot * SC_SLOT_FLOATS;
+          // this K block's scales from the ring (staged by the loader warp,
+          // SC_KB K blocks per slot: one barrier wait per slot)
+          const int q = kb % SC_KB;
+          if (q == 0) {
+            ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&sc_full[sslot]), sphase, lim, abort_flag));
+            if (!ok) break;
+          }
+          const float* scs = sc_ring + sslot * SC_SLOT_FLOATS + q * SC_KB_FLOATS;
           const float sc = scs[rit] * scs[BM + half];
-          __syncwarp();
-          if (lane == 0) mbar_arrive(smem_u32(&sc_empty[sslot]));
-          if (++sslot == SC_SLOTS) {
-            sslot = 0;
-            sphase ^= 1;
+          if (q == SC_KB - 1 || kb == p.num_kb - 1) {
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&sc_empty[sslot]));
+            if (++sslot == SC_SLOTS) {
+              sslot = 0;
+              sphase ^= 1;
+            }
           }
           ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&acc_full[ab]), aphase, lim, abort_flag));
           if (!ok) break;
@@ -405,10 +418,9 @@ __global__ void __launch_bounds__(THREADS, 1)
               if (lane == 0) mbar_arrive(smem_u32(&acc_empty[ab]));
             }
 #pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              z2[c * 16 + i].x = fmaf(__uint_as_float(cur[2 * i]), sc, z2[c * 16 + i].x);
-              z2[c * 16 + i].y = fmaf(__uint_as_float(cur[2 * i + 1]), sc, z2[c * 16 + i].y);
-            }
+            for (int i = 0; i < 16; ++i)
+              ffma2(z2[c * 16 + i].x, z2[c * 16 + i].y, __uint_as_float(cur[2 * i]),
+                    __uint_as_float(cur[2 * i + 1]), sc);
             if (c + 1 < CHUNK / 32) tmem_wait_ld(nxt);
           }
           ab ^= 1;
