@@ -20,6 +20,15 @@ Readings:
   tokens and 0 elsewhere.
 * w_t = 1 when no TIS weights are given.
 * Everything here is float64.
+
+Sequence-mean variant (GRPO's original normalisation, §2.1: the objective
+averages each response's token terms, 1/|o_i| sum_t, then the responses):
+
+    loss = (1/S) sum_{i : n_i > 0} (1/n_i) sum_{t in i, valid} l_t
+
+with n_i the valid tokens of sequence i and S the sequences that have any;
+g_t = -w_t A_t r_t / (S n_i) on unclipped valid tokens.  A sequence is the
+set of tokens with the same id (they need not be contiguous).
 """
 
 import numpy as np
@@ -74,3 +83,37 @@ def clipped_surrogate(r, adv, mask, w, lo, hi):
         "clip_frac_neg": c_neg / n_neg if n_neg else 0.0,
         "clip_frac": (c_pos + c_neg) / n_valid if n_valid else 0.0,
     }
+
+
+def clipped_surrogate_seq_mean(r, adv, mask, w, lo, hi, seq_id, n_seq):
+    """Sequence-mean of per-sequence token means of the clipped surrogate.
+
+    Explicit per-sequence loop: the token terms, clip bits and counts are those
+    of ``clipped_surrogate``; only the normalisation differs."""
+    base = clipped_surrogate(r, adv, mask, w, lo, hi)
+    r64 = np.asarray(r, np.float32).astype(np.float64)
+    a64 = np.asarray(adv, np.float32).astype(np.float64)
+    w64 = np.ones_like(r64) if w is None else np.asarray(w, np.float32).astype(np.float64)
+    valid = _valid(mask, r64.size)
+    sid = np.asarray(seq_id, np.int64)
+    if np.any(sid < 0) or np.any(sid >= n_seq):
+        raise ValueError("sequence id outside [0, n_seq)")
+    clipped = base["clip_mask"] != 0
+    n_i = np.zeros(n_seq, np.int64)
+    for t in range(r64.size):
+        if valid[t]:
+            n_i[sid[t]] += 1
+    S = int(np.sum(n_i > 0))
+    seq_sums = np.zeros(n_seq)
+    for t in range(r64.size):
+        if valid[t]:
+            seq_sums[sid[t]] += base["terms"][t]
+    loss_sum = float(sum(seq_sums[i] / n_i[i] for i in range(n_seq) if n_i[i] > 0))
+    grad = np.zeros_like(r64)
+    for t in range(r64.size):
+        if valid[t] and not clipped[t]:
+            grad[t] = -w64[t] * a64[t] * r64[t] / (S * n_i[sid[t]])
+    out = dict(base)
+    out.update({"loss": loss_sum / S if S else 0.0, "loss_sum": loss_sum, "grad": grad,
+                "n_seq_valid": S, "seq_valid_tokens": n_i})
+    return out

@@ -86,3 +86,85 @@ def test_absent_mask_means_all_valid():
     out = S.clipped_surrogate(r, a, None, None, 0.8, 1.2)
     ref = S.clipped_surrogate(r, a, np.ones(3, np.uint8), None, 0.8, 1.2)
     assert out["n_valid"] == 3 and out["loss"] == ref["loss"]
+
+
+# ---- sequence-mean variant (GRPO's 1/|o_i| normalisation) -------------------
+
+def _seq_inputs(rng, T, n_seq, equal=False):
+    r = np.exp(rng.normal(0, 0.3, T)).astype(np.float32)
+    A = rng.normal(0, 1, T).astype(np.float32)
+    w = rng.uniform(0.5, 2.0, T).astype(np.float32)
+    if equal:
+        sid = np.repeat(np.arange(n_seq), T // n_seq)
+        m = np.ones(T, np.uint8)
+    else:
+        sid = rng.integers(0, n_seq, T)
+        m = (rng.random(T) < 0.8).astype(np.uint8)
+    return r, A, w, m, sid
+
+
+def test_seq_mean_equals_token_mean_for_equal_lengths():
+    rng = np.random.default_rng(20)
+    r, A, w, m, sid = _seq_inputs(rng, 120, 6, equal=True)
+    tok = S.clipped_surrogate(r, A, m, w, 0.8, 1.2)
+    seq = S.clipped_surrogate_seq_mean(r, A, m, w, 0.8, 1.2, sid, 6)
+    assert abs(seq["loss"] - tok["loss"]) < 1e-12
+    assert np.allclose(seq["grad"], tok["grad"], rtol=0, atol=1e-15)
+
+
+def test_seq_mean_single_sequence_and_hand_case():
+    rng = np.random.default_rng(21)
+    r, A, w, m, _ = _seq_inputs(rng, 50, 1)
+    tok = S.clipped_surrogate(r, A, m, w, 0.8, 1.2)
+    seq = S.clipped_surrogate_seq_mean(r, A, m, w, 0.8, 1.2, np.zeros(50, int), 1)
+    assert abs(seq["loss"] - tok["loss"]) < 1e-12
+    # two sequences, lengths 1 and 3, unclipped ratios 1, A = 1 / 2 / 3 / 6:
+    # terms -1 | -2, -3, -6 -> means -1 and -11/3 -> loss -(1 + 11/3)/2 = -7/3
+    one = np.ones(4, np.float32)
+    res = S.clipped_surrogate_seq_mean(one, np.float32([1, 2, 3, 6]), None, None, 0.8, 1.2,
+                                       [0, 1, 1, 1], 3)  # sequence 2 has no tokens
+    assert abs(res["loss"] - (-7.0 / 3.0)) < 1e-15 and res["n_seq_valid"] == 2
+    assert np.allclose(res["grad"], [-1.0 / 2, -2.0 / 6, -3.0 / 6, -6.0 / 6], rtol=0, atol=1e-15)
+
+
+def test_seq_mean_permutation_invariance_and_empty():
+    rng = np.random.default_rng(22)
+    r, A, w, m, sid = _seq_inputs(rng, 200, 17)
+    a = S.clipped_surrogate_seq_mean(r, A, m, w, 0.8, 1.2, sid, 17)
+    p = rng.permutation(200)
+    b = S.clipped_surrogate_seq_mean(r[p], A[p], m[p], w[p], 0.8, 1.2, sid[p], 17)
+    assert abs(a["loss"] - b["loss"]) < 1e-12
+    assert np.allclose(a["grad"][p], b["grad"], rtol=0, atol=1e-15)
+    e = S.clipped_surrogate_seq_mean(r, A, np.zeros(200, np.uint8), w, 0.8, 1.2, sid, 17)
+    assert e["loss"] == 0.0 and e["n_seq_valid"] == 0 and not np.any(e["grad"])
+    with pytest.raises(ValueError):
+        S.clipped_surrogate_seq_mean(r, A, m, w, 0.8, 1.2, np.full(200, 17), 17)
+
+
+def test_seq_mean_gradient_finite_difference():
+    # the oracle's g_t against a central difference of the float64 loss as a
+    # function of logp (r = exp(logp - logp_old)), away from the clip kinks
+    rng = np.random.default_rng(23)
+    T, n = 30, 4
+    lp_old = rng.normal(-3, 1, T)
+    lp = lp_old + rng.normal(0, 0.05, T)
+    A = rng.normal(0, 1, T)
+    sid = rng.integers(0, n, T)
+    m = (rng.random(T) < 0.8).astype(np.uint8)
+    lo, hi = 0.5, 2.0
+
+    def loss(x):
+        rr = np.exp(x - lp_old)
+        term = -np.minimum(rr * A, np.clip(rr, lo, hi) * A) * (m != 0)
+        cnt = np.bincount(sid, weights=(m != 0).astype(float), minlength=n)
+        sums = np.bincount(sid, weights=term, minlength=n)
+        keep = cnt > 0
+        return np.sum(sums[keep] / cnt[keep]) / keep.sum()
+
+    g = S.clipped_surrogate_seq_mean(np.exp(lp - lp_old), A, m, None, lo, hi, sid, n)["grad"]
+    h = 1e-7
+    for t in range(T):
+        e = np.zeros(T)
+        e[t] = h
+        fd = (loss(lp + e) - loss(lp - e)) / (2 * h)
+        assert abs(fd - g[t]) < 5e-6 * max(1.0, abs(fd)), t
