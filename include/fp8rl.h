@@ -289,7 +289,7 @@ typedef struct fp8rl_clip_stats {
   int64_t clipped_neg;   /* A < 0 and r <= L   */
   float lo, hi;          /* bounds used        */
   int32_t flags;         /* 1 = no valid token */
-  int32_t reserved;
+  int32_t n_seq_valid;   /* sequence-mean call: sequences with a valid token (S); else 0 */
 } fp8rl_clip_stats;
 
 #define FP8RL_CLIP_HI 1  /* clip-mask bit: A > 0 and r >= H */
@@ -315,6 +315,27 @@ fp8rl_status fp8rl_clipped_surrogate(const float* r, const float* adv, const uin
                                      const float* bounds, float* grad_logp, uint8_t* clip_mask,
                                      fp8rl_clip_stats* stats,
                                      void* workspace, size_t workspace_bytes, void* stream);
+
+/* The same surrogate with GRPO's per-response normalisation (§2.1: each
+ * response's token terms are averaged, 1/|o_i| sum_t, then the responses):
+ *   loss = (1/S) sum_{i : n_i > 0} (1/n_i) sum_{t in i, valid} l_t
+ *   g_t  = -w_t A_t r_t / (S n_i) on unclipped valid tokens, 0 elsewhere
+ * n_i = valid tokens of sequence i, S = sequences with n_i > 0 (written to
+ * stats->n_seq_valid); loss_sum = S * loss.  seq_id int32 [T] gives each
+ * token's sequence in [0, n_seq) (tokens of a sequence need not be
+ * contiguous); an id outside that range sets FP8RL_EDEVICE and the token counts
+ * nowhere.  Other arguments, outputs and the clip semantics are those of
+ * fp8rl_clipped_surrogate; the workspace size depends on n_seq. */
+size_t fp8rl_surrogate_seq_mean_workspace_size(int64_t T, int64_t n_seq);
+
+fp8rl_status fp8rl_clipped_surrogate_seq_mean(const float* r, const float* adv,
+                                              const uint8_t* mask, const float* w_tis,
+                                              const int32_t* seq_id, int64_t n_seq, int64_t T,
+                                              float lo, float hi, const float* bounds,
+                                              float* grad_logp, uint8_t* clip_mask,
+                                              fp8rl_clip_stats* stats,
+                                              void* workspace, size_t workspace_bytes,
+                                              void* stream);
 
 /* Dense dLoss/dlogits for selected rows (a verification and debugging path;
  * the hot path keeps the factored form above).  For i < n_rows, t = rows[i]:

@@ -51,7 +51,7 @@ class ClipStats(ctypes.Structure):
                 ("n_valid", ctypes.c_int64), ("n_pos", ctypes.c_int64), ("n_neg", ctypes.c_int64),
                 ("clipped_pos", ctypes.c_int64), ("clipped_neg", ctypes.c_int64),
                 ("lo", ctypes.c_float), ("hi", ctypes.c_float),
-                ("flags", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+                ("flags", ctypes.c_int32), ("n_seq_valid", ctypes.c_int32)]
 
 
 class ClipDiag(ctypes.Structure):
@@ -93,6 +93,9 @@ _SIGS = {
     "fp8rl_dlogits_workspace_size": (_sz, [_i64, _i64, _i64, _i]),
     "fp8rl_dlogits_rows": (_i, [_p, _p, _p, _p, _i, _i64, _i64, _i64, _p, _p, _p, _p, _i64, _p, _p,
                                 _sz, _p]),
+    "fp8rl_surrogate_seq_mean_workspace_size": (_sz, [_i64, _i64]),
+    "fp8rl_clipped_surrogate_seq_mean": (_i, [_p, _p, _p, _p, _p, _i64, _i64, _f, _f, _p, _p, _p, _p, _p,
+                                              _sz, _p]),
     "fp8rl_clip_diagnostics_workspace_size": (_sz, [_i64]),
     "fp8rl_clip_diagnostics": (_i, [_p, _p, _p, _p, _p, _p, _i64, _f, _f, _p, _p, _sz, _p]),
     "fp8rl_tis_weights": (_i, [_p, _p, _i64, _f, _p, _p]),
@@ -377,6 +380,32 @@ def clipped_surrogate(r, adv, mask=None, w_tis=None, lo=0.8, hi=1.2, bounds=None
     _ok(lib.fp8rl_clipped_surrogate(_ptr(r), _ptr(adv), _ptr(mask), _ptr(w_tis), T, lo, hi,
                                     _ptr(bounds), _ptr(grad), _ptr(cm), _ptr(stats), _ptr(workspace),
                                     workspace.numel(), _stream(stream)), "fp8rl_clipped_surrogate")
+    return {"stats": stats, "grad": grad, "clip_mask": cm}
+
+
+def clipped_surrogate_seq_mean(r, adv, seq_id, n_seq, mask=None, w_tis=None, lo=0.8, hi=1.2, bounds=None,
+                               want_grad=True, want_clip_mask=True, stats=None, workspace=None, out=None,
+                               stream=None):
+    """fp8rl_clipped_surrogate_seq_mean (GRPO per-response normalisation)
+    -> dict(stats=<device buffer>, grad, clip_mask)."""
+    T = r.numel()
+    dev = r.device
+    _dev(r, torch.float32, "r")
+    _dev(adv, torch.float32, "adv", T)
+    _dev(seq_id, torch.int32, "seq_id", T)
+    _dev(mask, torch.uint8, "mask", T)
+    _dev(w_tis, torch.float32, "w_tis", T)
+    _dev(bounds, torch.float32, "bounds", 2)
+    o = out or {}
+    grad = o.get("grad", torch.empty(T, dtype=torch.float32, device=dev)) if want_grad else None
+    cm = o.get("clip_mask", torch.empty(T, dtype=torch.uint8, device=dev)) if want_clip_mask else None
+    stats = torch.zeros(ctypes.sizeof(ClipStats), dtype=torch.uint8, device=dev) if stats is None else stats
+    if workspace is None:
+        workspace = _workspace(lib.fp8rl_surrogate_seq_mean_workspace_size(T, n_seq), dev)
+    _ok(lib.fp8rl_clipped_surrogate_seq_mean(_ptr(r), _ptr(adv), _ptr(mask), _ptr(w_tis), _ptr(seq_id),
+                                             n_seq, T, lo, hi, _ptr(bounds), _ptr(grad), _ptr(cm),
+                                             _ptr(stats), _ptr(workspace), workspace.numel(),
+                                             _stream(stream)), "fp8rl_clipped_surrogate_seq_mean")
     return {"stats": stats, "grad": grad, "clip_mask": cm}
 
 

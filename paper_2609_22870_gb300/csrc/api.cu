@@ -304,6 +304,24 @@ fp8rl_status fp8rl_clipped_surrogate(const float* r, const float* adv, const uin
   return e == cudaSuccess ? FP8RL_OK : cuda_fail(e);
 }
 
+size_t fp8rl_surrogate_seq_mean_workspace_size(int64_t T, int64_t n_seq) {
+  return (T < 0 || n_seq < 0) ? 0 : seq_surrogate_workspace_bytes(T, n_seq);
+}
+
+fp8rl_status fp8rl_clipped_surrogate_seq_mean(const float* r, const float* adv, const uint8_t* mask,
+                                              const float* w_tis, const int32_t* seq_id,
+                                              int64_t n_seq, int64_t T, float lo, float hi,
+                                              const float* bounds, float* grad, uint8_t* clip_mask,
+                                              fp8rl_clip_stats* stats, void* ws, size_t ws_bytes,
+                                              void* stream) {
+  if (!stats || (T > 0 && (!r || !adv || !seq_id))) return FP8RL_EINVAL;
+  if (T < 0 || n_seq < 0 || n_seq > 0x7FFFFFFF) return FP8RL_ESHAPE;
+  if (!ws || ws_bytes < seq_surrogate_workspace_bytes(T, n_seq)) return FP8RL_EWORKSPACE;
+  cudaError_t e = launch_seq_surrogate(r, adv, mask, w_tis, seq_id, n_seq, T, lo, hi, bounds, grad,
+                                       clip_mask, stats, ws, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? FP8RL_OK : cuda_fail(e);
+}
+
 // ------------------------------------------------------------------ diagnostics
 size_t fp8rl_clip_diagnostics_workspace_size(int64_t T) { return T < 0 ? 0 : diag_workspace_bytes(T); }
 

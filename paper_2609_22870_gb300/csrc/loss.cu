@@ -15,6 +15,12 @@
 // the float32 sum to within one rounding; partials meet in float64 through a
 // fixed-order reduction by the last block, so the loss is bit-reproducible for
 // a given T and launch.
+//
+// Sequence-mean variant (GRPO's per-response normalisation, §2.1): a count
+// pass gives each sequence's valid tokens n_i (atomics aggregated over a warp's
+// tokens of the same sequence) and, in its last block, S = #{i : n_i > 0}; the
+// fused pass then weights each term by 1/n_i and each gradient by 1/(S n_i):
+//   loss = (1/S) sum_i (1/n_i) sum_{t in i} l_t,   g_t = -w_t A_t r_t / (S n_i).
 #include "common.cuh"
 #include "internal.h"
 
@@ -198,12 +204,156 @@ __global__ void __launch_bounds__(kThreads) surrogate_kernel(
     s.lo = b.lo;
     s.hi = b.hi;
     s.flags = n_valid ? 0 : 1;
-    s.reserved = 0;
+    s.n_seq_valid = 0;
     *stats = s;
   }
 }
 
 bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+// ------------------------------------------------------------ sequence mean
+struct SeqWork {
+  unsigned long long n_valid;
+  unsigned int ticket;
+  unsigned int n_seq_valid;
+  unsigned int ticket2;
+  unsigned int pad[59];
+  Partial part[1];  // [grid]; the per-sequence counts follow the partials
+};
+
+size_t seq_counts_offset(int64_t T) {
+  return align_up(sizeof(SeqWork) + sizeof(Partial) * static_cast<size_t>(grid_of(T)), 256);
+}
+
+// n_i per sequence (warp-aggregated atomics), n_valid, and in the last block
+// S = #{i : n_i > 0}.  Tokens with an id outside [0, n_seq) flag bad input and
+// count nowhere.
+__global__ void __launch_bounds__(kThreads) seq_count_kernel(const uint8_t* __restrict__ mask,
+                                                             const int32_t* __restrict__ sid,
+                                                             int64_t T, int64_t n_seq,
+                                                             unsigned int* __restrict__ cnt,
+                                                             SeqWork* w) {
+  __shared__ bool last;
+  __shared__ unsigned int sh_s[kThreads / 32];
+  const int lane = threadIdx.x & 31;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  uint32_t nv = 0;
+  bool bad = false;
+  // warp-uniform loop: every lane takes part in the match of each step
+  for (int64_t base = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) - lane; base < T; base += stride) {
+    const int64_t t = base + lane;
+    int id = -1;
+    if (t < T && (!mask || mask[t] != 0)) {
+      id = sid[t];
+      if (id < 0 || id >= n_seq) {
+        bad = true;
+        id = -1;
+      }
+    }
+    nv += id >= 0;
+    const unsigned peers = __match_any_sync(0xffffffffu, id);
+    if (id >= 0 && lane == __ffs(peers) - 1) atomicAdd(&cnt[id], static_cast<unsigned>(__popc(peers)));
+  }
+  if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(&d_status, kErrDevice);
+  const uint32_t s = __reduce_add_sync(0xffffffffu, nv);
+  if (lane == 0 && s) atomicAdd(&w->n_valid, static_cast<unsigned long long>(s));
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) last = atomicAdd(&w->ticket, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  unsigned int k = 0;
+  for (int64_t i = threadIdx.x; i < n_seq; i += blockDim.x) k += (reinterpret_cast<volatile unsigned*>(cnt))[i] > 0;
+  k = __reduce_add_sync(0xffffffffu, k);
+  if (lane == 0) sh_s[threadIdx.x >> 5] = k;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned int S = 0;
+    for (int i = 0; i < kThreads / 32; ++i) S += sh_s[i];
+    w->n_seq_valid = S;
+  }
+}
+
+__global__ void __launch_bounds__(kThreads) seq_surrogate_kernel(
+    const float* __restrict__ r, const float* __restrict__ adv, const uint8_t* __restrict__ mask,
+    const float* __restrict__ wts, const int32_t* __restrict__ sid, int64_t T, int64_t n_seq,
+    const unsigned int* __restrict__ cnt, float lo_arg, float hi_arg, const float* __restrict__ bounds,
+    float* __restrict__ grad, uint8_t* __restrict__ clip_mask, fp8rl_clip_stats* __restrict__ stats,
+    SeqWork* w) {
+  __shared__ double sh_d[kThreads / 32];
+  __shared__ unsigned long long sh_u[kThreads / 32];
+  __shared__ bool last;
+  Bounds b;
+  b.lo = bounds ? bounds[0] : lo_arg;
+  b.hi = bounds ? bounds[1] : hi_arg;
+  const unsigned int S = w->n_seq_valid;
+  const float inv_s = S ? 1.0f / static_cast<float>(S) : 0.f;
+  Acc a;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < T; t += stride) {
+    const int id = sid[t];
+    const bool in = id >= 0 && id < n_seq;
+    const bool valid = in && (mask ? mask[t] != 0 : true);
+    const unsigned int ni = valid ? cnt[id] : 1u;
+    b.inv_n = inv_s / static_cast<float>(ni);  // 1 / (S n_i)
+    float g;
+    uint32_t cm;
+    const float l = token(r[t], adv[t], valid, wts ? wts[t] : 1.f, b, a, g, cm);
+    a.add(l / static_cast<float>(ni));
+    if (grad) grad[t] = g;
+    if (clip_mask) clip_mask[t] = static_cast<uint8_t>(cm);
+  }
+  const double loss = block_sum(static_cast<double>(a.s) + static_cast<double>(a.c), sh_d);
+  const unsigned long long n_pos = block_sum<unsigned long long>(a.n_pos, sh_u);
+  const unsigned long long n_neg = block_sum<unsigned long long>(a.n_neg, sh_u);
+  const unsigned long long c_pos = block_sum<unsigned long long>(a.c_pos, sh_u);
+  const unsigned long long c_neg = block_sum<unsigned long long>(a.c_neg, sh_u);
+  if (threadIdx.x == 0) {
+    Partial& p = w->part[blockIdx.x];
+    p.loss = loss;
+    p.n_pos = n_pos;
+    p.n_neg = n_neg;
+    p.c_pos = c_pos;
+    p.c_neg = c_neg;
+    __threadfence();
+    last = atomicAdd(&w->ticket2, 1u) == gridDim.x - 1;
+  }
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  double L = 0.0;
+  unsigned long long np = 0, nn = 0, cp = 0, cn = 0;
+  for (unsigned k = threadIdx.x; k < gridDim.x; k += kThreads) {
+    const volatile Partial& p = w->part[k];
+    L += p.loss;
+    np += p.n_pos;
+    nn += p.n_neg;
+    cp += p.c_pos;
+    cn += p.c_neg;
+  }
+  L = block_sum(L, sh_d);
+  np = block_sum(np, sh_u);
+  nn = block_sum(nn, sh_u);
+  cp = block_sum(cp, sh_u);
+  cn = block_sum(cn, sh_u);
+  if (threadIdx.x == 0) {
+    const unsigned long long n_valid = w->n_valid;
+    fp8rl_clip_stats s;
+    s.loss_sum = L;
+    s.loss = S ? L / static_cast<double>(S) : 0.0;
+    s.n_valid = static_cast<int64_t>(n_valid);
+    s.n_pos = static_cast<int64_t>(np);
+    s.n_neg = static_cast<int64_t>(nn);
+    s.clipped_pos = static_cast<int64_t>(cp);
+    s.clipped_neg = static_cast<int64_t>(cn);
+    s.lo = b.lo;
+    s.hi = b.hi;
+    s.flags = n_valid ? 0 : 1;
+    s.n_seq_valid = static_cast<int32_t>(S);
+    *stats = s;
+  }
+}
 
 }  // namespace
 
@@ -224,6 +374,27 @@ cudaError_t launch_surrogate(const float* r, const float* adv, const uint8_t* ma
                    aligned(mask, 4) && aligned(clip_mask, 4);
   surrogate_kernel<<<grid, kThreads, 0, s>>>(r, adv, mask, w, T, lo, hi, bounds, grad, clip_mask,
                                               stats, work, vec);
+  return cudaGetLastError();
+}
+
+size_t seq_surrogate_workspace_bytes(int64_t T, int64_t n_seq) {
+  return seq_counts_offset(T) + align_up(static_cast<size_t>(n_seq > 0 ? n_seq : 1) * 4, 256);
+}
+
+cudaError_t launch_seq_surrogate(const float* r, const float* adv, const uint8_t* mask,
+                                 const float* w, const int32_t* sid, int64_t n_seq, int64_t T,
+                                 float lo, float hi, const float* bounds, float* grad,
+                                 uint8_t* clip_mask, fp8rl_clip_stats* stats, void* ws,
+                                 cudaStream_t s) {
+  SeqWork* work = static_cast<SeqWork*>(ws);
+  unsigned int* cnt = reinterpret_cast<unsigned int*>(static_cast<char*>(ws) + seq_counts_offset(T));
+  cudaError_t e = cudaMemsetAsync(work, 0, sizeof(SeqWork), s);
+  if (e == cudaSuccess && n_seq > 0) e = cudaMemsetAsync(cnt, 0, static_cast<size_t>(n_seq) * 4, s);
+  if (e != cudaSuccess) return e;
+  const int grid = grid_of(T);
+  seq_count_kernel<<<grid, kThreads, 0, s>>>(mask, sid, T, n_seq, cnt, work);
+  seq_surrogate_kernel<<<grid, kThreads, 0, s>>>(r, adv, mask, w, sid, T, n_seq, cnt, lo, hi, bounds,
+                                                  grad, clip_mask, stats, work);
   return cudaGetLastError();
 }
 

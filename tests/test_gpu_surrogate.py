@@ -72,3 +72,60 @@ def test_surrogate_deterministic(cuda_lib):
     a = cuda_lib.read_clip_stats(cuda_lib.clipped_surrogate(r, adv, mask, w)["stats"])
     b = cuda_lib.read_clip_stats(cuda_lib.clipped_surrogate(r, adv, mask, w)["stats"])
     assert a["loss"] == b["loss"] and a["loss_sum"] == b["loss_sum"]
+
+
+# ---- sequence-mean variant ---------------------------------------------------
+
+def _seq_ids(T, n_seq, seed, contiguous=True):
+    g = torch.Generator().manual_seed(seed + 7)
+    if contiguous:  # packed responses of random lengths
+        cuts = torch.sort(torch.randint(0, T + 1, (n_seq - 1,), generator=g)).values
+        sid = torch.bucketize(torch.arange(T), cuts, right=True)
+    else:
+        sid = torch.randint(0, n_seq, (T,), generator=g)
+    return sid.to(torch.int32)
+
+
+def _check_seq(api, r, adv, mask, w, sid, n_seq, lo, hi):
+    d = [None if t is None else t.cuda() for t in (r, adv, sid, mask, w)]
+    out = api.clipped_surrogate_seq_mean(d[0], d[1], d[2], n_seq, mask=d[3], w_tis=d[4], lo=lo, hi=hi)
+    api.check()
+    st = api.read_clip_stats(out["stats"])
+    ref = OS.clipped_surrogate_seq_mean(r.numpy(), adv.numpy(), None if mask is None else mask.numpy(),
+                                        None if w is None else w.numpy(), lo, hi, sid.numpy(), n_seq)
+    assert np.array_equal(out["clip_mask"].cpu().numpy(), ref["clip_mask"])
+    for k in ("n_valid", "n_pos", "n_neg", "clipped_pos", "clipped_neg", "n_seq_valid"):
+        assert st[k] == ref[k], k
+    n = max(1, ref["n_valid"])
+    scale = max(abs(ref["loss"]), np.sum(np.abs(ref["terms"])) / n, 1e-300)
+    assert abs(st["loss"] - ref["loss"]) <= 1e-4 * scale
+    g = out["grad"].cpu().numpy().astype(np.float64)
+    assert np.all(np.abs(g - ref["grad"]) <= 1e-6 * np.abs(ref["grad"]) + 1e-30)
+    assert np.all(g[ref["grad"] == 0] == 0)
+    return st
+
+
+@pytest.mark.parametrize("T,n_seq", [(1, 1), (100, 7), (5000, 32), (65536, 128), (131072, 8)])
+@pytest.mark.parametrize("contiguous", [True, False])
+def test_seq_mean_parity(cuda_lib, T, n_seq, contiguous):
+    r, adv, mask, w = _inputs(T, T + n_seq)
+    _check_seq(cuda_lib, r, adv, mask, w, _seq_ids(T, n_seq, T, contiguous), n_seq, 0.8, 1.2)
+
+
+def test_seq_mean_equal_lengths_match_token_mean_and_empty(cuda_lib):
+    T, n_seq = 4096, 8
+    r, adv, _, w = _inputs(T, 5)
+    sid = torch.arange(T, dtype=torch.int32) // (T // n_seq)
+    st = _check_seq(cuda_lib, r, adv, None, w, sid, n_seq, 0.8, 1.2)
+    tok = cuda_lib.read_clip_stats(cuda_lib.clipped_surrogate(r.cuda(), adv.cuda(), None, w.cuda())["stats"])
+    assert abs(st["loss"] - tok["loss"]) <= 1e-5 * max(abs(tok["loss"]), 1e-6)
+    st0 = _check_seq(cuda_lib, r, adv, torch.zeros(T, dtype=torch.uint8), w, sid, n_seq + 3, 0.8, 1.2)
+    assert st0["loss"] == 0 and st0["n_seq_valid"] == 0 and st0["flags"] == 1
+
+
+def test_seq_mean_bad_ids_flagged(cuda_lib):
+    r, adv, mask, w = (t.cuda() for t in _inputs(300, 6))
+    sid = torch.zeros(300, dtype=torch.int32, device="cuda")
+    sid[17] = 5  # n_seq = 5: out of range
+    cuda_lib.clipped_surrogate_seq_mean(r, adv, sid, 5, mask=mask, w_tis=w)
+    assert cuda_lib.check_status() == cuda_lib.EDEVICE
