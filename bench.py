@@ -537,6 +537,19 @@ def run_kernel_rooflines(args, local_rank):
     ms = timed(lambda: api.clipped_surrogate(r_fp, adv, mask, None, 0.8, 1.2, None, stats=st, workspace=sws,
                                              out={"grad": grad, "clip_mask": cm}), 10)
     line("clipped surrogate", [T], T * (4 + 4 + 1 + 4 + 1), ms)
+    n_seq = T // 512
+    sid = (torch.arange(T, device=dev, dtype=torch.int64) // 512).to(torch.int32)
+    qws = torch.empty(api.lib.fp8rl_surrogate_seq_mean_workspace_size(T, n_seq), dtype=torch.uint8, device=dev)
+    ms = timed(lambda: api.clipped_surrogate_seq_mean(r_fp, adv, sid, n_seq, mask, None, 0.8, 1.2, stats=st,
+                                                      workspace=qws, out={"grad": grad, "clip_mask": cm}), 10)
+    line("clipped surrogate, sequence mean", [T], T * (5 + 4 + 4 + 4 + 1 + 4 + 1), ms)
+    del qws, sid
+    lp8 = torch.log(r_fp)
+    lpb = torch.log(r_bf)
+    dbuf = torch.zeros(256, dtype=torch.uint8, device=dev)
+    dws = torch.empty(api.lib.fp8rl_clip_diagnostics_workspace_size(T), dtype=torch.uint8, device=dev)
+    ms = timed(lambda: api.clip_diagnostics(r_fp, r_bf, adv, mask, lp8, lpb, 0.2, 0.2, out=dbuf, workspace=dws), 10)
+    line("over-clip / NMAE diagnostics", [T], T * (4 * 5 + 1), ms)
     return out
 
 

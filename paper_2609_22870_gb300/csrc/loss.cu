@@ -18,7 +18,7 @@
 //
 // Sequence-mean variant (GRPO's per-response normalisation, §2.1): a count
 // pass gives each sequence's valid tokens n_i (atomics aggregated over a warp's
-// tokens of the same sequence) and, in its last block, S = #{i : n_i > 0}; the
+// tokens of the same sequence) and S = #{i : n_i > 0}; the
 // fused pass then weights each term by 1/n_i and each gradient by 1/(S n_i):
 //   loss = (1/S) sum_i (1/n_i) sum_{t in i} l_t,   g_t = -w_t A_t r_t / (S n_i).
 #include "common.cuh"
@@ -225,54 +225,75 @@ size_t seq_counts_offset(int64_t T) {
   return align_up(sizeof(SeqWork) + sizeof(Partial) * static_cast<size_t>(grid_of(T)), 256);
 }
 
-// n_i per sequence (warp-aggregated atomics), n_valid, and in the last block
-// S = #{i : n_i > 0}.  Tokens with an id outside [0, n_seq) flag bad input and
+// n_i per sequence, n_valid and S = #{i : n_i > 0} (counted by the atomics
+// that find a sequence's count still zero).  Each
+// warp walks its own contiguous range of tokens 32 at a time and carries the
+// count of the sequence it is in across steps (responses are usually
+// contiguous), so a sequence costs one atomic per warp that touches it rather
+// than one per step.  Tokens with an id outside [0, n_seq) flag bad input and
 // count nowhere.
 __global__ void __launch_bounds__(kThreads) seq_count_kernel(const uint8_t* __restrict__ mask,
                                                              const int32_t* __restrict__ sid,
                                                              int64_t T, int64_t n_seq,
                                                              unsigned int* __restrict__ cnt,
                                                              SeqWork* w) {
-  __shared__ bool last;
-  __shared__ unsigned int sh_s[kThreads / 32];
   const int lane = threadIdx.x & 31;
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const int64_t nwarps = static_cast<int64_t>(gridDim.x) * (kThreads / 32);
+  const int64_t wid = static_cast<int64_t>(blockIdx.x) * (kThreads / 32) + (threadIdx.x >> 5);
+  const int64_t per = ((T + nwarps - 1) / nwarps + 127) / 128 * 128;
+  const int64_t beg = wid * per, end = min(T, beg + per);
   uint32_t nv = 0;
   bool bad = false;
-  // warp-uniform loop: every lane takes part in the match of each step
-  for (int64_t base = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) - lane; base < T; base += stride) {
-    const int64_t t = base + lane;
-    int id = -1;
-    if (t < T && (!mask || mask[t] != 0)) {
-      id = sid[t];
-      if (id < 0 || id >= n_seq) {
-        bad = true;
-        id = -1;
+  int cur_id = -1;        // warp-uniform: the sequence being counted and its count
+  unsigned cur_cnt = 0;
+  unsigned s_new = 0;     // lane 0: sequences this warp found empty
+  for (int64_t base = beg; base < end; base += 128) {
+    // four steps of 32 tokens: all loads issued before any is used
+    int idv[4];
+    bool on[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int64_t t = base + u * 32 + lane;
+      idv[u] = t < end ? __ldg(sid + t) : -1;
+      on[u] = t < end && (!mask || __ldg(mask + t) != 0);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      // runs of equal (raw) ids among the 32 tokens, in lane order; masked
+      // tokens keep their id, so padding inside a response does not split its
+      // run, and each run adds the number of its valid tokens
+      const int id = idv[u];
+      const bool in_range = id >= 0 && id < n_seq;
+      const bool valid = on[u] && in_range;
+      if (base + u * 32 + lane < end && !in_range) bad = true;  // masked tokens too
+      nv += valid;
+      const unsigned vbits = __ballot_sync(0xffffffffu, valid);
+      const int prev = __shfl_up_sync(0xffffffffu, id, 1);
+      unsigned heads = __ballot_sync(0xffffffffu, lane == 0 || id != prev);
+      while (heads) {
+        const int h = __ffs(heads) - 1;
+        heads &= heads - 1;
+        const int next = heads ? __ffs(heads) - 1 : 32;
+        const unsigned run = (next == 32 ? 0xffffffffu : ((1u << next) - 1u)) & ~((1u << h) - 1u);
+        const unsigned n = __popc(vbits & run);
+        if (n == 0) continue;  // no valid token in this run
+        const int run_id = __shfl_sync(0xffffffffu, id, h);
+        if (run_id == cur_id) {
+          cur_cnt += n;
+        } else {
+          if (cur_id >= 0 && lane == 0) s_new += atomicAdd(&cnt[cur_id], cur_cnt) == 0u;
+          cur_id = run_id;
+          cur_cnt = n;
+        }
       }
     }
-    nv += id >= 0;
-    const unsigned peers = __match_any_sync(0xffffffffu, id);
-    if (id >= 0 && lane == __ffs(peers) - 1) atomicAdd(&cnt[id], static_cast<unsigned>(__popc(peers)));
   }
+  if (cur_id >= 0 && lane == 0) s_new += atomicAdd(&cnt[cur_id], cur_cnt) == 0u;
   if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(&d_status, kErrDevice);
   const uint32_t s = __reduce_add_sync(0xffffffffu, nv);
   if (lane == 0 && s) atomicAdd(&w->n_valid, static_cast<unsigned long long>(s));
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) last = atomicAdd(&w->ticket, 1u) == gridDim.x - 1;
-  __syncthreads();
-  if (!last) return;
-  __threadfence();
-  unsigned int k = 0;
-  for (int64_t i = threadIdx.x; i < n_seq; i += blockDim.x) k += (reinterpret_cast<volatile unsigned*>(cnt))[i] > 0;
-  k = __reduce_add_sync(0xffffffffu, k);
-  if (lane == 0) sh_s[threadIdx.x >> 5] = k;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    unsigned int S = 0;
-    for (int i = 0; i < kThreads / 32; ++i) S += sh_s[i];
-    w->n_seq_valid = S;
-  }
+  // S: the atomics that found a sequence's count still zero
+  if (lane == 0 && s_new) atomicAdd(&w->n_seq_valid, s_new);
 }
 
 __global__ void __launch_bounds__(kThreads) seq_surrogate_kernel(
@@ -280,7 +301,7 @@ __global__ void __launch_bounds__(kThreads) seq_surrogate_kernel(
     const float* __restrict__ wts, const int32_t* __restrict__ sid, int64_t T, int64_t n_seq,
     const unsigned int* __restrict__ cnt, float lo_arg, float hi_arg, const float* __restrict__ bounds,
     float* __restrict__ grad, uint8_t* __restrict__ clip_mask, fp8rl_clip_stats* __restrict__ stats,
-    SeqWork* w) {
+    SeqWork* w, bool vec) {
   __shared__ double sh_d[kThreads / 32];
   __shared__ unsigned long long sh_u[kThreads / 32];
   __shared__ bool last;
@@ -290,17 +311,35 @@ __global__ void __launch_bounds__(kThreads) seq_surrogate_kernel(
   const unsigned int S = w->n_seq_valid;
   const float inv_s = S ? 1.0f / static_cast<float>(S) : 0.f;
   Acc a;
+  const int64_t tid = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < T; t += stride) {
-    const int id = sid[t];
-    const bool in = id >= 0 && id < n_seq;
-    const bool valid = in && (mask ? mask[t] != 0 : true);
-    const unsigned int ni = valid ? cnt[id] : 1u;
-    b.inv_n = inv_s / static_cast<float>(ni);  // 1 / (S n_i)
+  // one token: 1/n_i (correctly rounded) scales its term, and 1/(S n_i) its gradient
+  auto one = [&](float rt, float at, bool present, float wt, int id, float& g, uint32_t& cm) {
+    const bool valid = present && id >= 0 && id < n_seq;
+    const float inv_ni = valid ? __frcp_rn(static_cast<float>(__ldg(cnt + id))) : 1.f;
+    b.inv_n = inv_s * inv_ni;
+    a.add(token(rt, at, valid, wt, b, a, g, cm) * inv_ni);
+  };
+  const int64_t T4 = vec ? T / 4 : 0;
+  for (int64_t i = tid; i < T4; i += stride) {
+    const float4 rv = __ldg(reinterpret_cast<const float4*>(r) + i);
+    const float4 av = __ldg(reinterpret_cast<const float4*>(adv) + i);
+    const int4 iv = __ldg(reinterpret_cast<const int4*>(sid) + i);
+    const float4 wv = wts ? __ldg(reinterpret_cast<const float4*>(wts) + i) : make_float4(1.f, 1.f, 1.f, 1.f);
+    const uint32_t mv = mask ? __ldg(reinterpret_cast<const uint32_t*>(mask) + i) : 0x01010101u;
+    float4 gv;
+    uint32_t c0, c1, c2, c3;
+    one(rv.x, av.x, (mv & 0xFFu) != 0, wv.x, iv.x, gv.x, c0);
+    one(rv.y, av.y, (mv & 0xFF00u) != 0, wv.y, iv.y, gv.y, c1);
+    one(rv.z, av.z, (mv & 0xFF0000u) != 0, wv.z, iv.z, gv.z, c2);
+    one(rv.w, av.w, (mv & 0xFF000000u) != 0, wv.w, iv.w, gv.w, c3);
+    if (grad) reinterpret_cast<float4*>(grad)[i] = gv;
+    if (clip_mask) reinterpret_cast<uint32_t*>(clip_mask)[i] = c0 | (c1 << 8) | (c2 << 16) | (c3 << 24);
+  }
+  for (int64_t t = T4 * 4 + tid; t < T; t += stride) {
     float g;
     uint32_t cm;
-    const float l = token(r[t], adv[t], valid, wts ? wts[t] : 1.f, b, a, g, cm);
-    a.add(l / static_cast<float>(ni));
+    one(r[t], adv[t], mask ? mask[t] != 0 : true, wts ? wts[t] : 1.f, sid[t], g, cm);
     if (grad) grad[t] = g;
     if (clip_mask) clip_mask[t] = static_cast<uint8_t>(cm);
   }
@@ -393,8 +432,10 @@ cudaError_t launch_seq_surrogate(const float* r, const float* adv, const uint8_t
   if (e != cudaSuccess) return e;
   const int grid = grid_of(T);
   seq_count_kernel<<<grid, kThreads, 0, s>>>(mask, sid, T, n_seq, cnt, work);
+  const bool vec = aligned(r, 16) && aligned(adv, 16) && aligned(sid, 16) && aligned(w, 16) &&
+                   aligned(grad, 16) && aligned(mask, 4) && aligned(clip_mask, 4);
   seq_surrogate_kernel<<<grid, kThreads, 0, s>>>(r, adv, mask, w, sid, T, n_seq, cnt, lo, hi, bounds,
-                                                  grad, clip_mask, stats, work);
+                                                  grad, clip_mask, stats, work, vec);
   return cudaGetLastError();
 }
 
