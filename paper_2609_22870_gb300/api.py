@@ -501,6 +501,45 @@ class StepBuffers:
         self.clip_mask = torch.empty(T, dtype=torch.uint8, device=device)
 
 
+class HostBatchPrefetcher:
+    """Double-buffered host -> device staging of each step's inputs on a side
+    stream, so the copy of step i + 1 overlaps the work of step i (the batch
+    prefetch of a training loop).  Copies and stream events only.
+
+    ``host`` maps names to pinned CPU tensors; ``prefetch(slot, host)`` copies
+    them into device slot ``slot`` (0 or 1) once that slot's previous user has
+    released it; ``acquire(slot)`` makes the compute stream wait for the copy
+    and returns the slot's device tensors; ``release(slot)`` marks them free
+    after the work queued so far on the compute stream."""
+
+    def __init__(self, host, device, stream=None):
+        self.device = torch.device(device)
+        self.bufs = [{k: torch.empty(v.shape, dtype=v.dtype, device=self.device) for k, v in host.items()}
+                     for _ in range(2)]
+        self.copy_stream = torch.cuda.Stream(self.device)
+        self.copied = [torch.cuda.Event() for _ in range(2)]
+        self.released = [torch.cuda.Event() for _ in range(2)]
+        self.stream = stream
+
+    def _compute_stream(self):
+        return torch.cuda.current_stream(self.device) if self.stream is None else self.stream
+
+    def prefetch(self, slot, host):
+        cs = self.copy_stream
+        cs.wait_event(self.released[slot])  # a never-recorded event is already complete
+        with torch.cuda.stream(cs):
+            for k, v in host.items():
+                self.bufs[slot][k].copy_(v, non_blocking=True)
+        self.copied[slot].record(cs)
+
+    def acquire(self, slot):
+        self._compute_stream().wait_event(self.copied[slot])
+        return self.bufs[slot]
+
+    def release(self, slot):
+        self.released[slot].record(self._compute_stream())
+
+
 def score_calibrate_loss(h, W, targets, logp_old, r_bf16, adv, mask, coef, gran, eps_low, eps_high,
                          opts=None, buffers=None, stream=None):
     """One pass of the whole hot path through the C ABI, in order:

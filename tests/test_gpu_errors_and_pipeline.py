@@ -2,6 +2,7 @@
 whole hot path in one call sequence (properties that hold at any size)."""
 
 import ctypes
+import dataclasses
 
 import numpy as np
 import pytest
@@ -139,3 +140,48 @@ def test_pipeline_full_size(cuda_lib, name):
     res = api.read_calib_result(b.cal_res)
     st = api.read_clip_stats(b.stats)
     _pipeline_properties(res, st, b, adv.numpy(), mask.numpy(), r_bf16.float().numpy(), w)
+
+
+def test_prefetched_steps_match_direct_steps(cuda_lib):
+    """Steps fed by the double-buffered host prefetcher (copies of step i + 1
+    overlapping step i on a side stream) give the same results as direct
+    steps: the copies are ordered before their use and after the slot's
+    previous user."""
+    api = cuda_lib
+    w = synth.scaled(synth.WORKLOADS["grpo_8b"], T=4096, H=512, V=3000, name="pf")
+    W = synth.lm_head_weight(w, "cuda")
+    hosts = []
+    for k in range(3):  # three different batches
+        wk = synth.scaled(synth.WORKLOADS["grpo_8b"], T=4096, H=512, V=3000, name=f"pf{k}")
+        wk = dataclasses.replace(wk, seed=100 + k)
+        adv, mask = synth.rollout(wk)
+        noise = synth.old_policy_noise(wk)
+        lpo = (torch.full((w.T,), -8.0) + noise).float()
+        hosts.append({"h": synth.hidden_states(wk, "cpu").pin_memory(), "y": synth.targets(wk, "cpu").pin_memory(),
+                      "logp_old": lpo.pin_memory(), "r_bf16": torch.exp(-noise).float().pin_memory(),
+                      "adv": adv.pin_memory(), "mask": mask.pin_memory(),
+                      "coef": torch.exp(lpo).pin_memory()})
+    stream = torch.cuda.current_stream()
+    direct = []
+    for hb in hosts:
+        d = {k: v.cuda() for k, v in hb.items()}
+        b = api.score_calibrate_loss(d["h"], W, d["y"], d["logp_old"], d["r_bf16"], d["adv"], d["mask"],
+                                     d["coef"], w.gran, w.eps_low, w.eps_high)
+        api.check()
+        direct.append((api.read_calib_result(b.cal_res), b.grad.cpu().clone()))
+    pf = api.HostBatchPrefetcher(hosts[0], "cuda", stream)
+    b = api.StepBuffers(w.T, w.H, w.V, w.gran, "cuda")
+    got = []
+    pf.prefetch(0, hosts[0])
+    for i in range(3):
+        d = pf.acquire(i % 2)
+        if i + 1 < 3:
+            pf.prefetch((i + 1) % 2, hosts[i + 1])
+        api.score_calibrate_loss(d["h"], W, d["y"], d["logp_old"], d["r_bf16"], d["adv"], d["mask"], d["coef"],
+                                 w.gran, w.eps_low, w.eps_high, None, b, stream)
+        pf.release(i % 2)
+        api.check()
+        got.append((api.read_calib_result(b.cal_res), b.grad.cpu().clone()))
+    for (r0, g0), (r1, g1) in zip(direct, got):
+        assert r0 == r1
+        assert torch.equal(g0, g1)
