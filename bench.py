@@ -43,7 +43,7 @@ GEMM_TRAFFIC = {"workload": "grpo_8b", "bytes": 1.478e9, "gemm_cu_sha256_prefix"
 
 def max_over_ranks(values, world, device="cpu"):
     """Per-rank timings -> their maxima over all ranks: a job of N replicas is as
-    slow as its slowest rank.  One process per GPU, NCCL on the GPU machine; the same
+    slow as its slowest rank.  One process per GPU with NCCL on GPUs; the same
     code runs over gloo on CPU in the tests."""
     if world <= 1:
         return [float(v) for v in values]

@@ -1,5 +1,5 @@
 """The N > 1 bench path on CPU: two gloo ranks (127.0.0.1) run the replica
-timing reduction bench.py uses on the GPU machine over NCCL, and a non-zero rank
+timing reduction bench.py uses over NCCL on GPUs, and a non-zero rank
 of the reference arm exits without work or output.
 
 The path itself has no data-path collective (each GPU scores its own replica
