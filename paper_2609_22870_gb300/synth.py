@@ -117,11 +117,16 @@ def targets(w, device="cpu"):
     return torch.randint(0, w.V, (w.T,), generator=g, dtype=torch.int64).to(torch.int32).to(device)
 
 
-def rollout(w):
-    """(adv float32 [T], mask uint8 [T]) for the workload's group layout (CPU)."""
+def rollout(w, force_equal_prompt=None):
+    """(adv float32 [T], mask uint8 [T]) for the workload's group layout (CPU).
+
+    ``force_equal_prompt``: index of a prompt whose responses all get reward 1
+    (an all-equal group, for tests of the DAPO dynamic-sampling filter)."""
     g = _gen(w.seed * 10 + 4, "cpu")
     n_resp = w.prompts * w.group
     R = (torch.rand(w.prompts, w.group, generator=g, dtype=torch.float64) < w.reward_p).double()
+    if force_equal_prompt is not None:
+        R[force_equal_prompt] = 1.0
     mean = R.mean(dim=1, keepdim=True)
     std = R.std(dim=1, keepdim=True) if w.group > 1 else torch.zeros_like(mean)
     A = ((R - mean) / (std + 1e-6)).float().reshape(n_resp)

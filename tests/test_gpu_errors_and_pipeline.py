@@ -101,6 +101,34 @@ def test_pipeline_small(cuda_lib, name, T, H, V):
     _pipeline_properties(res, st, b, adv.numpy(), mask.numpy(), r_bf16, w)
 
 
+def test_pipeline_dapo_filter_with_forced_all_equal_group(cuda_lib):
+    """DAPO workload with one group forced to all-equal rewards: the dynamic-
+    sampling filter masks it, and no stage counts, clips or differentiates it."""
+    api = cuda_lib
+    w = dataclasses.replace(synth.WORKLOADS["dapo_32b"], name="dapo_forced", T=3 * 16 * 32, H=640, V=3000,
+                            prompts=3, resp_len=32)
+    h, W, y = synth.hidden_states(w, "cuda"), synth.lm_head_weight(w, "cuda"), synth.targets(w, "cuda")
+    adv, mask = synth.rollout(w, force_equal_prompt=1)
+    forced = np.zeros(w.T, bool)
+    forced[16 * 32: 2 * 16 * 32] = True
+    assert not mask.numpy()[forced].any()
+    ref_lp, _, _ = oracle_logprobs_rows(h, W, w.gran, y, np.arange(w.T))
+    noise = synth.old_policy_noise(w).numpy()
+    logp_old = (ref_lp + noise).astype(np.float32)
+    r_bf16 = np.exp(-noise).astype(np.float32)
+    coef = np.exp(logp_old).astype(np.float32)
+    b = api.score_calibrate_loss(h, W, y, torch.from_numpy(logp_old).cuda(), torch.from_numpy(r_bf16).cuda(),
+                                 adv.cuda(), mask.cuda(), torch.from_numpy(coef).cuda(), w.gran,
+                                 w.eps_low, w.eps_high)
+    api.check()
+    res = api.read_calib_result(b.cal_res)
+    st = api.read_clip_stats(b.stats)
+    _pipeline_properties(res, st, b, adv.numpy(), mask.numpy(), r_bf16, w)
+    assert st["n_valid"] == int(mask.numpy().sum())
+    assert not b.clip_mask.cpu().numpy()[forced].any()
+    assert not b.grad.cpu().numpy()[forced].any()
+
+
 def _pipeline_properties(res, st, b, adv, mask, r_bf16, w):
     r = b.ratio.cpu().numpy()
     neg = (mask != 0) & (adv < 0)
