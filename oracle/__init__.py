@@ -25,7 +25,9 @@ logprobs    dequantised logits, log-softmax, target gather, importance
 calibrate   Calibrated Clipping: lower-bound alignment, upper-bound
             rebalancing, SmoothUpdate (§4, Eq. 5, Algorithm 1).
 surrogate   clipped PPO surrogate with TIS weights, token-mean
-            aggregation, clip fractions and dLoss/dlogp (Eq. 1, Eq. 4).
+            aggregation, clip fractions and dLoss/dlogp (Eq. 1, Eq. 4);
+            the sequence-mean aggregation (§2.1) and the sequence-level
+            ratio clipping of the related-work discussion (§6).
 diagnostics over-clipping counts, clip fractions and probability / ratio
             NMAE against BF16 references (§3); TIS weights (§2.3).
 """

@@ -29,6 +29,26 @@ averages each response's token terms, 1/|o_i| sum_t, then the responses):
 with n_i the valid tokens of sequence i and S the sequences that have any;
 g_t = -w_t A_t r_t / (S n_i) on unclipped valid tokens.  A sequence is the
 set of tokens with the same id (they need not be contiguous).
+
+Sequence-level ratio clipping (the GSPO-style trust region over whole
+responses that the related-work discussion names, with extending calibration
+to it left open): each response gets one ratio, the length-normalised
+sequence likelihood ratio
+
+    s_i = (pi(y_i) / pi_old(y_i))^(1/n_i) = exp((1/n_i) sum_{t in i, valid} d_t),
+    d_t = logp_t - logp_old_t  (the float32 log of the token ratio),
+
+i.e. the geometric mean of its token ratios, and one advantage A_i; the
+clipped term, the clip rule (A_i > 0 and s_i >= H, or A_i < 0 and s_i <= L,
+compared in float32 with s_i rounded to float32) and the aggregation over
+responses follow the token-level definitions with s_i in place of r_t:
+
+    loss = (1/S) sum_{i : n_i > 0} -A_i min(s_i, H)   (A_i >= 0)
+                                   -A_i max(s_i, L)   (A_i < 0)
+    g_t  = dloss/dlogp_t = -A_i s_i / (n_i S)  for valid t of unclipped i, else 0
+
+(ds_i/dlogp_t = s_i / n_i).  A token log-ratio outside [-128, 128] (the
+float32 token ratio would over- or underflow) or not finite is bad input.
 """
 
 import numpy as np
@@ -117,3 +137,65 @@ def clipped_surrogate_seq_mean(r, adv, mask, w, lo, hi, seq_id, n_seq):
     out.update({"loss": loss_sum / S if S else 0.0, "loss_sum": loss_sum, "grad": grad,
                 "n_seq_valid": S, "seq_valid_tokens": n_i})
     return out
+
+
+D_MAX = 128.0  # largest |logp - logp_old| a valid token may have
+
+
+def seq_level_clipped_surrogate(logp, logp_old, adv_seq, mask, seq_id, n_seq, lo, hi):
+    """Sequence-level clipped surrogate: one ratio per response, the geometric
+    mean of its token ratios, clipped like a token ratio.  Explicit loops over
+    tokens and sequences; float64 throughout except the float32 token
+    log-ratio and the float32 sequence ratio that the clip rule compares."""
+    d32 = np.asarray(logp, np.float32) - np.asarray(logp_old, np.float32)  # float32 difference
+    a_seq = np.asarray(adv_seq, np.float32).astype(np.float64)
+    T = d32.size
+    valid = _valid(mask, T)
+    sid = np.asarray(seq_id, np.int64)
+    if np.any(sid < 0) or np.any(sid >= n_seq):
+        raise ValueError("sequence id outside [0, n_seq)")
+    if not np.all(np.isfinite(d32[valid])) or np.any(np.abs(d32[valid]) > D_MAX):
+        raise ValueError("token log-ratio outside [-128, 128]")
+    n_i = np.zeros(n_seq, np.int64)
+    d_sum = np.zeros(n_seq)
+    for t in range(T):
+        if valid[t]:
+            n_i[sid[t]] += 1
+            d_sum[sid[t]] += float(d32[t])
+    S = int(np.sum(n_i > 0))
+    lo32, hi32 = np.float32(lo), np.float32(hi)
+    s64 = np.zeros(n_seq)
+    s32 = np.zeros(n_seq, np.float32)
+    cm = np.zeros(n_seq, np.uint8)
+    terms = np.zeros(n_seq)
+    coef = np.zeros(n_seq)  # g_t of the sequence's valid tokens
+    for i in range(n_seq):
+        if n_i[i] == 0:
+            continue
+        s64[i] = np.exp(d_sum[i] / n_i[i])
+        s32[i] = np.float32(s64[i])
+        A = a_seq[i]
+        up = A > 0 and s32[i] >= hi32
+        dn = A < 0 and s32[i] <= lo32
+        cm[i] = CLIP_HI * up + CLIP_LO * dn
+        s = float(s32[i])
+        m = min(s, float(hi32)) if A >= 0 else max(s, float(lo32))
+        terms[i] = -A * m
+        if not (up or dn):
+            coef[i] = -A * s / (n_i[i] * S)
+    grad = np.zeros(T)
+    for t in range(T):
+        if valid[t]:
+            grad[t] = coef[sid[t]]
+    live = n_i > 0
+    loss_sum = float(np.sum(terms[live]))
+    n_pos = int(np.sum(live & (a_seq > 0)))
+    n_neg = int(np.sum(live & (a_seq < 0)))
+    c_pos = int(np.sum((cm & CLIP_HI) != 0))
+    c_neg = int(np.sum((cm & CLIP_LO) != 0))
+    return {
+        "loss": loss_sum / S if S else 0.0, "loss_sum": loss_sum, "grad": grad,
+        "seq_ratio": s64, "seq_ratio32": s32, "seq_clip": cm, "seq_terms": terms,
+        "seq_valid_tokens": n_i, "n_seq_valid": S, "n_valid": int(valid.sum()),
+        "n_pos": n_pos, "n_neg": n_neg, "clipped_pos": c_pos, "clipped_neg": c_neg,
+    }

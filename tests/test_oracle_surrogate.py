@@ -168,3 +168,129 @@ def test_seq_mean_gradient_finite_difference():
         e[t] = h
         fd = (loss(lp + e) - loss(lp - e)) / (2 * h)
         assert abs(fd - g[t]) < 5e-6 * max(1.0, abs(fd)), t
+
+
+# ---- sequence-level ratio clipping (one geometric-mean ratio per response) ---
+
+def test_seq_level_hand_case():
+    # sequence 0: d = ln 2, 0 -> s = sqrt 2 >= H with A > 0: clipped, term -H
+    # sequence 1: d = 0, 0, 0 -> s = 1, A = -1: term +1, g = -A s / (n S) = 1/9
+    # sequence 2: d = -ln 4 -> s = 1/4 <= L with A < 0: clipped, term -A L = 0.5 L
+    lp = np.array([np.log(2), 0, 0, 0, 0, -np.log(4)], np.float32)
+    out = S.seq_level_clipped_surrogate(lp, np.zeros(6, np.float32), [1.0, -1.0, -0.5], None,
+                                        [0, 0, 1, 1, 1, 2], 3, 0.8, 1.2)
+    L32, H32 = float(np.float32(0.8)), float(np.float32(1.2))
+    assert np.allclose(out["seq_ratio"], [np.sqrt(2.0), 1.0, 0.25], rtol=1e-7, atol=0)
+    assert list(out["seq_clip"]) == [S.CLIP_HI, 0, S.CLIP_LO]
+    assert abs(out["loss"] - (-H32 + 1.0 + 0.5 * L32) / 3) < 1e-15
+    assert np.allclose(out["grad"], [0, 0, 1 / 9, 1 / 9, 1 / 9, 0], rtol=0, atol=1e-15)
+    assert out["n_seq_valid"] == 3 and out["clipped_pos"] == 1 and out["clipped_neg"] == 1
+
+
+def test_seq_level_ratio_is_geometric_mean_of_token_ratios():
+    # the literal definition (pi(y)/pi_old(y))^(1/|y|) with pi(y) the product of
+    # the token probabilities, on short sequences where the products stay finite
+    rng = np.random.default_rng(30)
+    n_seq, T = 9, 60
+    sid = rng.integers(0, n_seq, T)
+    lp = rng.normal(-2, 0.7, T).astype(np.float32)
+    lp_old = (lp + rng.normal(0, 0.2, T)).astype(np.float32)
+    m = (rng.random(T) < 0.85).astype(np.uint8)
+    out = S.seq_level_clipped_surrogate(lp, lp_old, np.ones(n_seq), m, sid, n_seq, 0.0, np.inf)
+    for i in range(n_seq):
+        sel = (sid == i) & (m != 0)
+        if not sel.any():
+            assert out["seq_ratio"][i] == 0 and out["seq_valid_tokens"][i] == 0
+            continue
+        d = (lp[sel] - lp_old[sel]).astype(np.float64)  # the float32 token log-ratios
+        geo = np.prod(np.exp(d)) ** (1.0 / sel.sum())
+        assert abs(out["seq_ratio"][i] - geo) < 1e-13 * geo, i
+
+
+def test_seq_level_single_token_sequences_reduce_to_token_level():
+    # one valid token per sequence: s_i is that token's ratio, S = n_valid, and
+    # the loss, clip bits and gradient are the token-mean surrogate's
+    rng = np.random.default_rng(31)
+    T = 300
+    d = rng.normal(0, 0.3, T).astype(np.float32)
+    lp_old = rng.normal(-3, 1, T).astype(np.float32)
+    lp = (lp_old + d).astype(np.float32)
+    A = rng.normal(0, 1, T).astype(np.float32)
+    A[::17] = 0
+    out = S.seq_level_clipped_surrogate(lp, lp_old, A, None, np.arange(T), T, 0.8, 1.2)
+    r = np.float32(np.exp((lp - lp_old).astype(np.float64)))
+    tok = S.clipped_surrogate(r, A, None, None, 0.8, 1.2)
+    assert abs(out["loss"] - tok["loss"]) < 1e-14
+    assert np.array_equal(out["seq_clip"], tok["clip_mask"])
+    assert np.allclose(out["grad"], tok["grad"], rtol=1e-15, atol=0)
+    assert (out["clipped_pos"], out["clipped_neg"]) == (tok["clipped_pos"], tok["clipped_neg"])
+
+
+def test_seq_level_unclipped_and_invariances():
+    rng = np.random.default_rng(32)
+    T, n = 400, 23
+    sid = rng.integers(0, n, T)
+    lp_old = rng.normal(-3, 1, T).astype(np.float32)
+    lp = (lp_old + rng.normal(0, 0.5, T)).astype(np.float32)
+    A = rng.normal(0, 1, n).astype(np.float32)
+    m = (rng.random(T) < 0.7).astype(np.uint8)
+    # bounds that clip nothing: loss = -(1/S) sum_i A_i s_i
+    free = S.seq_level_clipped_surrogate(lp, lp_old, A, m, sid, n, 0.0, np.inf)
+    live = free["seq_valid_tokens"] > 0
+    s32 = free["seq_ratio32"].astype(np.float64)
+    assert abs(free["loss"] - (-np.sum(A[live] * s32[live]) / live.sum())) < 1e-14
+    assert free["clipped_pos"] == 0 and free["clipped_neg"] == 0
+    # token order and sequence labels do not matter
+    a = S.seq_level_clipped_surrogate(lp, lp_old, A, m, sid, n, 0.8, 1.2)
+    p = rng.permutation(T)
+    relabel = rng.permutation(n)
+    b = S.seq_level_clipped_surrogate(lp[p], lp_old[p], A[np.argsort(relabel)], m[p], relabel[sid[p]],
+                                      n, 0.8, 1.2)
+    assert abs(a["loss"] - b["loss"]) < 1e-14
+    assert np.array_equal(a["grad"][p], b["grad"])
+    assert np.array_equal(a["seq_clip"], b["seq_clip"][relabel])
+
+
+def test_seq_level_empty_and_bad_input():
+    lp = np.zeros(8, np.float32)
+    out = S.seq_level_clipped_surrogate(lp, lp, np.ones(3), np.zeros(8, np.uint8), np.zeros(8, int), 3,
+                                        0.8, 1.2)
+    assert out["loss"] == 0 and out["n_seq_valid"] == 0 and not out["grad"].any()
+    with pytest.raises(ValueError):
+        S.seq_level_clipped_surrogate(lp, lp, np.ones(3), None, np.full(8, 3), 3, 0.8, 1.2)
+    big = lp.copy()
+    big[2] = 200.0
+    with pytest.raises(ValueError):
+        S.seq_level_clipped_surrogate(big, lp, np.ones(3), None, np.zeros(8, int), 3, 0.8, 1.2)
+    # a masked token may hold anything
+    m = np.ones(8, np.uint8)
+    m[2] = 0
+    S.seq_level_clipped_surrogate(big, lp, np.ones(3), m, np.zeros(8, int), 3, 0.8, 1.2)
+
+
+def test_seq_level_gradient_finite_difference():
+    rng = np.random.default_rng(33)
+    T, n = 40, 5
+    sid = rng.integers(0, n, T)
+    lp_old = rng.normal(-3, 1, T)
+    lp = lp_old + rng.normal(0, 0.2, T)
+    A = rng.normal(0, 1, n)
+    m = (rng.random(T) < 0.8).astype(np.uint8)
+    lo, hi = 0.9, 1.1
+
+    def loss(x):
+        v = m != 0
+        cnt = np.bincount(sid[v], minlength=n)
+        mu = np.bincount(sid[v], weights=(x - lp_old)[v], minlength=n)
+        keep = cnt > 0
+        s = np.exp(mu[keep] / cnt[keep])
+        a = A[keep]
+        return np.sum(-np.minimum(s * a, np.clip(s, lo, hi) * a)) / keep.sum()
+
+    g = S.seq_level_clipped_surrogate(lp, lp_old, A, m, sid, n, lo, hi)["grad"]
+    h = 1e-6
+    for t in range(T):
+        e = np.zeros(T)
+        e[t] = h
+        fd = (loss(lp + e) - loss(lp - e)) / (2 * h)
+        assert abs(fd - g[t]) < 1e-5 * max(1.0, abs(fd)), t
