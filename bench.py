@@ -547,6 +547,18 @@ def run_kernel_rooflines(args, local_rank):
     ms = timed(lambda: api.clipped_surrogate_seq_mean(r_fp, adv, sid, n_seq, mask, None, 0.8, 1.2, stats=st,
                                                       workspace=qws, out={"grad": grad, "clip_mask": cm}), 10)
     line("clipped surrogate, sequence mean", [T], T * (5 + 4 + 4 + 4 + 1 + 4 + 1), ms)
+    # sequence-level ratio clipping: logp, logp_old, ids, mask in; dloss/dlogp
+    # out; one advantage, ratio and clip byte per response
+    lp = torch.log(r_fp) - 3.0
+    lpo = torch.log(r_bf) - 3.0
+    a_seq = adv[:n_seq].contiguous()
+    lws = torch.empty(api.lib.fp8rl_seq_level_surrogate_workspace_size(T, n_seq), dtype=torch.uint8, device=dev)
+    s_ratio = torch.empty(n_seq, device=dev)
+    s_clip = torch.empty(n_seq, dtype=torch.uint8, device=dev)
+    ms = timed(lambda: api.seq_level_clipped_surrogate(lp, lpo, a_seq, sid, mask, 0.8, 1.2, stats=st,
+                                                       workspace=lws, out={"grad": grad, "seq_ratio": s_ratio,
+                                                                           "seq_clip": s_clip}), 10)
+    line("clipped surrogate, sequence-level ratio", [T], T * (4 + 4 + 4 + 1 + 4) + n_seq * 9, ms)
     del qws, sid
     lp8 = torch.log(r_fp)
     lpb = torch.log(r_bf)

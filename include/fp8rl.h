@@ -337,6 +337,45 @@ fp8rl_status fp8rl_clipped_surrogate_seq_mean(const float* r, const float* adv,
                                               void* workspace, size_t workspace_bytes,
                                               void* stream);
 
+/* Sequence-level ratio clipping: the response-level trust region that §6
+ * (related work) names, with one ratio per response instead of per token.
+ * For sequence i with n_i valid tokens:
+ *   s_i  = exp((1/n_i) sum_{t in i, valid} d_t),  d_t = logp_t - logp_old_t
+ *          (the geometric mean of the token ratios), rounded to float32
+ *   loss = (1/S) sum_{i : n_i > 0} -A_i m_i,  m_i = min(s_i, H) if A_i >= 0, else max(s_i, L)
+ *   clipped (gradient zeroed): A_i > 0 and s_i >= H, or A_i < 0 and s_i <= L
+ *   g_t  = dloss/dlogp_t = -A_i s_i / (n_i S) on valid tokens of unclipped
+ *          sequences (float64 quotient rounded to float32), 0 elsewhere
+ * S = sequences with n_i > 0.  The exponent sums are accumulated exactly on
+ * the 2^-32 grid (each |d_t| >= 2^-8 is exact there, smaller ones round to
+ * it), so the result is independent of token order; exact for sequences of
+ * up to 2^24 valid tokens.
+ *   logp, logp_old  float [T] (the scored and the old log-probs)
+ *   adv_seq     float [n_seq]: the response advantages A_i
+ *   mask        uint8 [T] or NULL;  seq_id int32 [T] in [0, n_seq) (tokens of
+ *               a sequence need not be contiguous)
+ *   lo, hi / bounds  as for fp8rl_clipped_surrogate
+ *   seq_ratio   float [n_seq] out or NULL: s_i (0 for a sequence without valid tokens)
+ *   seq_clip    uint8 [n_seq] out or NULL: FP8RL_CLIP_HI / FP8RL_CLIP_LO bits
+ *   grad_logp   float [T] out or NULL
+ *   stats       DEVICE fp8rl_clip_stats: loss, loss_sum = S loss, n_valid
+ *               (tokens), n_pos / n_neg / clipped_pos / clipped_neg counted
+ *               over SEQUENCES with n_i > 0, n_seq_valid = S, flags 1 when no
+ *               token is valid.
+ * A valid token with |d_t| > 128 or a NaN d_t (its float32 ratio would over-
+ * or underflow) and an id outside [0, n_seq) set FP8RL_EDEVICE; such a d_t
+ * counts as its clamp to [-128, 128] (NaN as 0), such an id nowhere. */
+size_t fp8rl_seq_level_surrogate_workspace_size(int64_t T, int64_t n_seq);
+
+fp8rl_status fp8rl_seq_level_clipped_surrogate(const float* logp, const float* logp_old,
+                                               const float* adv_seq, const uint8_t* mask,
+                                               const int32_t* seq_id, int64_t n_seq, int64_t T,
+                                               float lo, float hi, const float* bounds,
+                                               float* seq_ratio, uint8_t* seq_clip,
+                                               float* grad_logp, fp8rl_clip_stats* stats,
+                                               void* workspace, size_t workspace_bytes,
+                                               void* stream);
+
 /* Dense dLoss/dlogits for selected rows (a verification and debugging path;
  * the hot path keeps the factored form above).  For i < n_rows, t = rows[i]:
  *   out[i][v] = grad_logp[t] * (1{v == y_t} - exp(z[t][v] - lse[t])),  v < V,

@@ -96,6 +96,9 @@ _SIGS = {
     "fp8rl_surrogate_seq_mean_workspace_size": (_sz, [_i64, _i64]),
     "fp8rl_clipped_surrogate_seq_mean": (_i, [_p, _p, _p, _p, _p, _i64, _i64, _f, _f, _p, _p, _p, _p, _p,
                                               _sz, _p]),
+    "fp8rl_seq_level_surrogate_workspace_size": (_sz, [_i64, _i64]),
+    "fp8rl_seq_level_clipped_surrogate": (_i, [_p, _p, _p, _p, _p, _i64, _i64, _f, _f, _p, _p, _p, _p, _p,
+                                               _p, _sz, _p]),
     "fp8rl_clip_diagnostics_workspace_size": (_sz, [_i64]),
     "fp8rl_clip_diagnostics": (_i, [_p, _p, _p, _p, _p, _p, _i64, _f, _f, _p, _p, _sz, _p]),
     "fp8rl_tis_weights": (_i, [_p, _p, _i64, _f, _p, _p]),
@@ -407,6 +410,36 @@ def clipped_surrogate_seq_mean(r, adv, seq_id, n_seq, mask=None, w_tis=None, lo=
                                              _ptr(stats), _ptr(workspace), workspace.numel(),
                                              _stream(stream)), "fp8rl_clipped_surrogate_seq_mean")
     return {"stats": stats, "grad": grad, "clip_mask": cm}
+
+
+def seq_level_clipped_surrogate(logp, logp_old, adv_seq, seq_id, mask=None, lo=0.8, hi=1.2, bounds=None,
+                                want_grad=True, stats=None, workspace=None, out=None, stream=None):
+    """fp8rl_seq_level_clipped_surrogate (one geometric-mean ratio per
+    response, clipped like a token ratio) -> dict(stats=<device buffer>,
+    seq_ratio, seq_clip, grad).  ``adv_seq`` holds one advantage per sequence;
+    its length is n_seq."""
+    T = logp.numel()
+    n_seq = adv_seq.numel()
+    dev = logp.device
+    _dev(logp, torch.float32, "logp")
+    _dev(logp_old, torch.float32, "logp_old", T)
+    _dev(adv_seq, torch.float32, "adv_seq")
+    _dev(seq_id, torch.int32, "seq_id", T)
+    _dev(mask, torch.uint8, "mask", T)
+    _dev(bounds, torch.float32, "bounds", 2)
+    o = out or {}
+    ratio = o.get("seq_ratio", torch.empty(n_seq, dtype=torch.float32, device=dev))
+    clip = o.get("seq_clip", torch.empty(n_seq, dtype=torch.uint8, device=dev))
+    grad = o.get("grad", torch.empty(T, dtype=torch.float32, device=dev)) if want_grad else None
+    stats = torch.zeros(ctypes.sizeof(ClipStats), dtype=torch.uint8, device=dev) if stats is None else stats
+    if workspace is None:
+        workspace = _workspace(lib.fp8rl_seq_level_surrogate_workspace_size(T, n_seq), dev)
+    _ok(lib.fp8rl_seq_level_clipped_surrogate(_ptr(logp), _ptr(logp_old), _ptr(adv_seq), _ptr(mask),
+                                              _ptr(seq_id), n_seq, T, lo, hi, _ptr(bounds), _ptr(ratio),
+                                              _ptr(clip), _ptr(grad), _ptr(stats), _ptr(workspace),
+                                              workspace.numel(), _stream(stream)),
+        "fp8rl_seq_level_clipped_surrogate")
+    return {"stats": stats, "seq_ratio": ratio, "seq_clip": clip, "grad": grad}
 
 
 def read_clip_stats(buf):

@@ -322,6 +322,27 @@ fp8rl_status fp8rl_clipped_surrogate_seq_mean(const float* r, const float* adv, 
   return e == cudaSuccess ? FP8RL_OK : cuda_fail(e);
 }
 
+size_t fp8rl_seq_level_surrogate_workspace_size(int64_t T, int64_t n_seq) {
+  return (T < 0 || n_seq < 0) ? 0 : seq_level_workspace_bytes(T, n_seq);
+}
+
+fp8rl_status fp8rl_seq_level_clipped_surrogate(const float* logp, const float* logp_old,
+                                               const float* adv_seq, const uint8_t* mask,
+                                               const int32_t* seq_id, int64_t n_seq, int64_t T,
+                                               float lo, float hi, const float* bounds,
+                                               float* seq_ratio, uint8_t* seq_clip, float* grad,
+                                               fp8rl_clip_stats* stats, void* ws, size_t ws_bytes,
+                                               void* stream) {
+  if (!stats || (T > 0 && (!logp || !logp_old || !seq_id)) || (n_seq > 0 && !adv_seq))
+    return FP8RL_EINVAL;
+  if (T < 0 || n_seq < 0 || n_seq > 0x7FFFFFFF) return FP8RL_ESHAPE;
+  if (!ws || ws_bytes < seq_level_workspace_bytes(T, n_seq)) return FP8RL_EWORKSPACE;
+  cudaError_t e = launch_seq_level(logp, logp_old, adv_seq, mask, seq_id, n_seq, T, lo, hi, bounds,
+                                   seq_ratio, seq_clip, grad, stats, ws,
+                                   static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? FP8RL_OK : cuda_fail(e);
+}
+
 // ------------------------------------------------------------------ diagnostics
 size_t fp8rl_clip_diagnostics_workspace_size(int64_t T) { return T < 0 ? 0 : diag_workspace_bytes(T); }
 

@@ -73,6 +73,12 @@ cudaError_t launch_surrogate(const float* r, const float* adv, const uint8_t* ma
                              const float* w, int64_t T, float lo, float hi, const float* bounds,
                              float* grad, uint8_t* clip_mask, fp8rl_clip_stats* stats, void* ws,
                              cudaStream_t s);
+size_t seq_level_workspace_bytes(int64_t T, int64_t n_seq);
+cudaError_t launch_seq_level(const float* logp, const float* logp_old, const float* adv_seq,
+                             const uint8_t* mask, const int32_t* sid, int64_t n_seq, int64_t T,
+                             float lo, float hi, const float* bounds, float* seq_ratio,
+                             uint8_t* seq_clip, float* grad, fp8rl_clip_stats* stats, void* ws,
+                             cudaStream_t s);
 size_t seq_surrogate_workspace_bytes(int64_t T, int64_t n_seq);
 cudaError_t launch_seq_surrogate(const float* r, const float* adv, const uint8_t* mask,
                                  const float* w, const int32_t* sid, int64_t n_seq, int64_t T,

@@ -21,6 +21,17 @@
 // tokens of the same sequence) and S = #{i : n_i > 0}; the
 // fused pass then weights each term by 1/n_i and each gradient by 1/(S n_i):
 //   loss = (1/S) sum_i (1/n_i) sum_{t in i} l_t,   g_t = -w_t A_t r_t / (S n_i).
+//
+// Sequence-level ratio clipping (the response-level trust region of the
+// related-work discussion, §6): one ratio per response, the geometric mean of
+// its token ratios s_i = exp((1/n_i) sum_t d_t), d_t = logp_t - logp_old_t,
+// clipped like a token ratio with the response's advantage A_i:
+//   loss = (1/S) sum_i -A_i m_i,  m_i = min(s_i, H) (A_i >= 0) / max(s_i, L),
+//   g_t  = -A_i s_i / (n_i S) on valid tokens of unclipped responses.
+// The exponent sums are exact integers: each d_t (|d_t| <= 128) is taken to
+// the 2^-32 grid (exact for |d_t| >= 2^-8, where d_t 2^32 is already an
+// integer) and summed with 64-bit integer atomics, so the result does not
+// depend on the order of the tokens or of the atomics.
 #include "common.cuh"
 #include "internal.h"
 
@@ -394,6 +405,288 @@ __global__ void __launch_bounds__(kThreads) seq_surrogate_kernel(
   }
 }
 
+// ------------------------------------------------------------ sequence-level ratio
+constexpr float kSeqLvlDMax = 128.f;  // largest |d_t| of a valid token
+
+struct SeqLvlWork {
+  unsigned long long n_valid;
+  unsigned int n_seq_valid;
+  unsigned int ticket;
+  unsigned int pad[60];
+  // then: q[n_seq] (int64 fixed-point exponent sums), cnt[n_seq] (uint32),
+  // part[grid of the sequence pass], coef[n_seq] (float)
+};
+
+struct SeqLvlLayout {
+  size_t q, cnt, part, coef, zero_bytes, total;
+};
+
+int seq_grid_of(int64_t n_seq) {
+  const int64_t want = (n_seq + kThreads - 1) / kThreads;
+  const int64_t cap = static_cast<int64_t>(sm_count()) * kCtasPerSm;
+  return static_cast<int>(want < 1 ? 1 : (want > cap ? cap : want));
+}
+
+SeqLvlLayout seq_lvl_layout(int64_t n_seq) {
+  const size_t n = static_cast<size_t>(n_seq > 0 ? n_seq : 1);
+  SeqLvlLayout l;
+  l.q = sizeof(SeqLvlWork);
+  l.cnt = l.q + 8 * n;
+  l.zero_bytes = l.cnt + 4 * n;  // header, q and cnt are zeroed every call
+  l.part = align_up(l.zero_bytes, 256);
+  l.coef = align_up(l.part + sizeof(Partial) * static_cast<size_t>(seq_grid_of(n_seq)), 256);
+  l.total = align_up(l.coef + 4 * n, 256);
+  return l;
+}
+
+// Pass 1: per sequence the valid-token count n_i and the fixed-point sum
+// Q_i = sum_t RNE(d_t 2^32), plus S = #{i : n_i > 0}.  Each warp walks its
+// own contiguous range, 128 tokens a step (four consecutive tokens a lane).
+// Every lane accumulates the tokens of the warp's current sequence in
+// registers; only a step that holds a valid token of another sequence (a
+// response boundary) makes the warp cooperate: it flushes the current
+// sequence (warp sum, one pair of atomics), takes the step's last valid id as
+// the new current sequence, and sends any other token (a response shorter
+// than a step, or ids in no order) straight to the atomics.  Invalid tokens
+// add nothing whatever their id.
+template <bool VEC>
+__global__ void __launch_bounds__(kThreads) seq_lvl_accum_kernel(
+    const float* __restrict__ logp, const float* __restrict__ logp_old,
+    const uint8_t* __restrict__ mask, const int32_t* __restrict__ sid, int64_t T, int64_t n_seq,
+    unsigned long long* __restrict__ qsum, unsigned int* __restrict__ cnt, SeqLvlWork* w) {
+  const int lane = threadIdx.x & 31;
+  const int64_t nwarps = static_cast<int64_t>(gridDim.x) * (kThreads / 32);
+  const int64_t wid = static_cast<int64_t>(blockIdx.x) * (kThreads / 32) + (threadIdx.x >> 5);
+  const int64_t per = ((T + nwarps - 1) / nwarps + 127) / 128 * 128;
+  const int64_t beg = wid * per, end = min(T, beg + per);
+  uint32_t nv = 0, s_new = 0;
+  bool bad = false;
+  int cur = -1;  // warp-uniform current sequence
+  long long acc_q = 0;
+  unsigned acc_n = 0;
+  auto flush = [&]() {
+    long long q = acc_q;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
+    const unsigned n = __reduce_add_sync(0xffffffffu, acc_n);
+    if (lane == 0 && n) {
+      s_new += atomicAdd(&cnt[cur], n) == 0u;
+      atomicAdd(&qsum[cur], static_cast<unsigned long long>(q));
+    }
+    acc_q = 0;
+    acc_n = 0;
+  };
+  for (int64_t base = beg; base < end; base += 128) {
+    const int64_t t0 = base + 4 * lane;
+    int id[4];
+    float lp[4], lo[4];
+    bool on[4];
+    if (VEC && t0 + 3 < end) {
+      const int4 iv = __ldg(reinterpret_cast<const int4*>(sid + t0));
+      const float4 a = __ldg(reinterpret_cast<const float4*>(logp + t0));
+      const float4 b = __ldg(reinterpret_cast<const float4*>(logp_old + t0));
+      const uint32_t mv = mask ? __ldg(reinterpret_cast<const uint32_t*>(mask + t0)) : 0x01010101u;
+      id[0] = iv.x, id[1] = iv.y, id[2] = iv.z, id[3] = iv.w;
+      lp[0] = a.x, lp[1] = a.y, lp[2] = a.z, lp[3] = a.w;
+      lo[0] = b.x, lo[1] = b.y, lo[2] = b.z, lo[3] = b.w;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) on[k] = ((mv >> (8 * k)) & 0xFFu) != 0;
+    } else {
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int64_t t = t0 + k;
+        const bool in = t < end;
+        id[k] = in ? __ldg(sid + t) : 0;
+        lp[k] = in ? __ldg(logp + t) : 0.f;
+        lo[k] = in ? __ldg(logp_old + t) : 0.f;
+        on[k] = in && (!mask || __ldg(mask + t) != 0);
+        if (!in) id[k] = cur;  // past the end: nothing to add
+      }
+    }
+    long long q[4];
+    bool v[4];
+    bool match = true;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const bool in_range = id[k] >= 0 && id[k] < n_seq;
+      if (t0 + k < end && !in_range) bad = true;  // masked tokens too
+      v[k] = on[k] && in_range;
+      float d = lp[k] - lo[k];
+      if (v[k] && !(fabsf(d) <= kSeqLvlDMax)) {  // out of range or NaN
+        bad = true;
+        d = d != d ? 0.f : fminf(fmaxf(d, -kSeqLvlDMax), kSeqLvlDMax);
+      }
+      // d 2^32 is exact in float32; the conversion rounds to nearest even
+      q[k] = v[k] ? __float2ll_rn(d * 4294967296.0f) : 0ll;
+      nv += v[k];
+      match = match && (!v[k] || id[k] == cur);
+    }
+    if (__all_sync(0xffffffffu, match)) {  // the step continues the current sequence
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        acc_q += q[k];
+        acc_n += v[k];
+      }
+      continue;
+    }
+    // a boundary: finish the current sequence with this step's tokens of it
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      if (v[k] && id[k] == cur) {
+        acc_q += q[k];
+        acc_n += 1;
+        v[k] = false;
+      }
+    flush();
+    // the step's last valid token names the sequence that may run on
+    int last_id = -1;
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      if (v[k]) last_id = id[k];
+    const unsigned has = __ballot_sync(0xffffffffu, last_id >= 0);
+    if (has) cur = __shfl_sync(0xffffffffu, last_id, 31 - __clz(has));
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      if (v[k] && id[k] == cur) {
+        acc_q += q[k];
+        acc_n += 1;
+        v[k] = false;
+      }
+    // whatever is left belongs to neither: one pair of atomics per token
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      if (v[k]) {
+        s_new += atomicAdd(&cnt[id[k]], 1u) == 0u;
+        atomicAdd(&qsum[id[k]], static_cast<unsigned long long>(q[k]));
+      }
+  }
+  flush();
+  if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(&d_status, kErrDevice);
+  const uint32_t sv = __reduce_add_sync(0xffffffffu, nv);
+  const uint32_t sn = __reduce_add_sync(0xffffffffu, s_new);
+  if (lane == 0 && sv) atomicAdd(&w->n_valid, static_cast<unsigned long long>(sv));
+  if (lane == 0 && sn) atomicAdd(&w->n_seq_valid, sn);
+}
+
+// Pass 2, one thread per sequence: s_i = fl32(exp(Q_i 2^-32 / n_i)), the clip
+// bits, the term -A_i m_i (an exact float64 product) and the gradient
+// coefficient fl32(-A_i s_i / (n_i S)) of its valid tokens; the terms meet in
+// a fixed-order reduction (last block), which also writes the statistics.
+__global__ void __launch_bounds__(kThreads) seq_lvl_seq_kernel(
+    const float* __restrict__ adv_seq, int64_t n_seq, const unsigned long long* __restrict__ qsum,
+    const unsigned int* __restrict__ cnt, float lo_arg, float hi_arg, const float* __restrict__ bounds,
+    float* __restrict__ seq_ratio, uint8_t* __restrict__ seq_clip, float* __restrict__ coef,
+    Partial* __restrict__ part, fp8rl_clip_stats* __restrict__ stats, SeqLvlWork* w) {
+  __shared__ double sh_d[kThreads / 32];
+  __shared__ unsigned long long sh_u[kThreads / 32];
+  __shared__ bool last;
+  const float lo = bounds ? bounds[0] : lo_arg;
+  const float hi = bounds ? bounds[1] : hi_arg;
+  const unsigned int S = w->n_seq_valid;
+  double L = 0.0;
+  uint32_t np = 0, nn = 0, cp = 0, cn = 0;
+  for (int64_t i = blockIdx.x * (int64_t)kThreads + threadIdx.x; i < n_seq;
+       i += (int64_t)gridDim.x * kThreads) {
+    const unsigned n = cnt[i];
+    float s = 0.f, c = 0.f;
+    uint32_t cm = 0;
+    if (n) {
+      const double mu = static_cast<double>(static_cast<long long>(qsum[i])) * 0x1p-32 /
+                        static_cast<double>(n);
+      s = static_cast<float>(exp(mu));
+      const float A = adv_seq[i];
+      const bool up = A > 0.f && s >= hi;
+      const bool dn = A < 0.f && s <= lo;
+      const float m = A >= 0.f ? fminf(s, hi) : fmaxf(s, lo);
+      L += -static_cast<double>(A) * static_cast<double>(m);
+      np += A > 0.f;
+      nn += A < 0.f;
+      cp += up;
+      cn += dn;
+      cm = (up ? FP8RL_CLIP_HI : 0u) | (dn ? FP8RL_CLIP_LO : 0u);
+      if (!(up || dn))
+        c = static_cast<float>(-static_cast<double>(A) * static_cast<double>(s) /
+                               (static_cast<double>(n) * static_cast<double>(S)));
+    }
+    coef[i] = c;
+    if (seq_ratio) seq_ratio[i] = s;
+    if (seq_clip) seq_clip[i] = static_cast<uint8_t>(cm);
+  }
+  L = block_sum(L, sh_d);
+  const unsigned long long bnp = block_sum<unsigned long long>(np, sh_u);
+  const unsigned long long bnn = block_sum<unsigned long long>(nn, sh_u);
+  const unsigned long long bcp = block_sum<unsigned long long>(cp, sh_u);
+  const unsigned long long bcn = block_sum<unsigned long long>(cn, sh_u);
+  if (threadIdx.x == 0) {
+    Partial& p = part[blockIdx.x];
+    p.loss = L;
+    p.n_pos = bnp;
+    p.n_neg = bnn;
+    p.c_pos = bcp;
+    p.c_neg = bcn;
+    __threadfence();
+    last = atomicAdd(&w->ticket, 1u) == gridDim.x - 1;
+  }
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  double tl = 0.0;
+  unsigned long long tnp = 0, tnn = 0, tcp = 0, tcn = 0;
+  for (unsigned k = threadIdx.x; k < gridDim.x; k += kThreads) {
+    const volatile Partial& p = part[k];
+    tl += p.loss;
+    tnp += p.n_pos;
+    tnn += p.n_neg;
+    tcp += p.c_pos;
+    tcn += p.c_neg;
+  }
+  tl = block_sum(tl, sh_d);
+  tnp = block_sum(tnp, sh_u);
+  tnn = block_sum(tnn, sh_u);
+  tcp = block_sum(tcp, sh_u);
+  tcn = block_sum(tcn, sh_u);
+  if (threadIdx.x == 0) {
+    const unsigned long long n_valid = w->n_valid;
+    fp8rl_clip_stats st;
+    st.loss_sum = tl;
+    st.loss = S ? tl / static_cast<double>(S) : 0.0;
+    st.n_valid = static_cast<int64_t>(n_valid);
+    st.n_pos = static_cast<int64_t>(tnp);
+    st.n_neg = static_cast<int64_t>(tnn);
+    st.clipped_pos = static_cast<int64_t>(tcp);
+    st.clipped_neg = static_cast<int64_t>(tcn);
+    st.lo = lo;
+    st.hi = hi;
+    st.flags = n_valid ? 0 : 1;
+    st.n_seq_valid = static_cast<int32_t>(S);
+    *stats = st;
+  }
+}
+
+// Pass 3: g_t = coef[seq(t)] on valid tokens, 0 elsewhere; four tokens per
+// thread and step with 16-byte loads and stores when the arrays allow.
+__global__ void __launch_bounds__(kThreads) seq_lvl_grad_kernel(
+    const uint8_t* __restrict__ mask, const int32_t* __restrict__ sid, int64_t T, int64_t n_seq,
+    const float* __restrict__ coef, float* __restrict__ grad, bool vec) {
+  const int64_t tid = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  auto one = [&](int id, bool present) {
+    return present && id >= 0 && id < n_seq ? __ldg(coef + id) : 0.f;
+  };
+  const int64_t T4 = vec ? T / 4 : 0;
+  for (int64_t i = tid; i < T4; i += stride) {
+    const int4 iv = __ldg(reinterpret_cast<const int4*>(sid) + i);
+    const uint32_t mv = mask ? __ldg(reinterpret_cast<const uint32_t*>(mask) + i) : 0x01010101u;
+    float4 g;
+    g.x = one(iv.x, (mv & 0xFFu) != 0);
+    g.y = one(iv.y, (mv & 0xFF00u) != 0);
+    g.z = one(iv.z, (mv & 0xFF0000u) != 0);
+    g.w = one(iv.w, (mv & 0xFF000000u) != 0);
+    reinterpret_cast<float4*>(grad)[i] = g;
+  }
+  for (int64_t t = T4 * 4 + tid; t < T; t += stride) grad[t] = one(sid[t], mask ? mask[t] != 0 : true);
+}
+
 }  // namespace
 
 size_t surrogate_workspace_bytes(int64_t T) {
@@ -436,6 +729,36 @@ cudaError_t launch_seq_surrogate(const float* r, const float* adv, const uint8_t
                    aligned(grad, 16) && aligned(mask, 4) && aligned(clip_mask, 4);
   seq_surrogate_kernel<<<grid, kThreads, 0, s>>>(r, adv, mask, w, sid, T, n_seq, cnt, lo, hi, bounds,
                                                   grad, clip_mask, stats, work, vec);
+  return cudaGetLastError();
+}
+
+size_t seq_level_workspace_bytes(int64_t, int64_t n_seq) { return seq_lvl_layout(n_seq).total; }
+
+cudaError_t launch_seq_level(const float* logp, const float* logp_old, const float* adv_seq,
+                             const uint8_t* mask, const int32_t* sid, int64_t n_seq, int64_t T,
+                             float lo, float hi, const float* bounds, float* seq_ratio,
+                             uint8_t* seq_clip, float* grad, fp8rl_clip_stats* stats, void* ws,
+                             cudaStream_t s) {
+  const SeqLvlLayout l = seq_lvl_layout(n_seq);
+  char* base = static_cast<char*>(ws);
+  SeqLvlWork* work = reinterpret_cast<SeqLvlWork*>(base);
+  auto* q = reinterpret_cast<unsigned long long*>(base + l.q);
+  auto* cnt = reinterpret_cast<unsigned int*>(base + l.cnt);
+  auto* part = reinterpret_cast<Partial*>(base + l.part);
+  auto* coef = reinterpret_cast<float*>(base + l.coef);
+  cudaError_t e = cudaMemsetAsync(base, 0, l.zero_bytes, s);
+  if (e != cudaSuccess) return e;
+  const bool vec4 = aligned(logp, 16) && aligned(logp_old, 16) && aligned(sid, 16) && aligned(mask, 4);
+  if (vec4)
+    seq_lvl_accum_kernel<true><<<grid_of(T), kThreads, 0, s>>>(logp, logp_old, mask, sid, T, n_seq, q, cnt, work);
+  else
+    seq_lvl_accum_kernel<false><<<grid_of(T), kThreads, 0, s>>>(logp, logp_old, mask, sid, T, n_seq, q, cnt, work);
+  seq_lvl_seq_kernel<<<seq_grid_of(n_seq), kThreads, 0, s>>>(adv_seq, n_seq, q, cnt, lo, hi, bounds,
+                                                             seq_ratio, seq_clip, coef, part, stats, work);
+  if (grad) {
+    const bool vec = aligned(sid, 16) && aligned(grad, 16) && aligned(mask, 4);
+    seq_lvl_grad_kernel<<<grid_of(T), kThreads, 0, s>>>(mask, sid, T, n_seq, coef, grad, vec);
+  }
   return cudaGetLastError();
 }
 
