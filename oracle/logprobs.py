@@ -27,6 +27,15 @@ from the unquantised BF16 operands:
   z[t, v]   = sum_k  h[t, k] * W[v, k]                        (bf16 values)
 
 again in float64, followed by the same log-softmax and gather.
+
+Backward through the lm_head (the step after dLoss/dlogits): with P the
+dLoss/dlogits above and the FP8 logits z of the forward pass,
+
+  dh[t, :] = sum_v P[t, v] W[v, :]        dW[v, :] = sum_t P[t, v] h[t, :]
+
+Reading: the quantisers pass the gradient straight through (their derivative
+is taken as the identity), so the contractions use the bf16 operands h and W
+the codes were quantised from.
 """
 
 import numpy as np
@@ -94,3 +103,25 @@ def dlogits(z, targets, lse, g):
     onehot = np.zeros_like(p)
     onehot[np.arange(z.shape[0]), np.asarray(targets, np.int64)] = 1.0
     return np.asarray(g, np.float64)[:, None] * (onehot - p)
+
+
+def lm_head_backward(h_codes, h_scales, w_codes, w_scales, gran, targets, g, h, W, rows=None):
+    """dLoss/dh and dLoss/dW of the FP8-scored log-probs, given g_t = dL/dlogp_t.
+
+    z from ``logits`` (float64, dequantised operands), lse from
+    ``log_softmax_gather``, P from ``dlogits``; then the two contractions with
+    the bf16 operands in float64.  With ``rows`` only those tokens are scored
+    and only dh for them is returned (dW needs every token)."""
+    y = np.asarray(targets, np.int64)
+    gg = np.asarray(g, np.float64)
+    if rows is not None:
+        rows = np.asarray(rows, np.int64)
+        y, gg = y[rows], gg[rows]
+    z = logits(h_codes, h_scales, w_codes, w_scales, gran, rows)
+    _, lse = log_softmax_gather(z, y)
+    P = dlogits(z, y, lse, gg)
+    W64 = np.asarray(W, np.float32).astype(np.float64)
+    out = {"P": P, "lse": lse, "dh": P @ W64}
+    if rows is None:
+        out["dW"] = P.T @ np.asarray(h, np.float32).astype(np.float64)
+    return out

@@ -178,3 +178,95 @@ def test_bf16_path_equals_fp8_path_on_exact_e4m3_operands():
     hq2, hs2 = Q.quantize(h2, Q.TENSOR, Q.ACT)
     assert not np.array_equal(L.token_logprobs(hq2, hs2, wq, ws, Q.TENSOR, y)[0],
                               L.bf16_token_logprobs(h2, W, y)[0])
+
+
+# ---- backward through the lm_head -------------------------------------------
+
+def _exact_operands(rng, shape, amax):
+    """Values e/512 for finite E4M3 values e, with one entry +-448/512: the
+    per-tensor scale fl32(amax/448) is exactly 2^-9 and every value divided by
+    it is an E4M3 value, so the codes decode to the inputs exactly."""
+    finite = np.array([c for c in range(256) if c not in (0x7F, 0xFF)], np.uint8)
+    vals = e4m3.decode(finite).astype(np.float64) / 512
+    x = rng.choice(vals, size=shape)
+    x.flat[0] = amax
+    return x
+
+
+def test_lm_head_backward_finite_difference():
+    # L(h, W) = sum_t g_t log_softmax(h W^T)[t, y_t], written out in float64
+    # from the operands; at an on-grid point (quantisation changes nothing)
+    # its gradient is the oracle's dh, dW
+    rng = np.random.default_rng(40)
+    T, H, V = 5, 16, 11
+    h = _exact_operands(rng, (T, H), 448.0 / 512)
+    W = _exact_operands(rng, (V, H), -448.0 / 512)
+    hq, hs = Q.quantize(h.astype(np.float32), Q.TENSOR, Q.ACT)
+    wq, ws = Q.quantize(W.astype(np.float32), Q.TENSOR, Q.WEIGHT)
+    assert hs[0] == 2.0 ** -9 and ws[0] == 2.0 ** -9
+    assert np.array_equal(Q.dequantize(hq, hs, Q.TENSOR, Q.ACT), h)
+    assert np.array_equal(Q.dequantize(wq, ws, Q.TENSOR, Q.WEIGHT), W)
+    y = rng.integers(0, V, T)
+    g = rng.normal(0, 1, T)
+
+    def loss(hh, WW):
+        z = hh @ WW.T
+        m = z.max(axis=1, keepdims=True)
+        lse = (m + np.log(np.exp(z - m).sum(axis=1, keepdims=True)))[:, 0]
+        return float(np.sum(g * (z[np.arange(T), y] - lse)))
+
+    out = L.lm_head_backward(hq, hs, wq, ws, Q.TENSOR, y, g, h, W)
+    eps = 1e-6
+    for (t, k) in [(0, 1), (2, 5), (4, 15), (1, 0)]:
+        e = np.zeros_like(h)
+        e[t, k] = eps
+        fd = (loss(h + e, W) - loss(h - e, W)) / (2 * eps)
+        assert abs(fd - out["dh"][t, k]) < 1e-7 * max(1.0, abs(fd)), (t, k)
+    for (v, k) in [(0, 0), (3, 7), (10, 15), (6, 2)]:
+        e = np.zeros_like(W)
+        e[v, k] = eps
+        fd = (loss(h, W + e) - loss(h, W - e)) / (2 * eps)
+        assert abs(fd - out["dW"][v, k]) < 1e-7 * max(1.0, abs(fd)), (v, k)
+
+
+def test_lm_head_backward_uniform_softmax_closed_form():
+    # all weight rows equal: the softmax is uniform, dh = 0 and
+    # dW[v] = sum_{t: y_t = v} g_t h_t - (1/V) sum_t g_t h_t
+    rng = np.random.default_rng(41)
+    T, H, V = 9, 32, 7
+    h = rng.normal(0, 1, (T, H)).astype(np.float32)
+    W = np.tile(rng.normal(0, 0.1, (1, H)), (V, 1)).astype(np.float32)
+    hq, hs = Q.quantize(h, Q.ROWWISE, Q.ACT)
+    wq, ws = Q.quantize(W, Q.ROWWISE, Q.WEIGHT)
+    y = rng.integers(0, V, T)
+    g = rng.normal(0, 1, T)
+    out = L.lm_head_backward(hq, hs, wq, ws, Q.ROWWISE, y, g, h, W)
+    assert np.abs(out["dh"]).max() < 1e-12
+    gh = g[:, None] * h.astype(np.float64)
+    want = np.zeros((V, H))
+    for t in range(T):
+        want[y[t]] += gh[t]
+    want -= gh.sum(axis=0) / V
+    assert np.allclose(out["dW"], want, rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("gran", [Q.TENSOR, Q.ROWWISE, Q.BLOCK])
+def test_lm_head_backward_invariants(gran):
+    rng = np.random.default_rng(42 + gran)
+    T, H, V = 6, 256, 300
+    h = rng.normal(0, 1, (T, H)).astype(np.float32)
+    W = rng.normal(0, 0.05, (V, H)).astype(np.float32)
+    hq, hs = Q.quantize(h, gran, Q.ACT)
+    wq, ws = Q.quantize(W, gran, Q.WEIGHT)
+    y = rng.integers(0, V, T)
+    g = rng.normal(0, 1, T)
+    out = L.lm_head_backward(hq, hs, wq, ws, gran, y, g, h, W)
+    # every row of P sums to g_t (1 - 1) = 0, so the columns of dW sum to 0
+    assert np.abs(out["P"].sum(axis=1)).max() < 1e-12
+    assert np.abs(out["dW"].sum(axis=0)).max() < 1e-10 * np.abs(out["dW"]).sum(axis=0).max()
+    # g = 0 gives nothing; rows= gives the same dh rows
+    z = L.lm_head_backward(hq, hs, wq, ws, gran, y, np.zeros(T), h, W)
+    assert not z["dh"].any() and not z["dW"].any()
+    part = L.lm_head_backward(hq, hs, wq, ws, gran, y, g, h, W, rows=[4, 1])
+    assert np.allclose(part["dh"], out["dh"][[4, 1]], rtol=0, atol=1e-13 * np.abs(out["dh"]).max())
+    assert "dW" not in part
