@@ -154,10 +154,14 @@ def select_workload(args):
     return w
 
 
-def kernels_per_step(gran, mode):
+def kernels_per_step(gran, mode, T):
+    """Kernel launches of one FP8 step: quantise h and W (amax + encode each
+    for per-tensor scaling), the GEMM, the combine, calibration (one
+    cooperative launch up to 2^18 tokens, else a pass and a decide launch per
+    stage: 9 stages exact, 3 grid), valid-token count and surrogate."""
     q = 2 if gran == 0 else 1
-    calib = 6 if mode == 1 else 18
-    return 2 * q + 2 + calib + 2
+    calib = 1 if T <= (1 << 18) else (6 if mode == 1 else 18)
+    return 2 * q + 1 + 1 + calib + 2
 
 
 def run_ours(args, rank, world, local_rank):
@@ -254,6 +258,31 @@ def run_ours(args, rank, world, local_rank):
     s1.record(stream)
     torch.cuda.synchronize()
     shadow_ms = s0.elapsed_time(s1) / n_shadow
+
+    # backward through the lm_head from this step's g (dh = P W, dW = P^T h with
+    # P = dLoss/dlogits recomputed from the FP8 logits), timed on its own
+    bwd = None
+    if not args.no_backward:
+        bws = torch.empty(api.lib.fp8rl_lm_head_backward_workspace_size(T, H, V), dtype=torch.uint8, device=dev)
+        bout = {"dh": torch.empty(T, H, device=dev), "dW": torch.empty(V, H, device=dev)}
+
+        def backward():
+            api.lm_head_backward(b.h_codes, b.h_scales, b.w_codes, b.w_scales, gran, y, b.lse, b.grad, h, W,
+                                 out=bout, workspace=bws)
+
+        backward()
+        torch.cuda.synchronize()
+        n_bwd = 3
+        b0 = torch.cuda.Event(enable_timing=True)
+        b1 = torch.cuda.Event(enable_timing=True)
+        b0.record(stream)
+        for _ in range(n_bwd):
+            backward()
+        b1.record(stream)
+        torch.cuda.synchronize()
+        api.check()
+        bwd = {"ms": b0.elapsed_time(b1) / n_bwd, "workspace_gb": bws.numel() / 1e9}
+        del bws, bout
     api.check()
 
     # same step through the public API with host buffers (copies inside the region)
@@ -353,7 +382,7 @@ def run_ours(args, rank, world, local_rank):
                 "note": "h, targets, logp_old, r_bf16, adv, mask, coef copied in from pinned host memory "
                         "(step i+1's copy overlaps step i on a side stream, double-buffered); stats, "
                         "bounds, dloss/dlogp read back every step; lm_head W is resident model state"},
-        "gpu_launches": kernels_per_step(gran, args.calib_mode) * args.steps,
+        "gpu_launches": kernels_per_step(gran, args.calib_mode, T) * args.steps,
         "clocks": clk,
         "result": {"lo": res["lo_new"], "hi": res["hi_new"], "loss": st["loss"],
                    "clip_frac_pos": st["clip_frac_pos"], "clip_frac_neg": st["clip_frac_neg"]},
@@ -361,6 +390,15 @@ def run_ours(args, rank, world, local_rank):
                                              "clipped_hi_fp8", "clipped_lo_bf16", "clipped_hi_bf16",
                                              "nmae_prob", "nmae_ratio")},
     }
+    if bwd is not None:
+        ideal_ms = (flops / (fp8_peak * 1e12) + 2 * flops / (peaks["bf16_tflops_sustained"] * 1e12)) * 1e3
+        bwd.update({"tflop_per_call": 3 * flops / 1e12, "tflops": 3 * flops / (bwd["ms"] * 1e-3) / 1e12,
+                    "ideal_ms": ideal_ms, "frac_of_roofline": ideal_ms / bwd["ms"],
+                    "note": "dh and dW from this step's dloss/dlogp: z recomputed on the FP8 GEMM with "
+                            "dlogits written in bf16 (both orientations), W and h transposed, dh and dW on "
+                            "the tcgen05 BF16 GEMM; ideal = 2THV at the FP8 peak + 4THV at the measured "
+                            "BF16 sustained peak"})
+        line["lm_head_backward"] = bwd
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = oracle_step_estimate(w, budget_s=args.cpu_budget)
     return line
@@ -581,6 +619,7 @@ def main():
     ap.add_argument("--calib-mode", type=int, default=0)
     ap.add_argument("--cpu-budget", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-backward", action="store_true", help="skip timing the lm_head backward")
     ap.add_argument("--kernels", action="store_true",
                     help="print HBM rooflines of the memory-bound kernels at stress sizes instead")
     ap.add_argument("--stress-scale", type=float, default=1.0,

@@ -391,6 +391,39 @@ fp8rl_status fp8rl_dlogits_rows(const uint8_t* h_codes, const float* h_scales,
                                 float* out, void* workspace, size_t workspace_bytes,
                                 void* stream);
 
+/* Backward through the FP8 lm_head (the chain rule of a3/a4 past the logits;
+ * the paper trains with FP8 forward and backward passes, §3 and the
+ * performance appendix).  With g_t = grad_logp[t] (e.g. from
+ * fp8rl_clipped_surrogate) and lse from fp8rl_token_logprobs:
+ *   P[t][v] = g_t (1{v == y_t} - exp(z[t][v] - lse_t)),  z recomputed by the
+ *             FP8 GEMM of fp8rl_token_logprobs and rounded to bf16 (P is
+ *             written to the workspace in both orientations; the float32
+ *             logits are never stored)
+ *   dh[t][k] = sum_v P[t][v] W[v][k]        float32 [T][H]
+ *   dW[v][k] = sum_t P[t][v] h[t][k]        float32 [V][H]
+ * The quantisers pass the gradient straight through: the two contractions
+ * run on tcgen05 in BF16 with float32 accumulation over the bf16 operands
+ * h_bf16 [T][H] and w_bf16 [V][H] that the codes were quantised from.
+ *   h_codes ... targets   as for fp8rl_token_logprobs (same granularity)
+ *   lse, grad_logp        float [T] DEVICE
+ *   dh, dW                float out, 16-byte aligned; either may be NULL to
+ *                         skip that contraction (not both)
+ *   accumulate_dw         nonzero: dW += (several token chunks, one dW)
+ * T and V at most 2^21.  Workspace (16-byte aligned) holds P twice and the
+ * transposed operands: 2 (T V' + V T' + H V' + H T') bytes, V' and T' rounded
+ * up to multiples of 8 (about 11.3 GB at T 16384, H 4096, V 151936); callers
+ * with less memory pass token chunks and accumulate dW. */
+size_t fp8rl_lm_head_backward_workspace_size(int64_t T, int64_t H, int64_t V);
+
+fp8rl_status fp8rl_lm_head_backward(const uint8_t* h_codes, const float* h_scales,
+                                    const uint8_t* w_codes, const float* w_scales,
+                                    fp8rl_gran gran, int64_t T, int64_t H, int64_t V,
+                                    const int32_t* targets, const float* lse,
+                                    const float* grad_logp, const void* h_bf16,
+                                    const void* w_bf16, float* dh, float* dW,
+                                    int accumulate_dw, void* workspace, size_t workspace_bytes,
+                                    void* stream);
+
 /* ---------------------------------------------------------------------- */
 /* §3 diagnostics against BF16 references; TIS weights (§2.3)               */
 /* ---------------------------------------------------------------------- */

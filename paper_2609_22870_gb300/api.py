@@ -96,6 +96,9 @@ _SIGS = {
     "fp8rl_surrogate_seq_mean_workspace_size": (_sz, [_i64, _i64]),
     "fp8rl_clipped_surrogate_seq_mean": (_i, [_p, _p, _p, _p, _p, _i64, _i64, _f, _f, _p, _p, _p, _p, _p,
                                               _sz, _p]),
+    "fp8rl_lm_head_backward_workspace_size": (_sz, [_i64, _i64, _i64]),
+    "fp8rl_lm_head_backward": (_i, [_p, _p, _p, _p, _i, _i64, _i64, _i64, _p, _p, _p, _p, _p, _p, _p, _i,
+                                    _p, _sz, _p]),
     "fp8rl_seq_level_surrogate_workspace_size": (_sz, [_i64, _i64]),
     "fp8rl_seq_level_clipped_surrogate": (_i, [_p, _p, _p, _p, _p, _i64, _i64, _f, _f, _p, _p, _p, _p, _p,
                                                _p, _sz, _p]),
@@ -440,6 +443,40 @@ def seq_level_clipped_surrogate(logp, logp_old, adv_seq, seq_id, mask=None, lo=0
                                               workspace.numel(), _stream(stream)),
         "fp8rl_seq_level_clipped_surrogate")
     return {"stats": stats, "seq_ratio": ratio, "seq_clip": clip, "grad": grad}
+
+
+def lm_head_backward(h_codes, h_scales, w_codes, w_scales, gran, targets, lse, grad_logp, h, W,
+                     want_dh=True, want_dw=True, accumulate_dw=False, out=None, workspace=None, stream=None):
+    """fp8rl_lm_head_backward -> dict(dh=[T][H] float32, dW=[V][H] float32).
+    ``h`` [T][H] and ``W`` [V][H] are the bf16 operands the codes came from;
+    ``out`` may hold preallocated "dh" / "dW" (with ``accumulate_dw`` the
+    given dW is added to)."""
+    T, H = h.shape
+    V = W.shape[0]
+    dev = h.device
+    _dev(h_codes, torch.uint8, "h_codes", T * H)
+    _dev(w_codes, torch.uint8, "w_codes", V * H)
+    _dev(h_scales, torch.float32, "h_scales")
+    _dev(w_scales, torch.float32, "w_scales")
+    _dev(targets, torch.int32, "targets", T)
+    _dev(lse, torch.float32, "lse", T)
+    _dev(grad_logp, torch.float32, "grad_logp", T)
+    _dev(h, torch.bfloat16, "h")
+    _dev(W, torch.bfloat16, "W")
+    o = out or {}
+    dh = (o.get("dh") if o.get("dh") is not None else torch.empty(T, H, dtype=torch.float32, device=dev)) \
+        if want_dh else None
+    dW = (o.get("dW") if o.get("dW") is not None else torch.empty(V, H, dtype=torch.float32, device=dev)) \
+        if want_dw else None
+    _dev(dh, torch.float32, "dh", T * H)
+    _dev(dW, torch.float32, "dW", V * H)
+    if workspace is None:
+        workspace = _workspace(lib.fp8rl_lm_head_backward_workspace_size(T, H, V), dev)
+    _ok(lib.fp8rl_lm_head_backward(_ptr(h_codes), _ptr(h_scales), _ptr(w_codes), _ptr(w_scales), int(gran),
+                                   T, H, V, _ptr(targets), _ptr(lse), _ptr(grad_logp), _ptr(h), _ptr(W),
+                                   _ptr(dh), _ptr(dW), int(bool(accumulate_dw)), _ptr(workspace),
+                                   workspace.numel(), _stream(stream)), "fp8rl_lm_head_backward")
+    return {"dh": dh, "dW": dW}
 
 
 def read_clip_stats(buf):

@@ -424,5 +424,30 @@ fp8rl_status fp8rl_dlogits_rows(const uint8_t* hc, const float* hs, const uint8_
   return e == cudaSuccess ? FP8RL_OK : cuda_fail(e);
 }
 
+// ------------------------------------------------------------------ lm_head backward
+size_t fp8rl_lm_head_backward_workspace_size(int64_t T, int64_t H, int64_t V) {
+  return (T < 1 || H < 1 || V < 1) ? 0 : bwd_layout(T, H, V).total;
+}
+
+fp8rl_status fp8rl_lm_head_backward(const uint8_t* hc, const float* hs, const uint8_t* wc,
+                                    const float* wsc, fp8rl_gran g, int64_t T, int64_t H, int64_t V,
+                                    const int32_t* targets, const float* lse, const float* grad,
+                                    const void* h_bf16, const void* w_bf16, float* dh, float* dW,
+                                    int accumulate_dw, void* ws, size_t ws_bytes, void* stream) {
+  fp8rl_status st = check_gemm_shape(hc, hs, wc, wsc, g, T, H, V);
+  if (st != FP8RL_OK) return st;
+  if (!targets || !lse || !grad || !h_bf16 || !w_bf16 || (!dh && !dW)) return FP8RL_EINVAL;
+  if (T > (int64_t{1} << 21) || V > (int64_t{1} << 21)) return FP8RL_ESHAPE;  // transpose grid
+  if (!aligned16(h_bf16) || !aligned16(w_bf16) || (dh && !aligned16(dh)) || (dW && !aligned16(dW)))
+    return FP8RL_EALIGN;
+  if (!ws || ws_bytes < bwd_layout(T, H, V).total) return FP8RL_EWORKSPACE;
+  if (!aligned16(ws)) return FP8RL_EALIGN;
+  cudaError_t e = launch_lm_head_backward(hc, hs, wc, wsc, g, T, H, V, targets, lse, grad,
+                                          static_cast<const uint16_t*>(h_bf16),
+                                          static_cast<const uint16_t*>(w_bf16), dh, dW, accumulate_dw,
+                                          ws, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? FP8RL_OK : cuda_fail(e);
+}
+
 }  // extern "C"
 #pragma GCC visibility pop

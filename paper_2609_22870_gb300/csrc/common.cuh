@@ -8,9 +8,16 @@
 #pragma once
 
 #include <cstdint>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
 namespace fp8rl {
+
+// Two floats as bf16 (round to nearest even), `lo` in the low 16 bits.
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
 
 // Status bits kept in each translation unit's device status word.
 constexpr uint32_t kErrDevice = 1u;   // bad input data seen by a kernel

@@ -66,7 +66,11 @@ constexpr uint64_t kDrainNs = 1000000000ull;
 
 enum { kTensor = FP8RL_GRAN_TENSOR, kRow = FP8RL_GRAN_ROWWISE, kBlock = FP8RL_GRAN_BLOCK, kBf16 = 3 };
 static_assert(kBf16 == kGemmBf16, "BF16 mode id shared with the host interface");
-enum { kEpiLse = 0, kEpiDlogits = 1 };
+// Epilogues: streaming LSE partials + target logit; dense dlogits rows (fp32);
+// dlogits of every token in bf16, both [M][N] and transposed [N][M] (the
+// operands of the two backward contractions); plain store of the fp32
+// accumulators (optionally added to what is there).
+enum { kEpiLse = 0, kEpiDlogits = 1, kEpiDense = 2, kEpiStore = 3 };
 
 struct Params {
   const float* a_scales;
@@ -77,6 +81,12 @@ struct Params {
   const float* lse;
   const float* grad;
   float* out;
+  uint16_t* p_out;   // kEpiDense: bf16 [M][ld_p]
+  uint16_t* pt_out;  // kEpiDense: bf16 [N][ld_pt]
+  int64_t ld_p, ld_pt;
+  float* c_out;      // kEpiStore: fp32 [M][ld_c]
+  int64_t ld_c;
+  int accumulate;
   int M, N, K;
   int num_m, num_n, num_kb;
   int n_chunks;
@@ -112,7 +122,7 @@ __device__ __forceinline__ void epi_begin(const Params& p, EpiState& e, int row,
   e.s = 0.f;
   e.zy = 0.f;
   e.j = -1;
-  if (row < p.M) {
+  if (EPI != kEpiStore && row < p.M) {
     const int y = p.targets[row];
     if (y >= 0 && y < p.N) e.j = y - col0;
   }
@@ -143,13 +153,62 @@ __device__ __forceinline__ void epi_consume32(const Params& p, EpiState& e, cons
       for (int i = 0; i < 32; ++i)
         if (i == jj) e.zy = z[i];
     }
-  } else {
+  } else if (EPI == kEpiDlogits) {
     const float l = p.lse[row], g = p.grad[row];
     float* o = p.out + static_cast<size_t>(row) * p.N + col0 + base;
     const int jj = e.j - base;
 #pragma unroll
     for (int i = 0; i < 32; ++i)
       if (i < ncol) o[i] = g * ((i == jj ? 1.f : 0.f) - expf(z[i] - l));
+  } else if (EPI == kEpiDense) {
+    const float l = p.lse[row], g = p.grad[row];
+    const int jj = e.j - base;
+    const int c = col0 + base;
+    uint32_t w[16];  // bf16 pairs, column order
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const float v0 = g * ((2 * i == jj ? 1.f : 0.f) - expf(z[2 * i] - l));
+      const float v1 = g * ((2 * i + 1 == jj ? 1.f : 0.f) - expf(z[2 * i + 1] - l));
+      w[i] = pack_bf16x2(v0, v1);
+    }
+    uint16_t* pr = p.p_out + static_cast<size_t>(row) * p.ld_p + c;  // 64-byte aligned
+    uint16_t* pt = p.pt_out + static_cast<size_t>(c) * p.ld_pt + row;
+    if (ncol >= 32) {
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        reinterpret_cast<uint4*>(pr)[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+#pragma unroll
+      for (int i = 0; i < 32; ++i)  // lanes are consecutive rows: 64 contiguous bytes per column
+        pt[static_cast<size_t>(i) * p.ld_pt] = static_cast<uint16_t>(w[i >> 1] >> (16 * (i & 1)));
+    } else {
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        if (i < ncol) {
+          const uint16_t b = static_cast<uint16_t>(w[i >> 1] >> (16 * (i & 1)));
+          pr[i] = b;
+          pt[static_cast<size_t>(i) * p.ld_pt] = b;
+        }
+    }
+  } else {  // kEpiStore
+    float* cr = p.c_out + static_cast<size_t>(row) * p.ld_c + col0 + base;  // 16-byte aligned
+    if (ncol >= 32) {
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        float4 v = make_float4(z[4 * q], z[4 * q + 1], z[4 * q + 2], z[4 * q + 3]);
+        if (p.accumulate) {
+          const float4 o = reinterpret_cast<const float4*>(cr)[q];
+          v.x += o.x;
+          v.y += o.y;
+          v.z += o.z;
+          v.w += o.w;
+        }
+        reinterpret_cast<float4*>(cr)[q] = v;
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        if (i < ncol) cr[i] = p.accumulate ? cr[i] + z[i] : z[i];
+    }
   }
 }
 
@@ -608,6 +667,13 @@ cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s) {
   p.lse = a.lse;
   p.grad = a.grad;
   p.out = a.out;
+  p.p_out = a.p_out;
+  p.pt_out = a.pt_out;
+  p.ld_p = a.ld_p;
+  p.ld_pt = a.ld_pt;
+  p.c_out = a.c_out;
+  p.ld_c = a.ld_c;
+  p.accumulate = a.accumulate;
   p.M = static_cast<int>(a.M);
   p.N = static_cast<int>(a.N);
   p.K = static_cast<int>(a.K);
@@ -619,11 +685,22 @@ cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s) {
   p.wait_limit_ns = wait_limit_ns();
   const int64_t tiles = static_cast<int64_t>(p.num_m) * p.num_n;
   const int grid = static_cast<int>(tiles < sm_count() ? tiles : sm_count());
-  switch (a.gran) {
-    case kTensor: return launch_mode<kTensor, EPI>(ta, tb, p, grid, s);
-    case kRow: return launch_mode<kRow, EPI>(ta, tb, p, grid, s);
-    case kBf16: return launch_mode<kBf16, EPI>(ta, tb, p, grid, s);
-    default: return launch_mode<kBlock, EPI>(ta, tb, p, grid, s);
+  if constexpr (EPI == kEpiStore) {  // the backward contractions: bf16 operands only
+    return a.gran == kBf16 ? launch_mode<kBf16, EPI>(ta, tb, p, grid, s) : cudaErrorInvalidValue;
+  } else if constexpr (EPI == kEpiDense) {  // recomputed FP8 logits only
+    switch (a.gran) {
+      case kTensor: return launch_mode<kTensor, EPI>(ta, tb, p, grid, s);
+      case kRow: return launch_mode<kRow, EPI>(ta, tb, p, grid, s);
+      case kBlock: return launch_mode<kBlock, EPI>(ta, tb, p, grid, s);
+      default: return cudaErrorInvalidValue;
+    }
+  } else {
+    switch (a.gran) {
+      case kTensor: return launch_mode<kTensor, EPI>(ta, tb, p, grid, s);
+      case kRow: return launch_mode<kRow, EPI>(ta, tb, p, grid, s);
+      case kBf16: return launch_mode<kBf16, EPI>(ta, tb, p, grid, s);
+      default: return launch_mode<kBlock, EPI>(ta, tb, p, grid, s);
+    }
   }
 }
 
@@ -641,6 +718,12 @@ cudaError_t launch_gemm_lse(const GemmArgs& a, cudaStream_t s) { return launch_g
 cudaError_t launch_gemm_dlogits(const GemmArgs& a, cudaStream_t s) {
   return launch_gemm<kEpiDlogits>(a, s);
 }
+
+cudaError_t launch_gemm_dense_dlogits(const GemmArgs& a, cudaStream_t s) {
+  return launch_gemm<kEpiDense>(a, s);
+}
+
+cudaError_t launch_gemm_store(const GemmArgs& a, cudaStream_t s) { return launch_gemm<kEpiStore>(a, s); }
 
 cudaError_t launch_ratios(const float* lp_new, const float* lp_old, int64_t T, float* r,
                           cudaStream_t s) {

@@ -37,6 +37,14 @@ struct GemmArgs {
   const float* lse;         // [M]
   const float* grad;        // [M]
   float* out;               // [M][N]
+  // dense dlogits epilogue (bf16, both orientations)
+  uint16_t* p_out;          // [M][ld_p]
+  uint16_t* pt_out;         // [N][ld_pt]
+  int64_t ld_p, ld_pt;
+  // store epilogue (fp32 accumulators)
+  float* c_out;             // [M][ld_c], 16-byte aligned, ld_c % 4 == 0
+  int64_t ld_c;
+  int accumulate;           // add to c_out instead of overwriting it
 };
 constexpr int kGemmBf16 = 3;
 
@@ -45,6 +53,20 @@ constexpr int kGemmBf16 = 3;
 int64_t gemm_partials_per_token(int64_t N);
 cudaError_t launch_gemm_lse(const GemmArgs& a, cudaStream_t s);
 cudaError_t launch_gemm_dlogits(const GemmArgs& a, cudaStream_t s);
+cudaError_t launch_gemm_dense_dlogits(const GemmArgs& a, cudaStream_t s);
+cudaError_t launch_gemm_store(const GemmArgs& a, cudaStream_t s);
+struct BwdLayout {
+  int64_t vp, tp;             // padded row lengths of P [T][vp] and P^T, h^T [.][tp]
+  size_t p, pt, wt, ht, total;  // byte offsets in the workspace
+};
+BwdLayout bwd_layout(int64_t T, int64_t H, int64_t V);
+cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const uint8_t* wc,
+                                    const float* wsc, int gran, int64_t T, int64_t H, int64_t V,
+                                    const int32_t* targets, const float* lse, const float* grad,
+                                    const uint16_t* h, const uint16_t* W, float* dh, float* dW,
+                                    int accumulate_dw, void* ws, cudaStream_t s);
+cudaError_t launch_transpose_bf16(const uint16_t* in, int64_t rows, int64_t cols, int64_t ld_in,
+                                  uint16_t* out, int64_t ld_out, cudaStream_t s);
 cudaError_t launch_combine(const float2* partials, const float* zy, const int32_t* targets,
                            const float* logp_old, float* logp, float* lse, float* ratio,
                            int64_t M, int64_t N, cudaStream_t s);
