@@ -236,77 +236,6 @@ size_t seq_counts_offset(int64_t T) {
   return align_up(sizeof(SeqWork) + sizeof(Partial) * static_cast<size_t>(grid_of(T)), 256);
 }
 
-// n_i per sequence, n_valid and S = #{i : n_i > 0} (counted by the atomics
-// that find a sequence's count still zero).  Each
-// warp walks its own contiguous range of tokens 32 at a time and carries the
-// count of the sequence it is in across steps (responses are usually
-// contiguous), so a sequence costs one atomic per warp that touches it rather
-// than one per step.  Tokens with an id outside [0, n_seq) flag bad input and
-// count nowhere.
-__global__ void __launch_bounds__(kThreads) seq_count_kernel(const uint8_t* __restrict__ mask,
-                                                             const int32_t* __restrict__ sid,
-                                                             int64_t T, int64_t n_seq,
-                                                             unsigned int* __restrict__ cnt,
-                                                             SeqWork* w) {
-  const int lane = threadIdx.x & 31;
-  const int64_t nwarps = static_cast<int64_t>(gridDim.x) * (kThreads / 32);
-  const int64_t wid = static_cast<int64_t>(blockIdx.x) * (kThreads / 32) + (threadIdx.x >> 5);
-  const int64_t per = ((T + nwarps - 1) / nwarps + 127) / 128 * 128;
-  const int64_t beg = wid * per, end = min(T, beg + per);
-  uint32_t nv = 0;
-  bool bad = false;
-  int cur_id = -1;        // warp-uniform: the sequence being counted and its count
-  unsigned cur_cnt = 0;
-  unsigned s_new = 0;     // lane 0: sequences this warp found empty
-  for (int64_t base = beg; base < end; base += 128) {
-    // four steps of 32 tokens: all loads issued before any is used
-    int idv[4];
-    bool on[4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int64_t t = base + u * 32 + lane;
-      idv[u] = t < end ? __ldg(sid + t) : -1;
-      on[u] = t < end && (!mask || __ldg(mask + t) != 0);
-    }
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      // runs of equal (raw) ids among the 32 tokens, in lane order; masked
-      // tokens keep their id, so padding inside a response does not split its
-      // run, and each run adds the number of its valid tokens
-      const int id = idv[u];
-      const bool in_range = id >= 0 && id < n_seq;
-      const bool valid = on[u] && in_range;
-      if (base + u * 32 + lane < end && !in_range) bad = true;  // masked tokens too
-      nv += valid;
-      const unsigned vbits = __ballot_sync(0xffffffffu, valid);
-      const int prev = __shfl_up_sync(0xffffffffu, id, 1);
-      unsigned heads = __ballot_sync(0xffffffffu, lane == 0 || id != prev);
-      while (heads) {
-        const int h = __ffs(heads) - 1;
-        heads &= heads - 1;
-        const int next = heads ? __ffs(heads) - 1 : 32;
-        const unsigned run = (next == 32 ? 0xffffffffu : ((1u << next) - 1u)) & ~((1u << h) - 1u);
-        const unsigned n = __popc(vbits & run);
-        if (n == 0) continue;  // no valid token in this run
-        const int run_id = __shfl_sync(0xffffffffu, id, h);
-        if (run_id == cur_id) {
-          cur_cnt += n;
-        } else {
-          if (cur_id >= 0 && lane == 0) s_new += atomicAdd(&cnt[cur_id], cur_cnt) == 0u;
-          cur_id = run_id;
-          cur_cnt = n;
-        }
-      }
-    }
-  }
-  if (cur_id >= 0 && lane == 0) s_new += atomicAdd(&cnt[cur_id], cur_cnt) == 0u;
-  if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(&d_status, kErrDevice);
-  const uint32_t s = __reduce_add_sync(0xffffffffu, nv);
-  if (lane == 0 && s) atomicAdd(&w->n_valid, static_cast<unsigned long long>(s));
-  // S: the atomics that found a sequence's count still zero
-  if (lane == 0 && s_new) atomicAdd(&w->n_seq_valid, s_new);
-}
-
 __global__ void __launch_bounds__(kThreads) seq_surrogate_kernel(
     const float* __restrict__ r, const float* __restrict__ adv, const uint8_t* __restrict__ mask,
     const float* __restrict__ wts, const int32_t* __restrict__ sid, int64_t T, int64_t n_seq,
@@ -448,12 +377,13 @@ SeqLvlLayout seq_lvl_layout(int64_t n_seq) {
 // sequence (warp sum, one pair of atomics), takes the step's last valid id as
 // the new current sequence, and sends any other token (a response shorter
 // than a step, or ids in no order) straight to the atomics.  Invalid tokens
-// add nothing whatever their id.
-template <bool VEC>
-__global__ void __launch_bounds__(kThreads) seq_lvl_accum_kernel(
+// add nothing whatever their id.  Without SUMS only the counts are formed (the
+// sequence-mean surrogate's count pass).
+template <bool VEC, bool SUMS, typename WorkT>
+__global__ void __launch_bounds__(kThreads) seq_accum_kernel(
     const float* __restrict__ logp, const float* __restrict__ logp_old,
     const uint8_t* __restrict__ mask, const int32_t* __restrict__ sid, int64_t T, int64_t n_seq,
-    unsigned long long* __restrict__ qsum, unsigned int* __restrict__ cnt, SeqLvlWork* w) {
+    unsigned long long* __restrict__ qsum, unsigned int* __restrict__ cnt, WorkT* w) {
   const int lane = threadIdx.x & 31;
   const int64_t nwarps = static_cast<int64_t>(gridDim.x) * (kThreads / 32);
   const int64_t wid = static_cast<int64_t>(blockIdx.x) * (kThreads / 32) + (threadIdx.x >> 5);
@@ -466,12 +396,14 @@ __global__ void __launch_bounds__(kThreads) seq_lvl_accum_kernel(
   unsigned acc_n = 0;
   auto flush = [&]() {
     long long q = acc_q;
+    if (SUMS) {
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
+      for (int o = 16; o > 0; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
+    }
     const unsigned n = __reduce_add_sync(0xffffffffu, acc_n);
     if (lane == 0 && n) {
       s_new += atomicAdd(&cnt[cur], n) == 0u;
-      atomicAdd(&qsum[cur], static_cast<unsigned long long>(q));
+      if (SUMS) atomicAdd(&qsum[cur], static_cast<unsigned long long>(q));
     }
     acc_q = 0;
     acc_n = 0;
@@ -483,12 +415,17 @@ __global__ void __launch_bounds__(kThreads) seq_lvl_accum_kernel(
     bool on[4];
     if (VEC && t0 + 3 < end) {
       const int4 iv = __ldg(reinterpret_cast<const int4*>(sid + t0));
-      const float4 a = __ldg(reinterpret_cast<const float4*>(logp + t0));
-      const float4 b = __ldg(reinterpret_cast<const float4*>(logp_old + t0));
       const uint32_t mv = mask ? __ldg(reinterpret_cast<const uint32_t*>(mask + t0)) : 0x01010101u;
       id[0] = iv.x, id[1] = iv.y, id[2] = iv.z, id[3] = iv.w;
-      lp[0] = a.x, lp[1] = a.y, lp[2] = a.z, lp[3] = a.w;
-      lo[0] = b.x, lo[1] = b.y, lo[2] = b.z, lo[3] = b.w;
+      if (SUMS) {
+        const float4 a = __ldg(reinterpret_cast<const float4*>(logp + t0));
+        const float4 b = __ldg(reinterpret_cast<const float4*>(logp_old + t0));
+        lp[0] = a.x, lp[1] = a.y, lp[2] = a.z, lp[3] = a.w;
+        lo[0] = b.x, lo[1] = b.y, lo[2] = b.z, lo[3] = b.w;
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) lp[k] = lo[k] = 0.f;
+      }
 #pragma unroll
       for (int k = 0; k < 4; ++k) on[k] = ((mv >> (8 * k)) & 0xFFu) != 0;
     } else {
@@ -497,8 +434,8 @@ __global__ void __launch_bounds__(kThreads) seq_lvl_accum_kernel(
         const int64_t t = t0 + k;
         const bool in = t < end;
         id[k] = in ? __ldg(sid + t) : 0;
-        lp[k] = in ? __ldg(logp + t) : 0.f;
-        lo[k] = in ? __ldg(logp_old + t) : 0.f;
+        lp[k] = SUMS && in ? __ldg(logp + t) : 0.f;
+        lo[k] = SUMS && in ? __ldg(logp_old + t) : 0.f;
         on[k] = in && (!mask || __ldg(mask + t) != 0);
         if (!in) id[k] = cur;  // past the end: nothing to add
       }
@@ -512,12 +449,12 @@ __global__ void __launch_bounds__(kThreads) seq_lvl_accum_kernel(
       if (t0 + k < end && !in_range) bad = true;  // masked tokens too
       v[k] = on[k] && in_range;
       float d = lp[k] - lo[k];
-      if (v[k] && !(fabsf(d) <= kSeqLvlDMax)) {  // out of range or NaN
+      if (SUMS && v[k] && !(fabsf(d) <= kSeqLvlDMax)) {  // out of range or NaN
         bad = true;
         d = d != d ? 0.f : fminf(fmaxf(d, -kSeqLvlDMax), kSeqLvlDMax);
       }
       // d 2^32 is exact in float32; the conversion rounds to nearest even
-      q[k] = v[k] ? __float2ll_rn(d * 4294967296.0f) : 0ll;
+      q[k] = SUMS && v[k] ? __float2ll_rn(d * 4294967296.0f) : 0ll;
       nv += v[k];
       match = match && (!v[k] || id[k] == cur);
     }
@@ -557,7 +494,7 @@ __global__ void __launch_bounds__(kThreads) seq_lvl_accum_kernel(
     for (int k = 0; k < 4; ++k)
       if (v[k]) {
         s_new += atomicAdd(&cnt[id[k]], 1u) == 0u;
-        atomicAdd(&qsum[id[k]], static_cast<unsigned long long>(q[k]));
+        if (SUMS) atomicAdd(&qsum[id[k]], static_cast<unsigned long long>(q[k]));
       }
   }
   flush();
@@ -724,7 +661,10 @@ cudaError_t launch_seq_surrogate(const float* r, const float* adv, const uint8_t
   if (e == cudaSuccess && n_seq > 0) e = cudaMemsetAsync(cnt, 0, static_cast<size_t>(n_seq) * 4, s);
   if (e != cudaSuccess) return e;
   const int grid = grid_of(T);
-  seq_count_kernel<<<grid, kThreads, 0, s>>>(mask, sid, T, n_seq, cnt, work);
+  if (aligned(sid, 16) && aligned(mask, 4))
+    seq_accum_kernel<true, false><<<grid, kThreads, 0, s>>>(nullptr, nullptr, mask, sid, T, n_seq, nullptr, cnt, work);
+  else
+    seq_accum_kernel<false, false><<<grid, kThreads, 0, s>>>(nullptr, nullptr, mask, sid, T, n_seq, nullptr, cnt, work);
   const bool vec = aligned(r, 16) && aligned(adv, 16) && aligned(sid, 16) && aligned(w, 16) &&
                    aligned(grad, 16) && aligned(mask, 4) && aligned(clip_mask, 4);
   seq_surrogate_kernel<<<grid, kThreads, 0, s>>>(r, adv, mask, w, sid, T, n_seq, cnt, lo, hi, bounds,
@@ -750,9 +690,9 @@ cudaError_t launch_seq_level(const float* logp, const float* logp_old, const flo
   if (e != cudaSuccess) return e;
   const bool vec4 = aligned(logp, 16) && aligned(logp_old, 16) && aligned(sid, 16) && aligned(mask, 4);
   if (vec4)
-    seq_lvl_accum_kernel<true><<<grid_of(T), kThreads, 0, s>>>(logp, logp_old, mask, sid, T, n_seq, q, cnt, work);
+    seq_accum_kernel<true, true><<<grid_of(T), kThreads, 0, s>>>(logp, logp_old, mask, sid, T, n_seq, q, cnt, work);
   else
-    seq_lvl_accum_kernel<false><<<grid_of(T), kThreads, 0, s>>>(logp, logp_old, mask, sid, T, n_seq, q, cnt, work);
+    seq_accum_kernel<false, true><<<grid_of(T), kThreads, 0, s>>>(logp, logp_old, mask, sid, T, n_seq, q, cnt, work);
   seq_lvl_seq_kernel<<<seq_grid_of(n_seq), kThreads, 0, s>>>(adv_seq, n_seq, q, cnt, lo, hi, bounds,
                                                              seq_ratio, seq_clip, coef, part, stats, work);
   if (grad) {
