@@ -89,22 +89,28 @@ struct Params {
   int accumulate;
   int M, N, K;
   int num_m, num_n, num_kb;
+  int band_m;  // row blocks per band of the tile order
   int n_chunks;
   uint64_t wait_limit_ns;
 };
 
 __device__ __forceinline__ void flag(uint32_t bits) { atomicOr(&d_status, bits); }
 
-// Tile order: bands of kBandM token blocks, and within a band the token block
-// varies fastest.  The 152 tiles in flight then share one or two vocabulary
-// tiles and a band of h codes small enough to stay in L2, so the lm_head codes
-// are read once per band and h codes about once.
+// Tile order: bands of band_m row blocks, and within a band the row block
+// varies fastest.  For the scoring GEMM (band of 64 token blocks) the 152
+// tiles in flight then share one or two vocabulary tiles and a band of h codes
+// small enough to stay in L2, so the lm_head codes are read once per band and
+// h codes about once.  The backward contractions have only 16 column tiles
+// (N = H) and long rows: a band of 16 row blocks keeps about half of them in
+// flight per row block, which roughly halves the re-reads of the A operand
+// against 64 at the cost of more passes over the B operand.
 constexpr int kBandM = 64;
+constexpr int kBandStore = 16;
 __device__ __forceinline__ void tile_coords(int tile, const Params& p, int& m_blk, int& n_blk) {
-  const int band = tile / (kBandM * p.num_n);
-  const int m_base = band * kBandM;
-  const int band_m = min(kBandM, p.num_m - m_base);
-  const int local = tile - band * kBandM * p.num_n;
+  const int band = tile / (p.band_m * p.num_n);
+  const int m_base = band * p.band_m;
+  const int band_m = min(p.band_m, p.num_m - m_base);
+  const int local = tile - band * p.band_m * p.num_n;
   m_blk = m_base + local % band_m;
   n_blk = local / band_m;
 }
@@ -679,6 +685,7 @@ cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s) {
   p.K = static_cast<int>(a.K);
   p.num_m = static_cast<int>((a.M + BM - 1) / BM);
   p.num_n = static_cast<int>((a.N + BN - 1) / BN);
+  p.band_m = EPI == kEpiStore ? kBandStore : kBandM;
   const int64_t bk_elems = bf16 ? BK / 2 : BK;  // K elements per 128-byte stage row
   p.num_kb = static_cast<int>((a.K + bk_elems - 1) / bk_elems);
   p.n_chunks = static_cast<int>((a.N + CHUNK - 1) / CHUNK);
