@@ -38,7 +38,7 @@ GRAN_NAMES = {0: "tensor", 1: "row", 2: "block"}
 # DRAM bytes (read + write) per launch of the GEMM kernel on the default
 # workload, from one ncu capture (profiles/fp8_gemm_kernel_block_T2048_full_and_grpo8b_traffic.md);
 # reported only while the kernel source is the one that was measured.
-GEMM_TRAFFIC = {"workload": "grpo_8b", "bytes": 1.478e9, "gemm_cu_sha256_prefix": "fbcfc574c4744c66"}
+GEMM_TRAFFIC = {"workload": "grpo_8b", "bytes": 2.227e9, "gemm_cu_sha256_prefix": "70b262157825d9a0"}
 
 
 def max_over_ranks(values, world, device="cpu"):
