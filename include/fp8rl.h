@@ -409,7 +409,7 @@ fp8rl_status fp8rl_dlogits_rows(const uint8_t* h_codes, const float* h_scales,
  *   dh, dW                float out, 16-byte aligned; either may be NULL to
  *                         skip that contraction (not both)
  *   accumulate_dw         nonzero: dW += (several token chunks, one dW)
- * T and V at most 2^21.  Workspace (16-byte aligned) holds P twice and the
+ * T and V at most 2097120 (65535 x 32).  Workspace (16-byte aligned) holds P twice and the
  * transposed operands: 2 (T V' + V T' + H V' + H T') bytes, V' and T' rounded
  * up to multiples of 8 (about 11.3 GB at T 16384, H 4096, V 151936); callers
  * with less memory pass token chunks and accumulate dW. */

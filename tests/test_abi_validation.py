@@ -1,0 +1,88 @@
+"""Host-side argument checks of the C ABI (no GPU needed: every call below is
+rejected before any CUDA call, so only the host logic runs)."""
+
+import ctypes
+import importlib.util
+import os
+import shutil
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def api():
+    if shutil.which("nvcc") is None and not os.path.exists("/usr/local/cuda/bin/nvcc"):
+        pytest.skip("no CUDA toolkit")
+    from paper_2609_22870_gb300 import _build
+    _build.build()
+    spec = importlib.util.spec_from_file_location("_api_validation", os.path.join(
+        ROOT, "paper_2609_22870_gb300", "api.py"))
+    mod = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mod)  # loads the library; calls nothing on the GPU
+    return mod
+
+
+P = ctypes.c_void_p(4096)      # a non-null, 16-byte aligned stand-in (never dereferenced)
+ODD = ctypes.c_void_p(4096 + 8)
+NULL = None
+
+
+def _bwd(api, T=64, H=128, V=256, gran=2, h=P, dh=P, dW=P, ws=P, ws_bytes=None, hc=P, lse=P):
+    if ws_bytes is None:
+        ws_bytes = api.lib.fp8rl_lm_head_backward_workspace_size(T, H, V)
+    return api.lib.fp8rl_lm_head_backward(hc, P, P, P, gran, T, H, V, P, lse, P, h, P, dh, dW, 0, ws,
+                                          ws_bytes, NULL)
+
+
+def test_lm_head_backward_workspace_size(api):
+    T, H, V = 16384, 4096, 151936
+
+    def up(x, a):
+        return (x + a - 1) // a * a
+    vp, tp = up(V, 8), up(T, 8)
+    parts = [T * vp * 2, V * tp * 2, H * vp * 2, H * tp * 2]
+    want = sum(up(p, 256) for p in parts)
+    assert api.lib.fp8rl_lm_head_backward_workspace_size(T, H, V) == want  # 11.34 GB
+    assert api.lib.fp8rl_lm_head_backward_workspace_size(0, H, V) == 0
+    assert api.lib.fp8rl_lm_head_backward_workspace_size(T, H, -1) == 0
+
+
+def test_lm_head_backward_rejects_bad_arguments(api):
+    assert _bwd(api, hc=NULL) == api.EINVAL
+    assert _bwd(api, lse=NULL) == api.EINVAL
+    assert _bwd(api, dh=NULL, dW=NULL) == api.EINVAL
+    assert _bwd(api, gran=7) == api.EINVAL
+    assert _bwd(api, T=0) == api.ESHAPE
+    assert _bwd(api, H=100) == api.ESHAPE          # not a multiple of 16
+    assert _bwd(api, H=192, gran=2) == api.ESHAPE  # block scaling needs H % 128 == 0
+    assert _bwd(api, T=65535 * 32 + 1) == api.ESHAPE
+    assert _bwd(api, V=65535 * 32 + 1) == api.ESHAPE
+    assert _bwd(api, h=ODD) == api.EALIGN
+    assert _bwd(api, dW=ODD) == api.EALIGN
+    assert _bwd(api, ws=NULL) == api.EWORKSPACE
+    assert _bwd(api, ws_bytes=1024) == api.EWORKSPACE
+
+
+def test_seq_level_surrogate_rejects_bad_arguments(api):
+    f = api.lib.fp8rl_seq_level_clipped_surrogate
+    ws = api.lib.fp8rl_seq_level_surrogate_workspace_size(100, 10)
+    assert ws > 0 and api.lib.fp8rl_seq_level_surrogate_workspace_size(-1, 10) == 0
+    # stats missing; logp missing with tokens; advantages missing with sequences
+    assert f(P, P, P, NULL, P, 10, 100, 0.8, 1.2, NULL, NULL, NULL, NULL, NULL, P, ws, NULL) == api.EINVAL
+    assert f(NULL, P, P, NULL, P, 10, 100, 0.8, 1.2, NULL, NULL, NULL, NULL, P, P, ws, NULL) == api.EINVAL
+    assert f(P, P, NULL, NULL, P, 10, 100, 0.8, 1.2, NULL, NULL, NULL, NULL, P, P, ws, NULL) == api.EINVAL
+    assert f(P, P, P, NULL, P, -1, 100, 0.8, 1.2, NULL, NULL, NULL, NULL, P, P, ws, NULL) == api.ESHAPE
+    assert f(P, P, P, NULL, P, 1 << 31, 100, 0.8, 1.2, NULL, NULL, NULL, NULL, P, P, ws, NULL) == api.ESHAPE
+    assert f(P, P, P, NULL, P, 10, 100, 0.8, 1.2, NULL, NULL, NULL, NULL, P, P, ws - 1, NULL) \
+        == api.EWORKSPACE
+
+
+def test_seq_mean_surrogate_rejects_bad_arguments(api):
+    f = api.lib.fp8rl_clipped_surrogate_seq_mean
+    ws = api.lib.fp8rl_surrogate_seq_mean_workspace_size(100, 10)
+    assert f(P, P, NULL, NULL, P, 10, 100, 0.8, 1.2, NULL, NULL, NULL, NULL, P, ws, NULL) == api.EINVAL
+    assert f(P, P, NULL, NULL, NULL, 10, 100, 0.8, 1.2, NULL, NULL, NULL, P, P, ws, NULL) == api.EINVAL
+    assert f(P, P, NULL, NULL, P, 10, -5, 0.8, 1.2, NULL, NULL, NULL, P, P, ws, NULL) == api.ESHAPE
+    assert f(P, P, NULL, NULL, P, 10, 100, 0.8, 1.2, NULL, NULL, NULL, P, NULL, ws, NULL) == api.EWORKSPACE
