@@ -5,9 +5,10 @@
  * The library runs every step on the GPU (NVIDIA GB300, sm_103a).  All tensor
  * pointers are DEVICE pointers owned by the caller unless a comment says
  * "host".  The library keeps no device allocation of its own besides a few
- * status words; scratch memory comes from the caller as a workspace whose size
- * the matching *_workspace_size() query returns (any alignment of 256 bytes or
- * more; the library zeroes what it needs itself).
+ * status words and the fixed scratch array of fp8rl_token_logprobs_noalloc;
+ * scratch memory comes from the caller as a workspace whose size the matching
+ * *_workspace_size() query returns (any alignment of 256 bytes or more; the
+ * library zeroes what it needs itself).
  *
  * Every compute call is asynchronous on `stream` (a cudaStream_t; NULL is the
  * legacy default stream) and returns host-detectable errors synchronously:
@@ -409,10 +410,14 @@ fp8rl_status fp8rl_dlogits_rows(const uint8_t* h_codes, const float* h_scales,
  *   dh, dW                float out, 16-byte aligned; either may be NULL to
  *                         skip that contraction (not both)
  *   accumulate_dw         nonzero: dW += (several token chunks, one dW)
- * T and V at most 2097120 (65535 x 32).  Workspace (16-byte aligned) holds P twice and the
- * transposed operands: 2 (T V' + V T' + H V' + H T') bytes, V' and T' rounded
- * up to multiples of 8 (about 11.3 GB at T 16384, H 4096, V 151936); callers
- * with less memory pass token chunks and accumulate dW. */
+ * T and V at most 2097120 (65535 x 32), else FP8RL_ESHAPE; misaligned h_bf16,
+ * w_bf16, dh, dW or workspace give FP8RL_EALIGN.  The workspace holds P twice
+ * and the transposed operands: 2 (T V' + V T' + H V' + H T') bytes, V' and T'
+ * rounded up to multiples of 8 (about 11.3 GB at T 16384, H 4096, V 151936);
+ * callers with less memory pass token chunks (granularity other than per
+ * tensor, so the chunk's codes are the batch's) and accumulate dW.  Target
+ * ids are not checked again here (fp8rl_token_logprobs flags them): an id
+ * outside [0, V) adds no one-hot term to its row of P. */
 size_t fp8rl_lm_head_backward_workspace_size(int64_t T, int64_t H, int64_t V);
 
 fp8rl_status fp8rl_lm_head_backward(const uint8_t* h_codes, const float* h_scales,
