@@ -184,6 +184,8 @@ def quantize(x, gran, role=ROLE_ACT, codes=None, scales=None, workspace=None, st
     scales = torch.empty(max(n, 1), dtype=torch.float32, device=x.device) if scales is None else scales
     _dev(codes, torch.uint8, "codes", rows * cols)
     _dev(scales, torch.float32, "scales")
+    if scales.numel() < n:
+        raise ValueError(f"scales: expected at least {n} elements, got {scales.numel()}")
     wsz = lib.fp8rl_quantize_workspace_size(rows, cols, gran, role)
     if workspace is None and wsz:
         workspace = _workspace(wsz, x.device)
@@ -198,7 +200,7 @@ def token_logprobs_workspace_size(T, H, V, gran):
     return int(lib.fp8rl_token_logprobs_workspace_size(T, H, V, gran))
 
 
-def _gemm_args(h_codes, h_scales, w_codes, w_scales, targets):
+def _gemm_args(h_codes, h_scales, w_codes, w_scales, targets, gran):
     T, H = h_codes.shape
     V = w_codes.shape[0]
     _dev(h_codes, torch.uint8, "h_codes")
@@ -208,13 +210,16 @@ def _gemm_args(h_codes, h_scales, w_codes, w_scales, targets):
     _dev(targets, torch.int32, "targets", T)
     if w_codes.shape[1] != H:
         raise ValueError("h_codes and w_codes disagree on the hidden size")
+    if h_scales.numel() < scales_count(T, H, gran, ROLE_ACT) or \
+            w_scales.numel() < scales_count(V, H, gran, ROLE_WEIGHT):
+        raise ValueError("h_scales / w_scales: fewer scales than the granularity needs")
     return T, H, V
 
 
 def token_logprobs(h_codes, h_scales, w_codes, w_scales, gran, targets, logp_old=None,
                    want_lse=True, want_ratio=None, workspace=None, out=None, stream=None):
     """fp8rl_token_logprobs -> dict(logp, lse, ratio) of float32 [T] tensors."""
-    T, H, V = _gemm_args(h_codes, h_scales, w_codes, w_scales, targets)
+    T, H, V = _gemm_args(h_codes, h_scales, w_codes, w_scales, targets, gran)
     dev = h_codes.device
     want_ratio = logp_old is not None if want_ratio is None else want_ratio
     _dev(logp_old, torch.float32, "logp_old", T)
@@ -236,7 +241,7 @@ def token_logprobs_noalloc(h_codes, h_scales, w_codes, w_scales, gran, targets, 
     """fp8rl_token_logprobs_noalloc: like token_logprobs, but the scratch is the
     library's fixed static array, for callers that cannot allocate a workspace
     (shapes needing more than FP8RL_NOALLOC_SCRATCH_BYTES are refused)."""
-    T, H, V = _gemm_args(h_codes, h_scales, w_codes, w_scales, targets)
+    T, H, V = _gemm_args(h_codes, h_scales, w_codes, w_scales, targets, gran)
     dev = h_codes.device
     want_ratio = logp_old is not None if want_ratio is None else want_ratio
     _dev(logp_old, torch.float32, "logp_old", T)
@@ -253,7 +258,7 @@ def token_logprobs_noalloc(h_codes, h_scales, w_codes, w_scales, gran, targets, 
 
 def logit_partials(h_codes, h_scales, w_codes, w_scales, gran, targets, workspace, stream=None):
     """fp8rl_logit_partials: the FP8 GEMM + streaming logsumexp half."""
-    T, H, V = _gemm_args(h_codes, h_scales, w_codes, w_scales, targets)
+    T, H, V = _gemm_args(h_codes, h_scales, w_codes, w_scales, targets, gran)
     _ok(lib.fp8rl_logit_partials(_ptr(h_codes), _ptr(h_scales), _ptr(w_codes), _ptr(w_scales), gran,
                                  T, H, V, _ptr(targets), _ptr(workspace), workspace.numel(),
                                  _stream(stream)), "fp8rl_logit_partials")
@@ -451,18 +456,12 @@ def lm_head_backward(h_codes, h_scales, w_codes, w_scales, gran, targets, lse, g
     ``h`` [T][H] and ``W`` [V][H] are the bf16 operands the codes came from;
     ``out`` may hold preallocated "dh" / "dW" (with ``accumulate_dw`` the
     given dW is added to)."""
-    T, H = h.shape
-    V = W.shape[0]
+    T, H, V = _gemm_args(h_codes, h_scales, w_codes, w_scales, targets, gran)
     dev = h.device
-    _dev(h_codes, torch.uint8, "h_codes", T * H)
-    _dev(w_codes, torch.uint8, "w_codes", V * H)
-    _dev(h_scales, torch.float32, "h_scales")
-    _dev(w_scales, torch.float32, "w_scales")
-    _dev(targets, torch.int32, "targets", T)
     _dev(lse, torch.float32, "lse", T)
     _dev(grad_logp, torch.float32, "grad_logp", T)
-    _dev(h, torch.bfloat16, "h")
-    _dev(W, torch.bfloat16, "W")
+    _dev(h, torch.bfloat16, "h", T * H)
+    _dev(W, torch.bfloat16, "W", V * H)
     o = out or {}
     dh = (o.get("dh") if o.get("dh") is not None else torch.empty(T, H, dtype=torch.float32, device=dev)) \
         if want_dh else None
@@ -531,7 +530,7 @@ def tis_weights(logp_old, logp_sampler, C=2.0, out=None, stream=None):
 def dlogits_rows(h_codes, h_scales, w_codes, w_scales, gran, targets, lse, grad_logp, rows,
                  out=None, workspace=None, stream=None):
     """fp8rl_dlogits_rows -> float32 [n_rows][V] dense dLoss/dlogits."""
-    T, H, V = _gemm_args(h_codes, h_scales, w_codes, w_scales, targets)
+    T, H, V = _gemm_args(h_codes, h_scales, w_codes, w_scales, targets, gran)
     _dev(lse, torch.float32, "lse", T)
     _dev(grad_logp, torch.float32, "grad_logp", T)
     _dev(rows, torch.int64, "rows")
