@@ -77,3 +77,52 @@ def test_struct_layouts_match_binding(libpath, tmp_path):
     spec.loader.exec_module(api)  # loads the library; calls nothing on the GPU
     assert sizes == [ctypes.sizeof(api.CalibOpts), ctypes.sizeof(api.CalibResult),
                      ctypes.sizeof(api.ClipStats)]
+
+
+def test_c_program_links_and_runs(libpath, tmp_path):
+    """A plain C consumer links against libfp8rl.so and uses the host-side part
+    of the ABI: paper defaults, status strings, size queries and the argument
+    checks (every call below returns before any CUDA call)."""
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no gcc")
+    src = tmp_path / "consumer.c"
+    src.write_text(r'''
+#include <math.h>
+#include <stdio.h>
+#include <string.h>
+#include "fp8rl.h"
+#define CHECK(c) do { if (!(c)) { printf("FAIL %s\n", #c); return 1; } } while (0)
+int main(void) {
+  fp8rl_calib_opts o;
+  fp8rl_default_calib_opts(&o);
+  CHECK(o.mode == FP8RL_CALIB_EXACT && o.lo_min == 0.5 && o.lo_max == 0.9);
+  CHECK(o.hi_min == 1.2 && o.hi_max == 2.0 && o.step == 0.02);
+  CHECK(o.delta_lo == 0.05 && o.delta_hi == 0.1 && isnan(o.lo_old) && isnan(o.hi_old));
+  for (int s = FP8RL_OK; s <= FP8RL_ETIMEOUT; ++s)
+    CHECK(fp8rl_status_string((fp8rl_status)s) != NULL && strlen(fp8rl_status_string((fp8rl_status)s)) > 0);
+  CHECK(fp8rl_scales_count(16384, 4096, FP8RL_GRAN_BLOCK, FP8RL_ROLE_ACT) == 16384 * 32);
+  CHECK(fp8rl_scales_count(151936, 4096, FP8RL_GRAN_BLOCK, FP8RL_ROLE_WEIGHT) == 1187 * 32);
+  CHECK(fp8rl_scales_count(151936, 4096, FP8RL_GRAN_ROWWISE, FP8RL_ROLE_WEIGHT) == 151936);
+  CHECK(fp8rl_scales_count(7, 4096, FP8RL_GRAN_TENSOR, FP8RL_ROLE_ACT) == 1);
+  CHECK(fp8rl_token_logprobs_workspace_size(16384, 4096, 151936, FP8RL_GRAN_BLOCK) > 0);
+  CHECK(fp8rl_lm_head_backward_workspace_size(16384, 4096, 151936) > (size_t)11e9);
+  /* argument checks: null pointers, bad enums and shapes are refused on the host */
+  CHECK(fp8rl_quantize(NULL, 4, 128, 128, FP8RL_GRAN_ROWWISE, FP8RL_ROLE_ACT, NULL, NULL, NULL, 0, NULL)
+        == FP8RL_EINVAL);
+  CHECK(fp8rl_token_logprobs(NULL, NULL, NULL, NULL, FP8RL_GRAN_BLOCK, 16, 128, 64, NULL, NULL, NULL,
+                             NULL, NULL, NULL, 0, NULL) == FP8RL_EINVAL);
+  CHECK(fp8rl_calibrate_clip_bounds(NULL, NULL, NULL, NULL, NULL, 10, 0.2f, 0.2f, NULL, NULL, NULL, 0,
+                                    NULL) == FP8RL_EINVAL);
+  printf("ok\n");
+  return 0;
+}
+''')
+    exe = tmp_path / "consumer"
+    libdir = os.path.dirname(libpath)
+    r = subprocess.run([gcc, "-std=c99", "-Wall", "-Werror", str(src), "-I", os.path.join(ROOT, "include"),
+                        "-L", libdir, "-lfp8rl", "-Wl,-rpath," + libdir, "-lm", "-o", str(exe)],
+                       capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    run = subprocess.run([str(exe)], capture_output=True, text=True, timeout=60)
+    assert run.returncode == 0 and run.stdout.strip() == "ok", run.stdout + run.stderr
