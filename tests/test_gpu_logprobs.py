@@ -125,3 +125,16 @@ def test_dlogits_tiny_grpo_all_rows(cuda_lib):
     _, ref_lse, z = oracle_logprobs_rows(h, W, w.gran, y, np.arange(w.T))
     ref = OL.dlogits(z, y.cpu().numpy(), ref_lse, g.cpu().numpy())
     assert np.all(np.abs(d - ref) <= TOL * np.abs(g.cpu().numpy())[:, None] + 1e-12)
+
+
+@pytest.mark.parametrize("gran", [OQ.BLOCK, OQ.TENSOR])
+def test_logprobs_bit_reproducible_full_size(cuda_lib, gran):
+    """No atomics on the scoring path: two calls on the grpo_8b batch give the
+    same bits for logp, lse and the ratios."""
+    w = synth.WORKLOADS["grpo_8b"]
+    h, W, y = synth.hidden_states(w, "cuda"), synth.lm_head_weight(w, "cuda"), synth.targets(w, "cuda")
+    logp_old = (torch.full((w.T,), -12.0) + synth.old_policy_noise(w)).float().cuda()
+    a, _ = _score(cuda_lib, h, W, y, gran, logp_old)
+    b, _ = _score(cuda_lib, h, W, y, gran, logp_old)
+    for k in ("logp", "lse", "ratio"):
+        assert torch.equal(a[k], b[k]), k
