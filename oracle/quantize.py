@@ -23,6 +23,11 @@ Readings taken where the paper is silent:
   (V not a multiple of 128) takes its amax over the rows that exist; the
   hidden size must be a multiple of 128 in block mode.
 
+Power-of-two (UE8M0) variant, outside the paper (its S is amax / 448): the
+scale format that the hardware's block-scaled MMA takes.  S is rounded up to
+the smallest power of two not below fl32(amax / 448), so |x / S| <= 448 still
+holds and x / S is exact; amax == 0 gives S = 1.
+
 Scales are returned in their natural shapes:
   tensor: (1,);  row: (rows,);  act block: (rows, cols/128);
   weight block: (ceil(rows/128), cols/128).
@@ -45,17 +50,27 @@ def scale_from_amax(amax):
     return np.where(amax == 0, np.float32(1.0), s).astype(np.float32)
 
 
+def pow2_scale_from_amax(amax):
+    """S = 2^ceil(log2(fl32(amax / F_max))); 1.0 where amax == 0."""
+    s = scale_from_amax(amax).astype(np.float64)
+    m, e = np.frexp(s)  # s = m 2^e, m in [0.5, 1)
+    p = np.where(m == 0.5, s, np.ldexp(1.0, e))
+    return p.astype(np.float32)
+
+
 def _encode_block(x, s):
     """Q_FP8(fl32(x / S)) for a block x with its scale s (broadcastable)."""
     q = (x.astype(np.float32) / np.asarray(s, dtype=np.float32)).astype(np.float32)
     return e4m3.encode(q)
 
 
-def quantize(x, gran, role=ACT):
+def quantize(x, gran, role=ACT, pow2=False):
     """Quantise a 2-D float32 array (bf16-valued) at the given granularity.
 
     Returns (codes uint8 [rows][cols], scales float32 in natural shape).
+    ``pow2`` selects the power-of-two (UE8M0) scales.
     """
+    scale_from = pow2_scale_from_amax if pow2 else scale_from_amax
     x = np.asarray(x, dtype=np.float32)
     if x.ndim != 2:
         raise ValueError("quantize: 2-D input expected")
@@ -63,12 +78,12 @@ def quantize(x, gran, role=ACT):
     if not np.all(np.isfinite(x)):
         raise ValueError("quantize: non-finite input")
     if gran == TENSOR:
-        s = scale_from_amax(np.max(np.abs(x)) if x.size else np.float32(0))
+        s = scale_from(np.max(np.abs(x)) if x.size else np.float32(0))
         s = np.asarray(s, dtype=np.float32).reshape(1)
         return _encode_block(x, s[0]), s
     if gran == ROWWISE:
         amax = np.max(np.abs(x), axis=1) if cols else np.zeros(rows, np.float32)
-        s = scale_from_amax(amax)
+        s = scale_from(amax)
         return _encode_block(x, s[:, None]), s
     if gran != BLOCK:
         raise ValueError("quantize: unknown granularity")
@@ -77,7 +92,7 @@ def quantize(x, gran, role=ACT):
     nkb = cols // BLOCK_K
     if role == ACT:
         xb = x.reshape(rows, nkb, BLOCK_K)
-        s = scale_from_amax(np.max(np.abs(xb), axis=2))  # (rows, nkb)
+        s = scale_from(np.max(np.abs(xb), axis=2))  # (rows, nkb)
         codes = _encode_block(xb, s[:, :, None]).reshape(rows, cols)
         return codes, s
     # weight: 128 x 128 blocks, tail rows along V allowed; one 128-row strip
@@ -88,7 +103,7 @@ def quantize(x, gran, role=ACT):
     for rb in range(nrb):
         r0, r1 = rb * BLOCK_W, min(rows, (rb + 1) * BLOCK_W)
         strip = x[r0:r1].reshape(r1 - r0, nkb, BLOCK_K)
-        sb = scale_from_amax(np.max(np.abs(strip), axis=(0, 2)))  # (nkb,)
+        sb = scale_from(np.max(np.abs(strip), axis=(0, 2)))  # (nkb,)
         s[rb] = sb
         codes[r0:r1] = _encode_block(strip, sb[None, :, None]).reshape(r1 - r0, cols)
     return codes, s

@@ -128,3 +128,64 @@ def test_weight_block_tail_rows():
     assert s.shape == (2, 1)
     c2, s2 = Q.quantize(x[128:], Q.TENSOR)
     assert np.array_equal(c[128:], c2) and s[1, 0] == s2[0]
+
+
+# ---- power-of-two (UE8M0) scales ----------------------------------------------
+
+def test_pow2_scale_closed_form():
+    amax = np.array([0.0, 448.0, 224.0, 448.0 * 3, 1.0, 2.0 ** -130, 300.0], np.float32)
+    s = Q.pow2_scale_from_amax(amax)
+    plain = Q.scale_from_amax(amax).astype(np.float64)
+    assert s[0] == 1.0 and s[1] == 1.0 and s[2] == 0.5 and s[3] == 4.0
+    m, _ = np.frexp(s[1:].astype(np.float64))
+    assert np.all(m == 0.5)  # powers of two
+    assert np.all(s[1:] >= plain[1:]) and np.all(s[1:] < 2 * plain[1:])
+
+
+def _per_element(s, gran, role, rows, cols):
+    """Scales broadcast to the element grid."""
+    s = np.asarray(s, np.float64)
+    if gran == Q.TENSOR:
+        return np.full((rows, cols), s[0])
+    if gran == Q.ROWWISE:
+        return np.repeat(s[:, None], cols, axis=1)
+    if role == Q.ACT:
+        return np.repeat(s, 128, axis=1)
+    return np.repeat(np.repeat(s, 128, axis=0)[:rows], 128, axis=1)
+
+
+@pytest.mark.parametrize("gran,role", [(Q.TENSOR, Q.ACT), (Q.ROWWISE, Q.ACT), (Q.BLOCK, Q.ACT),
+                                       (Q.BLOCK, Q.WEIGHT)])
+def test_pow2_quantize_bounds_and_agreement(gran, role):
+    rng = np.random.default_rng(50 + gran + role)
+    rows, cols = 300, 256
+    x = (rng.standard_normal((rows, cols)) * np.exp2(rng.integers(-8, 8, (rows, 1)))).astype(np.float32)
+    codes, s = Q.quantize(x, gran, role, pow2=True)
+    m, _ = np.frexp(s.astype(np.float64))
+    assert np.all(m == 0.5)
+    S = _per_element(s, gran, role, rows, cols)
+    # x / S is exact and at most 448 in magnitude, so each code is x / S rounded
+    # to nearest: within half an E4M3 quantum (2^-4 relative in the normal
+    # range, 2^-10 absolute below 2^-6)
+    assert np.all(np.abs(x / S) <= 448)
+    err = np.abs(Q.dequantize(codes, s, gran, role) - x.astype(np.float64))
+    assert np.all(err <= np.maximum(np.abs(x) * 2.0 ** -4, S * 2.0 ** -10))
+    # where the paper's S is already a power of two the codes agree bit for bit:
+    # give every row / block an element of magnitude 448 * 2^k
+    # (rows scaled into [-1, 1]; every maximum over a row, block or the tensor is
+    # then one of the planted values)
+    y = (x / np.max(np.abs(x), axis=1, keepdims=True)).astype(np.float32)
+    for c0 in range(0, cols, 128):
+        y[:, c0] = np.float32(448.0) * np.exp2(rng.integers(-2, 6, rows)).astype(np.float32)
+    pc, ps = Q.quantize(y, gran, role, pow2=True)
+    qc, qs = Q.quantize(y, gran, role)
+    assert np.array_equal(ps, qs) and np.array_equal(pc, qc)
+
+
+def test_pow2_amax_element_keeps_at_least_half_the_range():
+    rng = np.random.default_rng(53)
+    x = rng.standard_normal((64, 128)).astype(np.float32)
+    codes, s = Q.quantize(x, Q.ROWWISE, Q.ACT, pow2=True)
+    amax_idx = np.argmax(np.abs(x), axis=1)
+    top = e4m3.decode(codes[np.arange(64), amax_idx] & 0x7F)
+    assert np.all(top >= 224) and np.all(top <= 448)  # S < 2 fl32(amax/448): amax / S > 224
