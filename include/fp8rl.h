@@ -105,6 +105,18 @@ fp8rl_status fp8rl_quantize(const void* x, int64_t rows, int64_t cols, int64_t l
                             uint8_t* codes, float* scales,
                             void* workspace, size_t workspace_bytes, void* stream);
 
+/* fp8rl_quantize with power-of-two (UE8M0) scales, a variant outside the paper
+ * (whose S is amax / 448): the scale format the hardware's block-scaled MMA
+ * takes.  S = 2^ceil(log2(fl32(amax / 448))), the smallest power of two not
+ * below the paper's scale (1 for an all-zero group), so |x / S| <= 448 and
+ * x / S is exact; codes = Q_FP8(x / S).  Arguments, layouts, workspace and
+ * errors are those of fp8rl_quantize; the codes and scales feed
+ * fp8rl_token_logprobs at the same granularity like any other. */
+fp8rl_status fp8rl_quantize_ue8m0(const void* x, int64_t rows, int64_t cols, int64_t ld,
+                                  fp8rl_gran gran, fp8rl_role role,
+                                  uint8_t* codes, float* scales,
+                                  void* workspace, size_t workspace_bytes, void* stream);
+
 /* ---------------------------------------------------------------------- */
 /* a3/a4: FP8 lm_head scoring with online logsumexp and target gather       */
 /* ---------------------------------------------------------------------- */

@@ -75,6 +75,7 @@ _SIGS = {
     "fp8rl_scales_count": (_i64, [_i64, _i64, _i, _i]),
     "fp8rl_quantize_workspace_size": (_sz, [_i64, _i64, _i, _i]),
     "fp8rl_quantize": (_i, [_p, _i64, _i64, _i64, _i, _i, _p, _p, _p, _sz, _p]),
+    "fp8rl_quantize_ue8m0": (_i, [_p, _i64, _i64, _i64, _i, _i, _p, _p, _p, _sz, _p]),
     "fp8rl_token_logprobs_workspace_size": (_sz, [_i64, _i64, _i64, _i]),
     "fp8rl_token_logprobs": (_i, [_p, _p, _p, _p, _i, _i64, _i64, _i64, _p, _p, _p, _p, _p, _p, _sz, _p]),
     "fp8rl_logit_partials": (_i, [_p, _p, _p, _p, _i, _i64, _i64, _i64, _p, _p, _sz, _p]),
@@ -174,8 +175,9 @@ def scales_count(rows, cols, gran, role):
     return int(lib.fp8rl_scales_count(rows, cols, gran, role))
 
 
-def quantize(x, gran, role=ROLE_ACT, codes=None, scales=None, workspace=None, stream=None):
-    """fp8rl_quantize of a 2-D bf16 CUDA tensor -> (codes uint8, scales float32)."""
+def quantize(x, gran, role=ROLE_ACT, codes=None, scales=None, workspace=None, stream=None, ue8m0=False):
+    """fp8rl_quantize of a 2-D bf16 CUDA tensor -> (codes uint8, scales float32);
+    with ``ue8m0`` fp8rl_quantize_ue8m0 (power-of-two scales)."""
     if x.dim() != 2 or x.dtype != torch.bfloat16 or not x.is_cuda or x.stride(1) != 1:
         raise ValueError("x: expected a 2-D CUDA bf16 tensor with unit column stride")
     rows, cols = x.shape
@@ -189,9 +191,10 @@ def quantize(x, gran, role=ROLE_ACT, codes=None, scales=None, workspace=None, st
     wsz = lib.fp8rl_quantize_workspace_size(rows, cols, gran, role)
     if workspace is None and wsz:
         workspace = _workspace(wsz, x.device)
-    _ok(lib.fp8rl_quantize(_ptr(x), rows, cols, x.stride(0), gran, role, _ptr(codes), _ptr(scales),
-                           _ptr(workspace), 0 if workspace is None else workspace.numel(),
-                           _stream(stream)), "fp8rl_quantize")
+    fn = lib.fp8rl_quantize_ue8m0 if ue8m0 else lib.fp8rl_quantize
+    _ok(fn(_ptr(x), rows, cols, x.stride(0), gran, role, _ptr(codes), _ptr(scales),
+           _ptr(workspace), 0 if workspace is None else workspace.numel(),
+           _stream(stream)), "fp8rl_quantize_ue8m0" if ue8m0 else "fp8rl_quantize")
     return codes, scales
 
 

@@ -132,9 +132,10 @@ size_t fp8rl_quantize_workspace_size(int64_t, int64_t, fp8rl_gran g, fp8rl_role)
   return g == FP8RL_GRAN_TENSOR ? 256 : 0;
 }
 
-fp8rl_status fp8rl_quantize(const void* x, int64_t rows, int64_t cols, int64_t ld, fp8rl_gran g,
-                            fp8rl_role role, uint8_t* codes, float* scales, void* ws,
-                            size_t ws_bytes, void* stream) {
+namespace {
+fp8rl_status quantize_impl(const void* x, int64_t rows, int64_t cols, int64_t ld, fp8rl_gran g,
+                           fp8rl_role role, uint8_t* codes, float* scales, void* ws,
+                           size_t ws_bytes, bool pow2, void* stream) {
   if (!x || !codes || !scales || !valid_gran(g)) return FP8RL_EINVAL;
   if (role != FP8RL_ROLE_ACT && role != FP8RL_ROLE_WEIGHT) return FP8RL_EINVAL;
   if (rows < 0 || cols < 16 || ld < cols) return FP8RL_ESHAPE;
@@ -142,9 +143,22 @@ fp8rl_status fp8rl_quantize(const void* x, int64_t rows, int64_t cols, int64_t l
   if (!aligned16(x) || !aligned16(codes) || ld % 8 != 0) return FP8RL_EALIGN;
   const size_t need = fp8rl_quantize_workspace_size(rows, cols, g, role);
   if (need && (!ws || ws_bytes < need)) return FP8RL_EWORKSPACE;
-  cudaError_t e = launch_quantize(x, rows, cols, ld, g, role, codes, scales, ws,
+  cudaError_t e = launch_quantize(x, rows, cols, ld, g, role, codes, scales, ws, pow2,
                                   static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? FP8RL_OK : cuda_fail(e);
+}
+}  // namespace
+
+fp8rl_status fp8rl_quantize(const void* x, int64_t rows, int64_t cols, int64_t ld, fp8rl_gran g,
+                            fp8rl_role role, uint8_t* codes, float* scales, void* ws,
+                            size_t ws_bytes, void* stream) {
+  return quantize_impl(x, rows, cols, ld, g, role, codes, scales, ws, ws_bytes, false, stream);
+}
+
+fp8rl_status fp8rl_quantize_ue8m0(const void* x, int64_t rows, int64_t cols, int64_t ld,
+                                  fp8rl_gran g, fp8rl_role role, uint8_t* codes, float* scales,
+                                  void* ws, size_t ws_bytes, void* stream) {
+  return quantize_impl(x, rows, cols, ld, g, role, codes, scales, ws, ws_bytes, true, stream);
 }
 
 // ------------------------------------------------------------------ scoring

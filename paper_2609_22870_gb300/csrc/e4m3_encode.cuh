@@ -58,9 +58,22 @@ __device__ __forceinline__ float amax_of(uint32_t m) {
   return __uint_as_float((hi > lo ? hi : lo) << 16);
 }
 
-// S = fl32(amax / 448), 1 when amax == 0 (an all-zero block keeps S = 1).
-__device__ __forceinline__ float e4m3_scale(float amax) {
-  return amax == 0.f ? 1.f : __fdiv_rn(amax, kE4M3Max);
+// The smallest power of two not below t (t > 0 and finite; t < 2^119 here).
+__device__ __forceinline__ float pow2_ceil(float t) {
+  const uint32_t b = __float_as_uint(t);
+  const uint32_t ex = b >> 23, man = b & 0x7FFFFFu;
+  if (man == 0) return t;                              // a normal power of two
+  if (ex != 0) return __uint_as_float((ex + 1) << 23);  // next binade
+  const int h = 31 - __clz(man);                       // subnormal: highest set bit
+  return man == (1u << h) ? t : __uint_as_float(1u << (h + 1));
+}
+
+// S = fl32(amax / 448), 1 when amax == 0 (an all-zero block keeps S = 1);
+// with pow2 (UE8M0 scales) rounded up to a power of two, so that |x / S|
+// stays within 448 and x / S is exact.
+__device__ __forceinline__ float e4m3_scale(float amax, bool pow2) {
+  const float s = amax == 0.f ? 1.f : __fdiv_rn(amax, kE4M3Max);
+  return pow2 ? pow2_ceil(s) : s;
 }
 
 // Per-scale constants of the packed encoder.

@@ -17,7 +17,8 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // ------------------------------------------------------------- quantize.cu
 cudaError_t launch_quantize(const void* x, int64_t rows, int64_t cols, int64_t ld, int gran,
-                            int role, uint8_t* codes, float* scales, void* ws, cudaStream_t s);
+                            int role, uint8_t* codes, float* scales, void* ws, bool pow2,
+                            cudaStream_t s);
 uint32_t quantize_status_take();
 
 // ----------------------------------------------------------------- gemm.cu

@@ -72,8 +72,8 @@ __global__ void amax_kernel(const uint16_t* __restrict__ x, int64_t rows, int64_
 __global__ void quant_tensor_kernel(const uint16_t* __restrict__ x, int64_t rows, int64_t cols,
                                     int64_t ld, uint8_t* __restrict__ codes,
                                     float* __restrict__ scales,
-                                    const unsigned int* __restrict__ amax) {
-  const float s = e4m3_scale(__uint_as_float(*amax));
+                                    const unsigned int* __restrict__ amax, bool pow2) {
+  const float s = e4m3_scale(__uint_as_float(*amax), pow2);
   const E4M3Enc e = e4m3_encoder(s);
   if (blockIdx.x == 0 && threadIdx.x == 0) scales[0] = s;
   const int64_t vpr = cols / 8;
@@ -94,7 +94,7 @@ constexpr int kRowVec = 4;
 
 __global__ void __launch_bounds__(kRowThreads) quant_row_kernel(
     const uint16_t* __restrict__ x, int64_t rows, int64_t cols, int64_t ld,
-    uint8_t* __restrict__ codes, float* __restrict__ scales) {
+    uint8_t* __restrict__ codes, float* __restrict__ scales, bool pow2) {
   __shared__ uint32_t red[kRowThreads / 32];
   const int64_t r = blockIdx.x;
   const uint16_t* xr = x + r * ld;
@@ -123,7 +123,7 @@ __global__ void __launch_bounds__(kRowThreads) quant_row_kernel(
 #pragma unroll
   for (int w = 1; w < kRowThreads / 32; ++w) b = max(b, red[w]);
   if (threadIdx.x == 0 && b >= kInfBits) flag_bad();
-  const float s = e4m3_scale(__uint_as_float(b));
+  const float s = e4m3_scale(__uint_as_float(b), pow2);
   const E4M3Enc e = e4m3_encoder(s);
   if (threadIdx.x == 0) scales[r] = s;
   if (cached) {
@@ -161,7 +161,7 @@ struct Stream {
   static constexpr size_t kSmem = kStages * kTileBytes + 1024 + 2 * 8 * kStages;
 };
 
-template <int R>
+template <int R, bool POW2>
 __global__ void __launch_bounds__(288) quant_block_stream_kernel(
     const __grid_constant__ CUtensorMap tmx, int64_t rows, int64_t cols,
     uint8_t* __restrict__ codes, float* __restrict__ scales, uint64_t limit_ns) {
@@ -234,7 +234,7 @@ __global__ void __launch_bounds__(288) quant_block_stream_kernel(
       b = max(b, __shfl_xor_sync(0xffffffffu, b, 2));
       b = max(b, __shfl_xor_sync(0xffffffffu, b, 1));
       finite &= b < kInfBits;
-      const float s = e4m3_scale(__uint_as_float(b));
+      const float s = e4m3_scale(__uint_as_float(b), POW2);
       const E4M3Enc e = e4m3_encoder(s);
       const uint2 c0 = e4m3_encode8(v0, e), c1 = e4m3_encode8(v1, e);
       const int64_t r = rb * R + rr;
@@ -266,7 +266,7 @@ __global__ void __launch_bounds__(288) quant_block_stream_kernel(
 #pragma unroll
       for (int w = 1; w < 8; ++w) b = max(b, red[w]);
       finite &= b < kInfBits;
-      const float s = e4m3_scale(__uint_as_float(b));
+      const float s = e4m3_scale(__uint_as_float(b), POW2);
       const E4M3Enc e = e4m3_encoder(s);
       if (tid == 0) scales[rb * nkb + kb] = s;
 #pragma unroll
@@ -297,12 +297,12 @@ bool make_bf16_tmap(CUtensorMap* tm, const void* x, int64_t rows, int64_t cols, 
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int R>
+template <int R, bool POW2>
 cudaError_t launch_stream(const void* x, int64_t rows, int64_t cols, int64_t ld, uint8_t* codes,
                           float* scales, cudaStream_t s) {
   CUtensorMap tm;
   if (!make_bf16_tmap(&tm, x, rows, cols, ld, R)) return cudaErrorInvalidValue;
-  auto kern = quant_block_stream_kernel<R>;
+  auto kern = quant_block_stream_kernel<R, POW2>;
   static int configured_device = -1;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -330,7 +330,8 @@ int grid_for(int64_t work_items, int threads) {
 }  // namespace
 
 cudaError_t launch_quantize(const void* x, int64_t rows, int64_t cols, int64_t ld, int gran,
-                            int role, uint8_t* codes, float* scales, void* ws, cudaStream_t s) {
+                            int role, uint8_t* codes, float* scales, void* ws, bool pow2,
+                            cudaStream_t s) {
   const uint16_t* xb = static_cast<const uint16_t*>(x);
   if (rows == 0) return cudaSuccess;
   if (gran == FP8RL_GRAN_TENSOR) {
@@ -340,14 +341,16 @@ cudaError_t launch_quantize(const void* x, int64_t rows, int64_t cols, int64_t l
     const int64_t nvec = rows * (cols / 8);
     amax_kernel<<<grid_for(nvec, 256), 256, 0, s>>>(xb, rows, cols, ld, amax);
     quant_tensor_kernel<<<grid_for(nvec, 256), 256, 0, s>>>(xb, rows, cols, ld, codes, scales,
-                                                             amax);
+                                                             amax, pow2);
   } else if (gran == FP8RL_GRAN_ROWWISE) {
     quant_row_kernel<<<static_cast<unsigned>(rows), kRowThreads, 0, s>>>(xb, rows, cols, ld,
-                                                                          codes, scales);
+                                                                          codes, scales, pow2);
   } else if (role == FP8RL_ROLE_ACT) {
-    return launch_stream<32>(x, rows, cols, ld, codes, scales, s);
+    return pow2 ? launch_stream<32, true>(x, rows, cols, ld, codes, scales, s)
+                : launch_stream<32, false>(x, rows, cols, ld, codes, scales, s);
   } else {
-    return launch_stream<128>(x, rows, cols, ld, codes, scales, s);
+    return pow2 ? launch_stream<128, true>(x, rows, cols, ld, codes, scales, s)
+                : launch_stream<128, false>(x, rows, cols, ld, codes, scales, s);
   }
   return cudaGetLastError();
 }

@@ -139,3 +139,35 @@ def test_quantize_every_bf16_scale_near_midpoints(cuda_lib, gran, role):
     got = codes.cpu().numpy()
     bad = np.argwhere(got != ref_c)
     assert bad.size == 0, (bad[:5], got[tuple(bad[0])], ref_c[tuple(bad[0])])
+
+
+# ---- power-of-two (UE8M0) scales ----------------------------------------------
+
+@pytest.mark.parametrize("gran,role", CASES)
+@pytest.mark.parametrize("rows,cols,ld", [(7, 256, None), (129, 384, 512), (1000, 4096, None)])
+def test_quantize_ue8m0_bit_exact(cuda_lib, gran, role, rows, cols, ld):
+    x = _input(rows, cols, rows * 17 + cols, ld)
+    codes, scales = cuda_lib.quantize(x, gran, role, ue8m0=True)
+    cuda_lib.check()
+    ref_c, ref_s = OQ.quantize(x.float().cpu().numpy(), gran, role, pow2=True)
+    assert np.array_equal(codes.cpu().numpy(), ref_c)
+    assert np.array_equal(scales_natural(scales, rows, cols, gran, role), ref_s)
+
+
+@pytest.mark.parametrize("gran", [OQ.TENSOR, OQ.ROWWISE, OQ.BLOCK])
+def test_logprobs_on_ue8m0_codes(cuda_lib, gran):
+    """The scoring GEMM takes power-of-two scales like any other."""
+    from oracle import logprobs as OL
+    api = cuda_lib
+    T, H, V = 300, 256, 1000
+    h = synth.normal_bf16(T, H, 1.0, 61, "cuda")
+    W = synth.normal_bf16(V, H, 0.05, 62, "cuda")
+    y = torch.randint(0, V, (T,), generator=torch.Generator().manual_seed(63)).to(torch.int32).cuda()
+    hc, hs = api.quantize(h, gran, api.ROLE_ACT, ue8m0=True)
+    wc, ws = api.quantize(W, gran, api.ROLE_WEIGHT, ue8m0=True)
+    out = api.token_logprobs(hc, hs, wc, ws, gran, y)
+    api.check()
+    hq, hsr = OQ.quantize(h.float().cpu().numpy(), gran, OQ.ACT, pow2=True)
+    wq, wsr = OQ.quantize(W.float().cpu().numpy(), gran, OQ.WEIGHT, pow2=True)
+    ref, _ = OL.token_logprobs(hq, hsr, wq, wsr, gran, y.cpu().numpy())
+    assert np.max(np.abs(out["logp"].cpu().numpy() - ref)) <= 2e-3
