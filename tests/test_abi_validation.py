@@ -86,3 +86,14 @@ def test_seq_mean_surrogate_rejects_bad_arguments(api):
     assert f(P, P, NULL, NULL, NULL, 10, 100, 0.8, 1.2, NULL, NULL, NULL, P, P, ws, NULL) == api.EINVAL
     assert f(P, P, NULL, NULL, P, 10, -5, 0.8, 1.2, NULL, NULL, NULL, P, P, ws, NULL) == api.ESHAPE
     assert f(P, P, NULL, NULL, P, 10, 100, 0.8, 1.2, NULL, NULL, NULL, P, NULL, ws, NULL) == api.EWORKSPACE
+
+
+def test_quantize_ue8m0_rejects_bad_arguments(api):
+    f = api.lib.fp8rl_quantize_ue8m0
+    assert f(NULL, 4, 128, 128, 2, 0, P, P, NULL, 0, NULL) == api.EINVAL      # no input
+    assert f(P, 4, 128, 128, 9, 0, P, P, NULL, 0, NULL) == api.EINVAL         # unknown granularity
+    assert f(P, 4, 128, 128, 2, 5, P, P, NULL, 0, NULL) == api.EINVAL         # unknown role
+    assert f(P, 4, 192, 192, 2, 0, P, P, NULL, 0, NULL) == api.ESHAPE         # block needs cols % 128
+    assert f(P, 4, 128, 100, 1, 0, P, P, NULL, 0, NULL) == api.ESHAPE         # ld < cols
+    assert f(ODD, 4, 128, 128, 1, 0, P, P, NULL, 0, NULL) == api.EALIGN
+    assert f(P, 4, 128, 128, 0, 0, P, P, NULL, 0, NULL) == api.EWORKSPACE     # per-tensor needs the amax word
