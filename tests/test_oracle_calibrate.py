@@ -8,6 +8,10 @@
   different algorithm from the oracle's interval construction), for L and for
   H, the latter against rho computed in exact rational arithmetic from the
   unrounded Eq. 5 terms;
+* GRID mode (Algorithm 1 as printed) by brute force over the grid in exact
+  rational arithmetic, on ratios placed exactly on grid points so that the
+  strict "<" of Eq. 5 and the tie-breaks decide the answer, and planted slips
+  of those rules caught;
 * a hand-worked example and SmoothUpdate values with the paper's constants;
 * degenerate inputs and the overflow bound of the fixed-point sums.
 """
@@ -203,3 +207,171 @@ def test_fixed_point_sums_never_overflow(scale):
     assert res["shift"] == C.fixed_shift(max(np.abs(e).max(), np.abs(C.update_terms(coef, r_fp, adv)[(mask != 0) & (adv != 0)]).max()),
                                          int(np.sum((mask != 0) & (adv != 0))))
     assert math.ldexp(float(np.abs(e).max()), res["shift"]) * len(e) <= 2.0 ** 62
+
+
+# ---------------------------------------------------------------- GRID mode
+# Algorithm 1 as printed: candidates on the 0.02 grid of I_L and I_H.  The
+# brute force below restates the search from the paper directly: every grid
+# candidate is scored in exact rational arithmetic (lower: |#{r <= L} - k|;
+# upper: |rho_FP8(L*, H) - rho_BF16| with the strict "<" of Eq. 5), the
+# minimisers are kept, and the tie goes to the candidate nearest the reference
+# bound, then to the smaller one.  Ratios sit exactly on grid points (and one
+# float32 step either side), coefficients and advantages are short dyadic
+# numbers, so every Eq. 5 term is exact in the oracle's fixed point and a tie
+# in the rational objective is a tie there too.  A slip such as "<=" for "<"
+# in P(H), or a reversed tie-break, changes the answer on these inputs.
+
+def _grid_points(lo_pct, hi_pct):
+    """fl32(k / 100) for the grid's percent values (computed independently of
+    the oracle's fl32(lo + i * step))."""
+    return [F32(p / 100) for p in range(lo_pct, hi_pct + 1, 2)]
+
+
+def _on_grid_ratios(rng, n, pts):
+    out = []
+    for _ in range(n):
+        v = pts[int(rng.integers(0, len(pts)))]
+        how = int(rng.integers(0, 4))
+        if how == 1:
+            v = np.nextafter(v, F32(np.inf))
+        elif how == 2:
+            v = np.nextafter(v, F32(-np.inf))
+        out.append(v)
+    return F32(out)
+
+
+def _brute_grid(r_fp, r_bf, adv, coef, c_lo, c_hi, lo_pts, hi_pts):
+    neg = [i for i in range(len(adv)) if adv[i] < 0]
+    pos = [i for i in range(len(adv)) if adv[i] > 0]
+    k = sum(1 for i in neg if r_bf[i] <= c_lo)
+
+    def pick(cands, key, ref):
+        best = min(key(c) for c in cands)
+        ties = [c for c in cands if key(c) == best]
+        return min(ties, key=lambda c: (abs(Fraction(float(c)) - Fraction(float(ref))), float(c)))
+
+    L = pick(lo_pts, lambda c: abs(sum(1 for i in neg if r_fp[i] <= c) - k), c_lo)
+
+    def e(i, r):
+        return Fraction(float(coef[i])) * Fraction(float(r[i])) * Fraction(float(adv[i]))
+
+    n_bf = abs(sum((e(i, r_bf) for i in pos if r_bf[i] < c_hi), Fraction(0)))
+    d_bf = abs(sum((e(i, r_bf) for i in neg if r_bf[i] > c_lo), Fraction(0)))
+    d_fp = abs(sum((e(i, r_fp) for i in neg if r_fp[i] > L), Fraction(0)))
+    if not pos or d_bf == 0 or d_fp == 0:
+        return L, None
+    rho_bf = n_bf / d_bf
+
+    def obj(c):
+        p = sum((e(i, r_fp) for i in pos if r_fp[i] < c), Fraction(0))
+        return abs(p / d_fp - rho_bf)
+
+    return L, pick(hi_pts, obj, c_hi)
+
+
+def _grid_case(seed):
+    rng = np.random.default_rng(7000 + seed)
+    n = int(rng.integers(5, 16))
+    lo_pts, hi_pts = _grid_points(50, 90), _grid_points(120, 200)
+    adv = F32(rng.choice([-2.0, -1.0, -0.5, 0.5, 1.0, 1.5], n))
+    adv[0], adv[1] = -1.0, 1.0
+    coef = F32(rng.choice([0.25, 0.5, 1.0, 2.0], n))
+    r_fp = _on_grid_ratios(rng, n, lo_pts + hi_pts)
+    r_bf = _on_grid_ratios(rng, n, lo_pts + hi_pts)
+    eps_hi = [0.2, 0.28, 0.24][seed % 3]
+    return r_fp, r_bf, adv, coef, eps_hi, lo_pts, hi_pts
+
+
+@pytest.mark.parametrize("seed", range(60))
+def test_grid_bounds_brute_force_on_grid_ratios(seed):
+    r_fp, r_bf, adv, coef, eps_hi, lo_pts, hi_pts = _grid_case(seed)
+    res = C.calibrate_clip_bounds(r_fp, r_bf, adv, np.ones(len(adv), np.uint8), coef, 0.2, eps_hi,
+                                  {"mode": C.GRID})
+    c_lo, c_hi = C.reference_bounds(0.2, eps_hi)
+    L, H = _brute_grid(r_fp, r_bf, adv, coef, c_lo, c_hi, lo_pts, hi_pts)
+    assert res["lo_star"] == L
+    if H is None:
+        assert res["flags"] & (C.FLAG_NO_POS | C.FLAG_ZERO_D_BF16 | C.FLAG_ZERO_D_FP8)
+    else:
+        assert res["flags"] == 0
+        assert res["hi_star"] == H
+
+
+def test_grid_candidates_match_percent_values():
+    """The oracle's fl32(lo + i * step) grid is the float32 of k/100."""
+    assert C.grid(0.5, 0.9, 0.02) == _grid_points(50, 90)
+    assert C.grid(1.2, 2.0, 0.02) == _grid_points(120, 200)
+
+
+def test_grid_brute_force_catches_planted_slips(monkeypatch):
+    """Plant the slips the pin must catch into the oracle (on the CPU) and
+    require that the brute force disagrees on at least one case each."""
+    def le_instead_of_lt(r_pos, q_pos, d_bf, x, c_hi, cands):
+        r_pos = np.asarray(r_pos, np.float32)
+        q_pos = np.asarray(q_pos, np.int64)
+        best = None
+        for c in cands:
+            p = C._isum(q_pos[r_pos <= c])
+            key = (abs(p * d_bf - x), abs(float(c) - float(c_hi)), float(c))
+            if best is None or key < best[0]:
+                best = (key, c)
+        return np.float32(best[1])
+
+    def far_tie_break(r_pos, q_pos, d_bf, x, c_hi, cands):
+        r_pos = np.asarray(r_pos, np.float32)
+        q_pos = np.asarray(q_pos, np.int64)
+        best = None
+        for c in cands:
+            p = C._isum(q_pos[r_pos < c])
+            key = (abs(p * d_bf - x), -abs(float(c) - float(c_hi)), float(c))
+            if best is None or key < best[0]:
+                best = (key, c)
+        return np.float32(best[1])
+
+    for slip in (le_instead_of_lt, far_tie_break):
+        monkeypatch.setattr(C, "upper_bound_grid", slip)
+        caught = 0
+        for seed in range(60):
+            r_fp, r_bf, adv, coef, eps_hi, lo_pts, hi_pts = _grid_case(seed)
+            res = C.calibrate_clip_bounds(r_fp, r_bf, adv, np.ones(len(adv), np.uint8), coef, 0.2, eps_hi,
+                                          {"mode": C.GRID})
+            c_lo, c_hi = C.reference_bounds(0.2, eps_hi)
+            _, H = _brute_grid(r_fp, r_bf, adv, coef, c_lo, c_hi, lo_pts, hi_pts)
+            caught += H is not None and res["hi_star"] != H
+        assert caught > 0, slip.__name__
+        monkeypatch.undo()
+
+
+def test_grid_brute_force_catches_planted_lower_slips(monkeypatch):
+    """The same for the lower bound: "<" for the CDF's "<=", and the tie going
+    to the larger candidate instead of the one nearer c_low."""
+    def lt_instead_of_le(r_neg, k, c_lo, cands):
+        r_neg = np.asarray(r_neg, np.float32)
+        best = None
+        for c in cands:
+            key = (abs(int(np.sum(r_neg < c)) - k), abs(float(c) - float(c_lo)), float(c))
+            if best is None or key < best[0]:
+                best = (key, c)
+        return np.float32(best[1])
+
+    def larger_first(r_neg, k, c_lo, cands):
+        r_neg = np.asarray(r_neg, np.float32)
+        best = None
+        for c in cands:
+            key = (abs(int(np.sum(r_neg <= c)) - k), -float(c))
+            if best is None or key < best[0]:
+                best = (key, c)
+        return np.float32(best[1])
+
+    for slip in (lt_instead_of_le, larger_first):
+        monkeypatch.setattr(C, "lower_bound_grid", slip)
+        caught = 0
+        for seed in range(60):
+            r_fp, r_bf, adv, coef, eps_hi, lo_pts, hi_pts = _grid_case(seed)
+            res = C.calibrate_clip_bounds(r_fp, r_bf, adv, np.ones(len(adv), np.uint8), coef, 0.2, eps_hi,
+                                          {"mode": C.GRID})
+            c_lo, c_hi = C.reference_bounds(0.2, eps_hi)
+            L, _ = _brute_grid(r_fp, r_bf, adv, coef, c_lo, c_hi, lo_pts, hi_pts)
+            caught += res["lo_star"] != L
+        assert caught > 0, slip.__name__
+        monkeypatch.undo()
