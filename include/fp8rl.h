@@ -303,6 +303,12 @@ typedef struct fp8rl_clip_stats {
   float lo, hi;          /* bounds used        */
   int32_t flags;         /* 1 = no valid token */
   int32_t n_seq_valid;   /* sequence-mean call: sequences with a valid token (S); else 0 */
+  /* Clip fractions (§3; PPO's clip fraction split by advantage sign), each 0
+   * when its denominator is 0, float64 quotients of the exact counts:       */
+  double clip_frac_pos;  /* clipped_pos / n_pos                              */
+  double clip_frac_neg;  /* clipped_neg / n_neg                              */
+  double clip_frac;      /* (clipped_pos + clipped_neg) / n_valid; for
+                            sequence-level clipping / n_seq_valid (responses) */
 } fp8rl_clip_stats;
 
 #define FP8RL_CLIP_HI 1  /* clip-mask bit: A > 0 and r >= H */

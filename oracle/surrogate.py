@@ -198,4 +198,8 @@ def seq_level_clipped_surrogate(logp, logp_old, adv_seq, mask, seq_id, n_seq, lo
         "seq_ratio": s64, "seq_ratio32": s32, "seq_clip": cm, "seq_terms": terms,
         "seq_valid_tokens": n_i, "n_seq_valid": S, "n_valid": int(valid.sum()),
         "n_pos": n_pos, "n_neg": n_neg, "clipped_pos": c_pos, "clipped_neg": c_neg,
+        # clip fractions over responses (the unit this variant clips)
+        "clip_frac_pos": c_pos / n_pos if n_pos else 0.0,
+        "clip_frac_neg": c_neg / n_neg if n_neg else 0.0,
+        "clip_frac": (c_pos + c_neg) / S if S else 0.0,
     }

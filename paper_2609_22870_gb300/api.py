@@ -51,7 +51,9 @@ class ClipStats(ctypes.Structure):
                 ("n_valid", ctypes.c_int64), ("n_pos", ctypes.c_int64), ("n_neg", ctypes.c_int64),
                 ("clipped_pos", ctypes.c_int64), ("clipped_neg", ctypes.c_int64),
                 ("lo", ctypes.c_float), ("hi", ctypes.c_float),
-                ("flags", ctypes.c_int32), ("n_seq_valid", ctypes.c_int32)]
+                ("flags", ctypes.c_int32), ("n_seq_valid", ctypes.c_int32),
+                ("clip_frac_pos", ctypes.c_double), ("clip_frac_neg", ctypes.c_double),
+                ("clip_frac", ctypes.c_double)]
 
 
 class ClipDiag(ctypes.Structure):
@@ -484,11 +486,7 @@ def lm_head_backward(h_codes, h_scales, w_codes, w_scales, gran, targets, lse, g
 def read_clip_stats(buf):
     raw = bytes(buf.cpu().numpy().tobytes())
     s = ClipStats.from_buffer_copy(raw)
-    d = {f: getattr(s, f) for f, _ in ClipStats._fields_}
-    d["clip_frac_pos"] = d["clipped_pos"] / d["n_pos"] if d["n_pos"] else 0.0
-    d["clip_frac_neg"] = d["clipped_neg"] / d["n_neg"] if d["n_neg"] else 0.0
-    d["clip_frac"] = (d["clipped_pos"] + d["clipped_neg"]) / d["n_valid"] if d["n_valid"] else 0.0
-    return d
+    return {f: getattr(s, f) for f, _ in ClipStats._fields_}
 
 
 # ------------------------------------------------------------------ diagnostics

@@ -114,6 +114,16 @@ struct Bounds {
   float lo, hi, inv_n;
 };
 
+// Clip fractions of §3 (PPO's clip fraction, split by advantage sign): the
+// share of A > 0 units clipped at H, of A < 0 units clipped at L, and of all
+// valid units clipped; 0 where the denominator is 0.  Units are tokens for the
+// token-level calls and responses for sequence-level clipping.
+__device__ __forceinline__ void set_clip_fractions(fp8rl_clip_stats& s, unsigned long long n_all) {
+  s.clip_frac_pos = s.n_pos ? static_cast<double>(s.clipped_pos) / static_cast<double>(s.n_pos) : 0.0;
+  s.clip_frac_neg = s.n_neg ? static_cast<double>(s.clipped_neg) / static_cast<double>(s.n_neg) : 0.0;
+  s.clip_frac = n_all ? static_cast<double>(s.clipped_pos + s.clipped_neg) / static_cast<double>(n_all) : 0.0;
+}
+
 // One token: its term, its gradient and clip-mask byte; counts into `a`.
 __device__ __forceinline__ float token(float rt, float at, bool valid, float wt, const Bounds& b,
                                        Acc& a, float& g, uint32_t& cm) {
@@ -216,6 +226,7 @@ __global__ void __launch_bounds__(kThreads) surrogate_kernel(
     s.hi = b.hi;
     s.flags = n_valid ? 0 : 1;
     s.n_seq_valid = 0;
+    set_clip_fractions(s, n_valid);
     *stats = s;
   }
 }
@@ -330,6 +341,7 @@ __global__ void __launch_bounds__(kThreads) seq_surrogate_kernel(
     s.hi = b.hi;
     s.flags = n_valid ? 0 : 1;
     s.n_seq_valid = static_cast<int32_t>(S);
+    set_clip_fractions(s, n_valid);
     *stats = s;
   }
 }
@@ -596,6 +608,7 @@ __global__ void __launch_bounds__(kThreads) seq_lvl_seq_kernel(
     st.hi = hi;
     st.flags = n_valid ? 0 : 1;
     st.n_seq_valid = static_cast<int32_t>(S);
+    set_clip_fractions(st, S);  // over responses
     *stats = st;
   }
 }

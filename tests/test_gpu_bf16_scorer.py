@@ -8,7 +8,8 @@ float64 product of the same bf16 values (the workload statement's log-prob
 tolerance); the observed error is far smaller because the products are exact
 in fp32 and only the fp32 accumulation rounds.  Shapes span several 128 x 256
 tiles, hidden sizes that are multiples of 64 but not of 128, ragged T and V,
-strided rows, T = 1 and V = 1, and the 8B / 32B lm_head shapes on sampled rows.
+strided rows, T = 1 and V = 1, and the full workloads on 1024 random rows
+plus every tile and band boundary.
 """
 
 import numpy as np
@@ -17,11 +18,10 @@ import torch
 
 from oracle import logprobs as OL
 from paper_2609_22870_gb300 import synth
-from tests.gpu_helpers import sample_rows
+from tests.gpu_helpers import full_size_rows, oracle_bf16_logprobs_rows
 
 pytestmark = pytest.mark.gpu
 TOL = 2e-3
-STRIP = 8192
 
 
 def _data(T, H, V, seed, wstd=0.02):
@@ -37,11 +37,7 @@ def _data(T, H, V, seed, wstd=0.02):
 def _oracle(h, W, y, rows):
     """Oracle (logp, lse) for the selected rows, one vocabulary strip of
     logits at a time (each z[t][v] is its own dot product)."""
-    rows = np.asarray(rows, dtype=np.int64)
-    hx = h[torch.as_tensor(rows, device=h.device)].float().cpu().numpy()
-    z = np.concatenate([OL.bf16_logits(hx, W[v0:v0 + STRIP].float().cpu().numpy())
-                        for v0 in range(0, W.shape[0], STRIP)], axis=1)
-    return OL.log_softmax_gather(z, y.cpu().numpy()[rows])
+    return oracle_bf16_logprobs_rows(h, W, y, rows)
 
 
 @pytest.mark.parametrize("T,H,V", [(1, 64, 1), (5, 64, 37), (300, 192, 1000), (257, 512, 4096),
@@ -88,15 +84,17 @@ def test_bf16_large_logits_stay_finite(cuda_lib):
     assert np.max(np.abs(lp - ref_lp)) <= TOL * max(1.0, np.max(np.abs(ref_lp)) / 100)
 
 
-@pytest.mark.parametrize("name", ["grpo_8b", "dapo_32b"])
+@pytest.mark.parametrize("name", ["grpo_8b", "dapo_32b", "long_8b"])
 def test_bf16_full_size_sampled_rows(cuda_lib, name):
+    """1024 random rows, both sides of every 128-row tile boundary and of every
+    band boundary of the tile order, first and last rows."""
     w = synth.WORKLOADS[name]
     h, W, y = synth.hidden_states(w, "cuda"), synth.lm_head_weight(w, "cuda"), synth.targets(w, "cuda")
     out = cuda_lib.bf16_token_logprobs(h, W, y)
     cuda_lib.check()
     lp = out["logp"].cpu().numpy()
     assert np.all(np.isfinite(lp))
-    rows = sample_rows(w.T, 24, 9)
+    rows = full_size_rows(w.T, 9)
     ref_lp, _ = _oracle(h, W, y, rows)
     assert np.max(np.abs(lp[rows] - ref_lp)) <= TOL
 

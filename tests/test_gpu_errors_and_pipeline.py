@@ -10,6 +10,7 @@ import torch
 
 from oracle import calibrate as OC
 from oracle import quantize as OQ
+from oracle import surrogate as OS
 from paper_2609_22870_gb300 import synth
 from tests.gpu_helpers import oracle_logprobs_rows, sample_rows
 
@@ -150,7 +151,9 @@ def _pipeline_properties(res, st, b, adv, mask, r_bf16, w):
 @pytest.mark.parametrize("name", ["grpo_8b", "dapo_32b", "long_8b"])
 def test_pipeline_full_size(cuda_lib, name):
     """The whole path at the full configurations: logp on sampled rows against
-    the oracle, every other stage by the properties it must satisfy."""
+    the oracle (the scoring tests check 1024+ rows per workload), every stage
+    by the properties it must satisfy, and calibration and the loss bit for bit
+    against the oracle run on the pipeline's own ratios."""
     api = cuda_lib
     w = synth.WORKLOADS[name]
     h, W, y = synth.hidden_states(w, "cuda"), synth.lm_head_weight(w, "cuda"), synth.targets(w, "cuda")
@@ -168,6 +171,29 @@ def test_pipeline_full_size(cuda_lib, name):
     res = api.read_calib_result(b.cal_res)
     st = api.read_clip_stats(b.stats)
     _pipeline_properties(res, st, b, adv.numpy(), mask.numpy(), r_bf16.float().numpy(), w)
+    # Calibration and the loss on the pipeline's own FP8 ratios: the oracle,
+    # given the same ratios, must select the same bounds bit for bit (every
+    # count and fixed-point sum too), and its surrogate with those bounds must
+    # give the same clip mask, counts and fractions, the loss within 1e-4 and
+    # the gradient within 1e-6.
+    r = b.ratio.cpu().numpy()
+    a_np, m_np = adv.numpy(), mask.numpy()
+    ref = OC.calibrate_clip_bounds(r, r_bf16.float().numpy(), a_np, m_np, coef.float().numpy(),
+                                   w.eps_low, w.eps_high)
+    for k in ("lo_star", "hi_star", "lo_new", "hi_new", "c_lo", "c_hi"):
+        assert np.float32(res[k]) == ref[k], (k, res[k], ref[k])
+    for k in ("n_neg", "n_pos", "k_bf16", "k_fp8", "flags", "shift", "sum_pos_bf16", "sum_neg_bf16",
+              "sum_neg_fp8", "sum_pos_fp8"):
+        assert res[k] == ref[k], (k, res[k], ref[k])
+    sref = OS.clipped_surrogate(r, a_np, m_np, None, ref["lo_new"], ref["hi_new"])
+    assert np.array_equal(b.clip_mask.cpu().numpy(), sref["clip_mask"])
+    for k in ("n_valid", "n_pos", "n_neg", "clipped_pos", "clipped_neg", "clip_frac_pos", "clip_frac_neg",
+              "clip_frac"):
+        assert st[k] == sref[k], (k, st[k], sref[k])
+    scale = max(abs(sref["loss"]), np.sum(np.abs(sref["terms"])) / max(1, sref["n_valid"]))
+    assert abs(st["loss"] - sref["loss"]) <= 1e-4 * scale
+    g = b.grad.cpu().numpy().astype(np.float64)
+    assert np.all(np.abs(g - sref["grad"]) <= 1e-6 * np.abs(sref["grad"]) + 1e-30)
 
 
 def test_prefetched_steps_match_direct_steps(cuda_lib):

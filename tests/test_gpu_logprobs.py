@@ -3,7 +3,8 @@
 Log-probs within 2e-3 absolute of the oracle's float64 log-softmax of its own
 dequantised logits; ratios to the matching relative bound; dlogits within
 2e-3 |g_t| per element.  Shapes span several 128x256 tiles, ragged T and V,
-V = 1, T = 1, and the full configurations on sampled rows.
+V = 1, T = 1, and the full configurations on 1024 random rows plus every
+tile and band boundary.
 """
 
 import numpy as np
@@ -13,7 +14,7 @@ import torch
 from oracle import logprobs as OL
 from oracle import quantize as OQ
 from paper_2609_22870_gb300 import synth
-from tests.gpu_helpers import oracle_logprobs_rows, sample_rows
+from tests.gpu_helpers import full_size_rows, oracle_logprobs_rows
 
 pytestmark = pytest.mark.gpu
 TOL = 2e-3
@@ -85,15 +86,18 @@ def test_large_logits_stay_finite(cuda_lib):
                                        ("grpo_8b", OQ.ROWWISE), ("dapo_32b", OQ.BLOCK),
                                        ("long_8b", OQ.BLOCK)])
 def test_logprobs_full_size_sampled_rows(cuda_lib, name, gran):
-    """Full configurations, in the launch configuration the bench uses; sampled rows."""
+    """Full configurations, in the launch configuration the bench uses: 1024
+    random rows, both sides of every 128-row tile boundary and of every band
+    boundary of the GEMM's tile order (64 token tiles), first and last rows."""
     w = synth.WORKLOADS[name]
     h, W, y = synth.hidden_states(w, "cuda"), synth.lm_head_weight(w, "cuda"), synth.targets(w, "cuda")
     out, _ = _score(cuda_lib, h, W, y, gran)
     lp = out["logp"].cpu().numpy()
     assert np.all(np.isfinite(lp))
-    rows = sample_rows(w.T, 24, 5)
-    ref_lp, _, _ = oracle_logprobs_rows(h, W, gran, y, rows)
+    rows = full_size_rows(w.T, 5)
+    ref_lp, ref_lse, _ = oracle_logprobs_rows(h, W, gran, y, rows)
     assert np.max(np.abs(lp[rows] - ref_lp)) <= TOL
+    assert np.max(np.abs(out["lse"].cpu().numpy()[rows] - ref_lse)) <= TOL
 
 
 @pytest.mark.parametrize("gran", [OQ.TENSOR, OQ.BLOCK])

@@ -75,6 +75,13 @@ def _check(api, lp, lpo, A, mask, sid, lo=0.8, hi=1.2, bounds=None):
         assert st[k] == ref[k], k
     if same.all():
         assert st["clipped_pos"] == ref["clipped_pos"] and st["clipped_neg"] == ref["clipped_neg"]
+        for k in ("clip_frac_pos", "clip_frac_neg", "clip_frac"):
+            assert st[k] == ref[k], k
+    # the fractions the library reports are those of its own counts
+    assert st["clip_frac_pos"] == (st["clipped_pos"] / st["n_pos"] if st["n_pos"] else 0.0)
+    assert st["clip_frac_neg"] == (st["clipped_neg"] / st["n_neg"] if st["n_neg"] else 0.0)
+    S = st["n_seq_valid"]
+    assert st["clip_frac"] == ((st["clipped_pos"] + st["clipped_neg"]) / S if S else 0.0)
     scale = max(abs(ref["loss"]), np.sum(np.abs(ref["seq_terms"])) / max(1, ref["n_seq_valid"]), 1e-300)
     assert abs(st["loss"] - ref["loss"]) <= 1e-6 * scale
     assert st["flags"] == (0 if ref["n_valid"] else 1)

@@ -1,6 +1,6 @@
 """GPU parity: clipped surrogate, clip masks, counts and dloss/dlogp (a6/a7).
 
-Clip masks and counts bit-exact; loss within 1e-4 relative (also against the
+Clip masks, counts and clip fractions (computed by the library) bit-exact; loss within 1e-4 relative (also against the
 mean |term|, the loss being a cancelling sum); gradient within 1e-6 relative.
 """
 
@@ -36,7 +36,8 @@ def _check(api, r, adv, mask, w, lo, hi, bounds=None):
     ref = OS.clipped_surrogate(r.numpy(), adv.numpy(), None if mask is None else mask.numpy(),
                                None if w is None else w.numpy(), L, H)
     assert np.array_equal(out["clip_mask"].cpu().numpy(), ref["clip_mask"])
-    for k in ("n_valid", "n_pos", "n_neg", "clipped_pos", "clipped_neg"):
+    for k in ("n_valid", "n_pos", "n_neg", "clipped_pos", "clipped_neg", "clip_frac_pos", "clip_frac_neg",
+              "clip_frac"):
         assert st[k] == ref[k], k
     scale = max(abs(ref["loss"]), np.sum(np.abs(ref["terms"])) / max(1, ref["n_valid"]), 1e-300)
     assert abs(st["loss"] - ref["loss"]) <= 1e-4 * abs(ref["loss"]) + 1e-12 * scale
@@ -94,7 +95,8 @@ def _check_seq(api, r, adv, mask, w, sid, n_seq, lo, hi):
     ref = OS.clipped_surrogate_seq_mean(r.numpy(), adv.numpy(), None if mask is None else mask.numpy(),
                                         None if w is None else w.numpy(), lo, hi, sid.numpy(), n_seq)
     assert np.array_equal(out["clip_mask"].cpu().numpy(), ref["clip_mask"])
-    for k in ("n_valid", "n_pos", "n_neg", "clipped_pos", "clipped_neg", "n_seq_valid"):
+    for k in ("n_valid", "n_pos", "n_neg", "clipped_pos", "clipped_neg", "n_seq_valid", "clip_frac_pos",
+              "clip_frac_neg", "clip_frac"):
         assert st[k] == ref[k], k
     n = max(1, ref["n_valid"])
     scale = max(abs(ref["loss"]), np.sum(np.abs(ref["terms"])) / n, 1e-300)

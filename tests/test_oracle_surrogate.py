@@ -28,6 +28,9 @@ def test_hand_worked_table():
     assert np.array_equal(out["clip_mask"] != 0, clipped != 0)
     assert abs(out["loss"] - 0.3 / 7) < 1e-6
     assert out["n_valid"] == 7 and out["clipped_pos"] == 2 and out["clipped_neg"] == 2
+    # clip fractions by sign (§3): 2 of the 4 valid A>0 tokens, 2 of the 3 A<0
+    # tokens, 4 of the 7 valid tokens
+    assert out["clip_frac_pos"] == 2 / 4 and out["clip_frac_neg"] == 2 / 3 and out["clip_frac"] == 4 / 7
 
 
 def test_unclipped_ratio_one():
@@ -185,6 +188,8 @@ def test_seq_level_hand_case():
     assert abs(out["loss"] - (-H32 + 1.0 + 0.5 * L32) / 3) < 1e-15
     assert np.allclose(out["grad"], [0, 0, 1 / 9, 1 / 9, 1 / 9, 0], rtol=0, atol=1e-15)
     assert out["n_seq_valid"] == 3 and out["clipped_pos"] == 1 and out["clipped_neg"] == 1
+    # fractions over responses: 1 of 1 with A > 0, 1 of 2 with A < 0, 2 of 3
+    assert out["clip_frac_pos"] == 1.0 and out["clip_frac_neg"] == 0.5 and out["clip_frac"] == 2 / 3
 
 
 def test_seq_level_ratio_is_geometric_mean_of_token_ratios():
