@@ -164,23 +164,25 @@ fp8rl_status fp8rl_combine_logprobs(int64_t T, int64_t H, int64_t V, fp8rl_gran 
                                     void* workspace, size_t workspace_bytes, void* stream);
 
 /* fp8rl_token_logprobs without a caller workspace.  The paper has no
- * counterpart: this call exists for callers that cannot allocate device
- * memory at the point where they score tokens -- for example code running in
- * a host function enqueued on a stream (where CUDA API calls such as
- * cudaMalloc are not allowed), or serving loops that forbid the allocation
- * (and the implicit device synchronisation cudaMalloc / cudaFree may cause)
- * on the hot path -- and so cannot provide the workspace fp8rl_token_logprobs
- * needs.  Arguments and results are those of fp8rl_token_logprobs.
+ * counterpart: this call exists for callers that may not allocate device
+ * memory at the point where they score tokens -- serving loops and other hot
+ * paths that forbid allocation there (cudaMalloc / cudaFree can synchronise
+ * the whole device and stall every stream), or processes whose device memory
+ * is all reserved up front by another allocator -- and so cannot provide the
+ * workspace fp8rl_token_logprobs needs.  Arguments and results are those of
+ * fp8rl_token_logprobs (same kernels, same bits).
  *
  * The scratch is one array of FP8RL_NOALLOC_SCRATCH_BYTES compiled into the
  * library; every GPU that loads the library holds it until the process exits.
  * Shapes whose fp8rl_token_logprobs_workspace_size() exceeds it are refused
  * with FP8RL_EWORKSPACE (about T <= 1760 tokens at V = 151936; T <= 64000 at
- * V = 4096).  The call allocates nothing.  Its first call on a device looks up
- * the array's device address (cudaGetSymbolAddress); make that first call
- * before any stream capture.  All calls share the array and it keeps the last
- * call's contents: calls that can overlap on the GPU (other streams, other
- * host threads) race on it and must be ordered by the caller. */
+ * V = 4096).  The call allocates nothing.  Its first call on a device (and the
+ * first after the device's context was reset) looks up the array's device
+ * address with cudaGetSymbolAddress; make that first call before any stream
+ * capture.  All calls share the array and it keeps the last call's contents
+ * (no part of it needs to start at zero): calls that can overlap on the GPU
+ * (other streams, other host threads) race on it and must be ordered by the
+ * caller. */
 #define FP8RL_NOALLOC_SCRATCH_BYTES (16u << 20)
 
 fp8rl_status fp8rl_token_logprobs_noalloc(const uint8_t* h_codes, const float* h_scales,

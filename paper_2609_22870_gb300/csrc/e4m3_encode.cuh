@@ -58,11 +58,13 @@ __device__ __forceinline__ float amax_of(uint32_t m) {
   return __uint_as_float((hi > lo ? hi : lo) << 16);
 }
 
-// The smallest power of two not below t (t > 0 and finite; t < 2^119 here).
+// The smallest power of two not below t (t > 0; finite t < 2^119 here).
+// +inf and NaN (a block with a non-finite input) come back unchanged, so the
+// stored scale shows the bad block as in the paper-scale mode.
 __device__ __forceinline__ float pow2_ceil(float t) {
   const uint32_t b = __float_as_uint(t);
   const uint32_t ex = b >> 23, man = b & 0x7FFFFFu;
-  if (man == 0) return t;                              // a normal power of two
+  if (ex == 0xFFu || man == 0) return t;               // inf / NaN, or a power of two
   if (ex != 0) return __uint_as_float((ex + 1) << 23);  // next binade
   const int h = 31 - __clz(man);                       // subnormal: highest set bit
   return man == (1u << h) ? t : __uint_as_float(1u << (h + 1));

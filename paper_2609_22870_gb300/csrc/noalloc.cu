@@ -1,8 +1,13 @@
 // fp8rl_token_logprobs_noalloc: the scoring call of fp8rl_token_logprobs for
-// callers that cannot hand the library a workspace, because they are not
-// allowed to allocate device memory when they call it.  Its scratch (the
-// per-token logsumexp partials and the gathered target logits) lives in one
-// fixed array compiled into the library instead.
+// callers that may not allocate device memory when they score tokens (serving
+// loops and other hot paths that forbid allocation and the device-wide
+// synchronisation cudaMalloc / cudaFree can cause, or processes whose device
+// memory is all reserved up front), so they cannot hand the library a
+// workspace.  Its scratch (the per-token logsumexp partials and the gathered
+// target logits) lives in one fixed array compiled into the library instead.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include <mutex>
 
 #include "internal.h"
@@ -17,24 +22,60 @@ static __device__ __align__(256) unsigned char g_scratch[kScratchBytes];
 
 constexpr int kMaxDevices = 64;
 std::mutex g_mutex;
-void* g_scratch_ptr[kMaxDevices] = {};
+struct Cached {
+  unsigned long long ctx_id;  // 0 = nothing cached
+  void* ptr;
+};
+Cached g_cache[kMaxDevices] = {};
+
+// Unique id of the context current on this thread (0 if none or if the driver
+// lacks the query).  Ids are never reused within a process, so a context
+// created after cudaDeviceReset gets a new one.
+unsigned long long current_context_id() {
+  static PFN_cuCtxGetCurrent_v4000 get_current = nullptr;
+  static PFN_cuCtxGetId_v12000 get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 4000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(f);
+    f = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<PFN_cuCtxGetId_v12000>(f);
+  });
+  if (get_current == nullptr || get_id == nullptr) return 0;
+  CUcontext ctx = nullptr;
+  if (get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr) return 0;
+  unsigned long long id = 0;
+  return get_id(ctx, &id) == CUDA_SUCCESS ? id : 0;
+}
 
 // Device address of g_scratch on the current device.  In host code the name
 // g_scratch only stands in for the symbol, so the address comes from the
-// runtime, once per device, with that device current.
+// runtime (cudaGetSymbolAddress) with that device current.  It is looked up
+// once per device context and again whenever the context changes (after
+// cudaDeviceReset the module is loaded anew and the old address is stale).
 cudaError_t scratch_address(void** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
   std::lock_guard<std::mutex> lock(g_mutex);
-  if (g_scratch_ptr[dev] == nullptr) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_scratch);
-    if (e != cudaSuccess) return e;
-    g_scratch_ptr[dev] = p;
+  const unsigned long long id = current_context_id();
+  if (id != 0 && g_cache[dev].ctx_id == id) {
+    *out = g_cache[dev].ptr;
+    return cudaSuccess;
   }
-  *out = g_scratch_ptr[dev];
+  void* p = nullptr;
+  e = cudaGetSymbolAddress(&p, g_scratch);
+  if (e != cudaSuccess) return e;
+  // the lookup above made the device's primary context current if it was not
+  g_cache[dev].ctx_id = id != 0 ? id : current_context_id();
+  g_cache[dev].ptr = p;
+  *out = p;
   return cudaSuccess;
 }
 

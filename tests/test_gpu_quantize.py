@@ -171,3 +171,41 @@ def test_logprobs_on_ue8m0_codes(cuda_lib, gran):
     wq, wsr = OQ.quantize(W.float().cpu().numpy(), gran, OQ.WEIGHT, pow2=True)
     ref, _ = OL.token_logprobs(hq, hsr, wq, wsr, gran, y.cpu().numpy())
     assert np.max(np.abs(out["logp"].cpu().numpy() - ref)) <= 2e-3
+
+
+@pytest.mark.parametrize("ue8m0", [False, True])
+@pytest.mark.parametrize("gran,role", [(2, 0), (2, 1), (1, 0)])
+def test_non_finite_block_shows_in_its_scale(cuda_lib, ue8m0, gran, role):
+    """A NaN or inf input flags the call and leaves a non-finite scale for its
+    own block (NaN stays NaN, inf stays inf, in both scale modes); every other
+    block's scale is the oracle's."""
+    api = cuda_lib
+    rows, cols = 256, 384
+    x = synth.normal_bf16(rows, cols, 1.0, 77, "cuda")
+    x[3, 5] = float("nan")
+    x[200, 300] = float("inf")
+    codes, scales = api.quantize(x, gran, role, ue8m0=ue8m0)
+    assert api.check_status() == api.EDEVICE
+    got = scales_natural(scales, rows, cols, gran, role)
+    if gran == 1:
+        bad = {(3,): "nan", (200,): "inf"}
+        idx = lambda r, c: (r,)  # noqa: E731
+    elif role == 0:
+        bad = {(3, 0): "nan", (200, 2): "inf"}
+        idx = lambda r, c: (r, c // 128)  # noqa: E731
+    else:
+        bad = {(0, 0): "nan", (1, 2): "inf"}
+        idx = lambda r, c: (r // 128, c // 128)  # noqa: E731
+    for k, kind in bad.items():
+        v = got[k]
+        assert (np.isnan(v) if kind == "nan" else np.isposinf(v)), (k, v)
+    clean = x.float().cpu().numpy()
+    clean[3, 5] = 0.0
+    clean[200, 300] = 0.0
+    _, ref = OQ.quantize(clean, gran, role, pow2=ue8m0)
+    keep = np.ones(ref.shape, bool)
+    for k in bad:
+        keep[k] = False
+    # blocks without a bad element match (the zeroed ones may differ only if
+    # the bad element was their maximum, which the mask above excludes)
+    assert np.array_equal(got[keep], ref[keep])
