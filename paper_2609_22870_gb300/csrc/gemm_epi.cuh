@@ -1,0 +1,179 @@
+// Parameters, tile order and epilogues shared by the two lm_head GEMM
+// kernels: the one-CTA kernel (gemm.cu: every scaling mode, 128 x 256 tiles)
+// and the CTA-pair kernel for block scaling (gemm_pair.cu: 256 x 128 tiles on
+// two SMs).  Included by those two translation units only.
+#pragma once
+
+#include <cmath>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace fp8rl {
+namespace {
+
+constexpr int CHUNK = 128;        // vocabulary columns per LSE partial
+constexpr float kLog2e = 1.4426950408889634f;
+
+enum { kTensor = FP8RL_GRAN_TENSOR, kRow = FP8RL_GRAN_ROWWISE, kBlock = FP8RL_GRAN_BLOCK, kBf16 = 3 };
+static_assert(kBf16 == kGemmBf16, "BF16 mode id shared with the host interface");
+// Epilogues: streaming LSE partials + target logit; dense dlogits rows (fp32);
+// dlogits of every token in bf16, both [M][N] and transposed [N][M] (the
+// operands of the two backward contractions); plain store of the fp32
+// accumulators (optionally added to what is there).
+enum { kEpiLse = 0, kEpiDlogits = 1, kEpiDense = 2, kEpiStore = 3 };
+
+struct Params {
+  const float* a_scales;
+  const float* b_scales;
+  const int32_t* targets;
+  float2* partials;
+  float* zy;
+  const float* lse;
+  const float* grad;
+  float* out;
+  uint16_t* p_out;   // kEpiDense: bf16 [M][ld_p]
+  uint16_t* pt_out;  // kEpiDense: bf16 [N][ld_pt]
+  int64_t ld_p, ld_pt;
+  float* c_out;      // kEpiStore: fp32 [M][ld_c]
+  int64_t ld_c;
+  int accumulate;
+  int M, N, K;
+  int num_m, num_n, num_kb;
+  int band_m;  // row blocks per band of the tile order
+  int n_chunks;
+  uint64_t wait_limit_ns;
+};
+
+// Tile order: bands of band_m row blocks, and within a band the row block
+// varies fastest.  For the scoring GEMM (band of 64 token blocks) the 152
+// tiles in flight then share one or two vocabulary tiles and a band of h codes
+// small enough to stay in L2, so the lm_head codes are read once per band and
+// h codes about once.  The backward contractions have only 16 column tiles
+// (N = H) and long rows: a band of 16 row blocks keeps about half of them in
+// flight per row block, which roughly halves the re-reads of the A operand
+// against 64 at the cost of more passes over the B operand.
+constexpr int kBandM = 64;
+constexpr int kBandStore = 16;
+__device__ __forceinline__ void tile_coords(int tile, const Params& p, int& m_blk, int& n_blk) {
+  const int band = tile / (p.band_m * p.num_n);
+  const int m_base = band * p.band_m;
+  const int band_m = min(p.band_m, p.num_m - m_base);
+  const int local = tile - band * p.band_m * p.num_n;
+  m_blk = m_base + local % band_m;
+  n_blk = local / band_m;
+}
+
+// Running epilogue state of one thread: row `row`, vocabulary columns
+// [col0, col0 + 128) consumed 32 at a time (values already scaled).
+struct EpiState {
+  float m, s, zy;
+  int j;  // target column relative to col0 (outside [0, 128): not here)
+};
+
+template <int EPI>
+__device__ __forceinline__ void epi_begin(const Params& p, EpiState& e, int row, int col0) {
+  e.m = -INFINITY;
+  e.s = 0.f;
+  e.zy = 0.f;
+  e.j = -1;
+  if (EPI != kEpiStore && row < p.M) {
+    const int y = p.targets[row];
+    if (y >= 0 && y < p.N) e.j = y - col0;
+  }
+}
+
+// Columns [col0 + base, col0 + base + 32).
+template <int EPI>
+__device__ __forceinline__ void epi_consume32(const Params& p, EpiState& e, const float* z, int row,
+                                              int col0, int base) {
+  const int ncol = p.N - (col0 + base);  // valid columns in this piece (may be <= 0 or >= 32)
+  if (ncol <= 0 || row >= p.M) return;
+  if (EPI == kEpiLse) {
+    float cm = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      if (i < ncol) cm = fmaxf(cm, z[i]);
+    const float mn = fmaxf(e.m, cm);
+    const float mb = mn * kLog2e;
+    float acc = 0.f;
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      if (i < ncol) acc += exp2f(fmaf(z[i], kLog2e, -mb));
+    e.s = e.s * exp2f((e.m - mn) * kLog2e) + acc;
+    e.m = mn;
+    const int jj = e.j - base;
+    if (jj >= 0 && jj < 32) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        if (i == jj) e.zy = z[i];
+    }
+  } else if (EPI == kEpiDlogits) {
+    const float l = p.lse[row], g = p.grad[row];
+    float* o = p.out + static_cast<size_t>(row) * p.N + col0 + base;
+    const int jj = e.j - base;
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      if (i < ncol) o[i] = g * ((i == jj ? 1.f : 0.f) - expf(z[i] - l));
+  } else if (EPI == kEpiDense) {
+    const float l = p.lse[row], g = p.grad[row];
+    const int jj = e.j - base;
+    const int c = col0 + base;
+    uint32_t w[16];  // bf16 pairs, column order
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const float v0 = g * ((2 * i == jj ? 1.f : 0.f) - expf(z[2 * i] - l));
+      const float v1 = g * ((2 * i + 1 == jj ? 1.f : 0.f) - expf(z[2 * i + 1] - l));
+      w[i] = pack_bf16x2(v0, v1);
+    }
+    uint16_t* pr = p.p_out + static_cast<size_t>(row) * p.ld_p + c;  // 64-byte aligned
+    uint16_t* pt = p.pt_out + static_cast<size_t>(c) * p.ld_pt + row;
+    if (ncol >= 32) {
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        reinterpret_cast<uint4*>(pr)[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+#pragma unroll
+      for (int i = 0; i < 32; ++i)  // lanes are consecutive rows: 64 contiguous bytes per column
+        pt[static_cast<size_t>(i) * p.ld_pt] = static_cast<uint16_t>(w[i >> 1] >> (16 * (i & 1)));
+    } else {
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        if (i < ncol) {
+          const uint16_t b = static_cast<uint16_t>(w[i >> 1] >> (16 * (i & 1)));
+          pr[i] = b;
+          pt[static_cast<size_t>(i) * p.ld_pt] = b;
+        }
+    }
+  } else {  // kEpiStore
+    float* cr = p.c_out + static_cast<size_t>(row) * p.ld_c + col0 + base;  // 16-byte aligned
+    if (ncol >= 32) {
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        float4 v = make_float4(z[4 * q], z[4 * q + 1], z[4 * q + 2], z[4 * q + 3]);
+        if (p.accumulate) {
+          const float4 o = reinterpret_cast<const float4*>(cr)[q];
+          v.x += o.x;
+          v.y += o.y;
+          v.z += o.z;
+          v.w += o.w;
+        }
+        reinterpret_cast<float4*>(cr)[q] = v;
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        if (i < ncol) cr[i] = p.accumulate ? cr[i] + z[i] : z[i];
+    }
+  }
+}
+
+template <int EPI>
+__device__ __forceinline__ void epi_finish(const Params& p, const EpiState& e, int row, int chunk) {
+  if (EPI != kEpiLse || row >= p.M || chunk >= p.n_chunks) return;
+  p.partials[static_cast<size_t>(chunk) * p.M + row] = make_float2(e.m, e.s);
+  if (e.j >= 0 && e.j < CHUNK) p.zy[row] = e.zy;
+}
+
+
+}  // namespace
+}  // namespace fp8rl
