@@ -16,7 +16,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libfp8rl.so")
-SOURCES = ["api.cu", "quantize.cu", "gemm.cu", "gemm_pair.cu", "combine.cu", "calib.cu", "loss.cu", "diag.cu",
+SOURCES = ["api.cu", "quantize.cu", "gemm.cu", "combine.cu", "calib.cu", "loss.cu", "diag.cu",
            "backward.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-fvisibility=hidden",

@@ -85,7 +85,7 @@ extern "C" {
 
 fp8rl_status fp8rl_check(void* stream) {
   cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
-  uint32_t bits = quantize_status_take() | gemm_status_take() | gemm_pair_status_take() |
+  uint32_t bits = quantize_status_take() | gemm_status_take() |
                   combine_status_take() | calib_status_take() | loss_status_take();
   if (bits & kErrTimeout) return FP8RL_ETIMEOUT;
   if (bits & kErrDevice) return FP8RL_EDEVICE;

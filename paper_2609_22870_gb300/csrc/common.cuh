@@ -337,105 +337,6 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(uint32_t M, uint32_t N) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((N >> 3) << 17) | ((M >> 4) << 24);
 }
 
-// ---------------------------------------------------------------- clusters
-// Rank of this CTA in its cluster.
-__device__ __forceinline__ uint32_t cluster_ctarank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
-
-// Address in the shared::cluster window of the variable at shared::cta
-// address `saddr` in the CTA of cluster rank `rank`.
-__device__ __forceinline__ uint32_t mapa_shared(uint32_t saddr, uint32_t rank) {
-  uint32_t d;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(d) : "r"(saddr), "r"(rank));
-  return d;
-}
-
-// Arrive on an mbarrier of any CTA of the cluster (release at cluster scope).
-__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
-               : "memory");
-}
-
-// try_wait with acquire at cluster scope, for barriers that other CTAs of the
-// cluster arrive on; the hardware may suspend the thread for up to hint_ns.
-__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity, uint32_t hint_ns) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity), "r"(hint_ns)
-      : "memory");
-  return ok != 0;
-}
-
-// The bounded wait of mbar_wait with cluster-scope acquire.
-__device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity, uint64_t limit_ns,
-                                                  const volatile int* abort) {
-  if (mbar_try_wait_cluster(bar, parity, 0)) return true;
-  const uint64_t t0 = globaltimer_ns();
-  const uint32_t hint = limit_ns < 200000u ? static_cast<uint32_t>(limit_ns) : 200000u;
-  while (true) {
-    if (mbar_try_wait_cluster(bar, parity, hint)) return true;
-    if (abort != nullptr && *abort) return false;
-    if (globaltimer_ns() - t0 > limit_ns) return false;
-  }
-}
-
-// Every thread of every CTA of the cluster arrives, then waits for all of
-// them; memory operations before it are visible to the cluster after it.
-__device__ __forceinline__ void cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-
-// TMEM allocation shared by a CTA pair: one warp of EACH CTA of the pair
-// executes it, and both receive the same TMEM address.
-__device__ __forceinline__ void tmem_alloc_pair(uint32_t dst_smem, uint32_t ncols) {
-  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem),
-               "r"(ncols)
-               : "memory");
-}
-
-__device__ __forceinline__ void tmem_relinquish_pair() {
-  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
-}
-
-__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
-  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
-               : "memory");
-}
-
-// D (+)= A * B^T on a CTA pair: M = 256 rows of A, 128 in each CTA's shared
-// memory at the same offset; the N columns of B split in halves, the first in
-// the even CTA; each CTA's TMEM receives its own 128 rows of D.  Issued by one
-// elected lane of the even CTA (warp-converged call).
-__device__ __forceinline__ void mma_f8f6f4_pair_elect(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
-                                                      uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p, e;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "elect.sync _|e, 0xffffffff;\n\t"
-      "@e tcgen05.mma.cta_group::2.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-
-// Arrive once on the mbarrier at shared::cta offset `bar` in every CTA of
-// `cta_mask` when the pair MMAs issued so far have completed (one elected
-// lane of a converged warp issues it).
-__device__ __forceinline__ void mma_commit_pair_elect(uint32_t bar, uint16_t cta_mask) {
-  asm volatile(
-      "{\n\t.reg .pred e;\n\t"
-      "elect.sync _|e, 0xffffffff;\n\t"
-      "@e tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;\n\t}" ::"r"(bar),
-      "h"(cta_mask)
-      : "memory");
-}
-
 // ---------------------------------------------------------------- misc
 __device__ __forceinline__ float warp_max(float v) {
 #pragma unroll

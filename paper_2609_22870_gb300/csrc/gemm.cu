@@ -499,8 +499,6 @@ cudaError_t launch_mode(const CUtensorMap& ta, const CUtensorMap& tb, const Para
 template <int EPI>
 cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s) {
   if (a.M == 0 || a.N == 0) return cudaSuccess;
-  // block scaling runs on CTA pairs (four TMEM buffers per SM for the promotion)
-  if (a.gran == kBlock && EPI != kEpiStore) return launch_gemm_pair(a, EPI, s);
   const bool bf16 = a.gran == kBf16;
   CUtensorMap ta, tb;
   if (!make_tmap(&ta, a.a_codes, a.M, a.K, a.lda ? a.lda : a.K, BM, bf16) ||
@@ -540,6 +538,7 @@ cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s) {
     switch (a.gran) {
       case kTensor: return launch_mode<kTensor, EPI>(ta, tb, p, grid, s);
       case kRow: return launch_mode<kRow, EPI>(ta, tb, p, grid, s);
+      case kBlock: return launch_mode<kBlock, EPI>(ta, tb, p, grid, s);
       default: return cudaErrorInvalidValue;
     }
   } else {
@@ -547,7 +546,7 @@ cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s) {
       case kTensor: return launch_mode<kTensor, EPI>(ta, tb, p, grid, s);
       case kRow: return launch_mode<kRow, EPI>(ta, tb, p, grid, s);
       case kBf16: return launch_mode<kBf16, EPI>(ta, tb, p, grid, s);
-      default: return cudaErrorInvalidValue;
+      default: return launch_mode<kBlock, EPI>(ta, tb, p, grid, s);
     }
   }
 }

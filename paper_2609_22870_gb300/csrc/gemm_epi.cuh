@@ -1,7 +1,5 @@
-// Parameters, tile order and epilogues shared by the two lm_head GEMM
-// kernels: the one-CTA kernel (gemm.cu: every scaling mode, 128 x 256 tiles)
-// and the CTA-pair kernel for block scaling (gemm_pair.cu: 256 x 128 tiles on
-// two SMs).  Included by those two translation units only.
+// Parameters, tile order and epilogues of the lm_head GEMM kernels
+// (gemm.cu).
 #pragma once
 
 #include <cmath>

@@ -56,10 +56,6 @@ cudaError_t launch_gemm_lse(const GemmArgs& a, cudaStream_t s);
 cudaError_t launch_gemm_dlogits(const GemmArgs& a, cudaStream_t s);
 cudaError_t launch_gemm_dense_dlogits(const GemmArgs& a, cudaStream_t s);
 cudaError_t launch_gemm_store(const GemmArgs& a, cudaStream_t s);
-// Block scaling on CTA pairs (gemm_pair.cu); `epi` is the epilogue id of
-// gemm_epi.cuh (LSE partials, dlogits rows, dense bf16 dlogits).
-cudaError_t launch_gemm_pair(const GemmArgs& a, int epi, cudaStream_t s);
-uint32_t gemm_pair_status_take();
 struct BwdLayout {
   int64_t vp, tp;             // padded row lengths of P [T][vp] and P^T, h^T [.][tp]
   size_t p, pt, wt, ht, total;  // byte offsets in the workspace
