@@ -98,6 +98,21 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint64_
   }
 }
 
+// mbar_wait for a phase that has usually completed already: a non-blocking
+// test first (try_wait costs ~100 clocks even when the phase is complete).
+__device__ __forceinline__ bool mbar_wait_likely_done(uint32_t bar, uint32_t parity, uint64_t limit_ns,
+                                                      const volatile int* abort) {
+  uint32_t done_now;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(done_now)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return done_now != 0 || mbar_wait(bar, parity, limit_ns, abort);
+}
+
 // 4-byte asynchronous copy global -> shared (no register round trip).
 __device__ __forceinline__ void cp_async_4(uint32_t dst, const void* src) {
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(dst), "l"(src) : "memory");

@@ -301,11 +301,11 @@ __global__ void __launch_bounds__(THREADS, 1)
               sphase ^= 1;
             }
           }
-          ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&acc_full[ab]), aphase, lim, abort_flag));
+          // the epilogue trails the MMA, so this phase has usually completed
+          ok = __all_sync(0xffffffffu, mbar_wait_likely_done(smem_u32(&acc_full[ab]), aphase, lim, abort_flag));
           if (!ok) break;
           tc_fence_after();
           const uint32_t taddr = tmem_base + t_row + static_cast<uint32_t>(ab * BN + half * CHUNK);
-          const float2 sc2 = make_float2(sc, sc);
           // four 32-column chunks, double-buffered: the load of chunk c + 1
           // is in flight while chunk c is promoted; the TMEM buffer goes back
           // to the MMA as soon as the last chunk has landed in registers
