@@ -36,6 +36,19 @@ dLoss/dlogits above and the FP8 logits z of the forward pass,
 Reading: the quantisers pass the gradient straight through (their derivative
 is taken as the identity), so the contractions use the bf16 operands h and W
 the codes were quantised from.
+
+FP8 backward (the paper trains with FP8 GEMMs in the backward pass too, §3
+and the performance appendix; it prints no quantisation for them): the same
+two contractions with every operand E4M3-quantised by Eq. 3 before it is
+multiplied.  Readings: each contraction runs along its own K axis (V for dh,
+T for dW), so each operand is quantised along that axis; the gradient P gets
+the activation granularity of the forward pass, 1x128 blocks along K, where
+each thread of a tile holds one token's 128 vocabulary entries (P for dh);
+its transpose (the A operand of dW, K = T) gets 128 x 128 blocks, as do the
+transposed bf16 weight W^T and hidden states h^T (the B operands; the weight
+granularity of the forward pass).  P is taken in float32 (the value the
+hardware holds) before it is quantised; V and T are padded with zeros to
+multiples of 128 along K.
 """
 
 import numpy as np
@@ -125,3 +138,41 @@ def lm_head_backward(h_codes, h_scales, w_codes, w_scales, gran, targets, g, h, 
     if rows is None:
         out["dW"] = P.T @ np.asarray(h, np.float32).astype(np.float64)
     return out
+
+
+def _pad_cols(x, mult=128):
+    """x (rows, cols) float32, zero-padded to a multiple of `mult` columns."""
+    rows, cols = x.shape
+    cp = -(-cols // mult) * mult
+    out = np.zeros((rows, cp), np.float32)
+    out[:, :cols] = x
+    return out
+
+
+def lm_head_backward_fp8(h_codes, h_scales, w_codes, w_scales, gran, targets, g, h, W):
+    """dLoss/dh and dLoss/dW with both contractions on E4M3 operands.
+
+    P (float64 from the FP8 logits) is rounded to float32 and quantised twice:
+    P [T][V] with 1x128 blocks along V (A operand of dh = P W), P^T [V][T]
+    with 128 x 128 blocks (A operand of dW = P^T h); W^T [H][V] and h^T [H][T]
+    are quantised from the bf16 values with 128 x 128 blocks (B operands).
+    The products of the dequantised operands are summed in float64.  Returns
+    the quantised operands too (codes and scales in natural shape)."""
+    y = np.asarray(targets, np.int64)
+    gg = np.asarray(g, np.float64)
+    z = logits(h_codes, h_scales, w_codes, w_scales, gran)
+    _, lse = log_softmax_gather(z, y)
+    P32 = dlogits(z, y, lse, gg).astype(np.float32)
+    T, V = P32.shape
+    pq, ps = Q.quantize(_pad_cols(P32), Q.BLOCK, Q.ACT)              # (T, V') codes, (T, V'/128)
+    ptq, pts = Q.quantize(_pad_cols(P32.T), Q.BLOCK, Q.WEIGHT)       # (V, T'),  (ceil(V/128), T'/128)
+    wtq, wts = Q.quantize(_pad_cols(np.asarray(W, np.float32).T), Q.BLOCK, Q.WEIGHT)   # (H, V')
+    htq, hts = Q.quantize(_pad_cols(np.asarray(h, np.float32).T), Q.BLOCK, Q.WEIGHT)   # (H, T')
+    P_hat = Q.dequantize(pq, ps, Q.BLOCK, Q.ACT)
+    Pt_hat = Q.dequantize(ptq, pts, Q.BLOCK, Q.WEIGHT)
+    Wt_hat = Q.dequantize(wtq, wts, Q.BLOCK, Q.WEIGHT)
+    ht_hat = Q.dequantize(htq, hts, Q.BLOCK, Q.WEIGHT)
+    return {"P": P32, "lse": lse, "dh": P_hat @ Wt_hat.T, "dW": Pt_hat @ ht_hat.T,
+            "P_hat": P_hat[:, :V], "Pt_hat": Pt_hat[:, :T], "Wt_hat": Wt_hat[:, :V], "ht_hat": ht_hat[:, :T],
+            "p_codes": pq, "p_scales": ps, "pt_codes": ptq, "pt_scales": pts,
+            "wt_codes": wtq, "wt_scales": wts, "ht_codes": htq, "ht_scales": hts}

@@ -270,3 +270,88 @@ def test_lm_head_backward_invariants(gran):
     part = L.lm_head_backward(hq, hs, wq, ws, gran, y, g, h, W, rows=[4, 1])
     assert np.allclose(part["dh"], out["dh"][[4, 1]], rtol=0, atol=1e-13 * np.abs(out["dh"]).max())
     assert "dW" not in part
+
+
+# ---- FP8 backward (both contractions on E4M3 operands) -----------------------
+
+def test_fp8_backward_equals_exact_backward_when_quantisation_is_exact():
+    # 128 identical tokens, V = 2: every row of P is (a, -a) or (-a, a), so each
+    # 1x128 block of P and each 128 x 128 block of P^T holds one magnitude and
+    # encodes to +-448 exactly; W and h sit on the E4M3 grid with amax 448 2^-9,
+    # so their 128 x 128 quantisation is exact too.  The FP8 backward must then
+    # equal the exact one up to the float32 rounding of P and of its scales.
+    rng = np.random.default_rng(71)
+    T, H, V = 128, 128, 2
+    h_row = _exact_operands(rng, (1, H), 448.0 / 512)
+    h = np.repeat(h_row, T, axis=0)
+    W = _exact_operands(rng, (V, H), -448.0 / 512)
+    hq, hs = Q.quantize(h.astype(np.float32), Q.BLOCK, Q.ACT)
+    wq, ws = Q.quantize(W.astype(np.float32), Q.BLOCK, Q.WEIGHT)
+    y = np.zeros(T, np.int64)
+    g = np.full(T, 0.37)
+    ref = L.lm_head_backward(hq, hs, wq, ws, Q.BLOCK, y, g, h, W)
+    out = L.lm_head_backward_fp8(hq, hs, wq, ws, Q.BLOCK, y, g, h, W)
+    assert np.array_equal(out["Wt_hat"], W.T) and np.array_equal(out["ht_hat"], h.T)
+    assert np.all(np.abs(out["p_codes"][:, :V]) != 0)
+    for k in ("dh", "dW"):
+        bound = 2.0 ** -22 * (np.abs(ref["P"]) @ np.abs(W) if k == "dh" else np.abs(ref["P"]).T @ np.abs(h))
+        assert np.all(np.abs(out[k] - ref[k]) <= bound + 1e-300), k
+    assert np.max(np.abs(ref["dh"])) > 0 and np.max(np.abs(ref["dW"])) > 0
+
+
+def _e4m3_abs_err_bound(x, scale_of):
+    # |Q(x) - x| <= max(2^-4 |x|, 2^-10 S): half a step of the 3-bit mantissa
+    # in the normal range, half the subnormal step 2^-9 S below it
+    return np.maximum(2.0 ** -4 * np.abs(x), 2.0 ** -10 * scale_of)
+
+
+@pytest.mark.parametrize("gran", [Q.TENSOR, Q.ROWWISE, Q.BLOCK])
+def test_fp8_backward_within_quantisation_error_of_exact_backward(gran):
+    # dh = sum_v P W and dW = sum_t P^T h with every operand quantised: the
+    # difference to the exact contraction is bounded term by term by the E4M3
+    # rounding of both factors.  A dropped or misplaced scale, a transposed
+    # operand or a wrong block index breaks the bound by orders of magnitude.
+    rng = np.random.default_rng(72 + gran)
+    T, H, V = 130, 256, 300
+    h = rng.normal(0, 1, (T, H)).astype(np.float32)
+    W = (rng.normal(0, 0.05, (V, H))).astype(np.float32)
+    hq, hs = Q.quantize(h, gran, Q.ACT)
+    wq, ws = Q.quantize(W, gran, Q.WEIGHT)
+    y = rng.integers(0, V, T)
+    g = rng.normal(0, 1, T) / T
+    ref = L.lm_head_backward(hq, hs, wq, ws, gran, y, g, h, W)
+    out = L.lm_head_backward_fp8(hq, hs, wq, ws, gran, y, g, h, W)
+    P = out["P"].astype(np.float64)
+    # per-element scales of each quantised operand
+    sp = np.repeat(out["p_scales"], 128, axis=1)[:, :V]
+    spt = np.repeat(np.repeat(out["pt_scales"], 128, axis=0), 128, axis=1)[:V, :T]
+    swt = np.repeat(np.repeat(out["wt_scales"], 128, axis=0), 128, axis=1)[:H, :V]
+    sht = np.repeat(np.repeat(out["ht_scales"], 128, axis=0), 128, axis=1)[:H, :T]
+    ep, ept = _e4m3_abs_err_bound(P, sp), _e4m3_abs_err_bound(P.T, spt)
+    ew, eh = _e4m3_abs_err_bound(W.T, swt), _e4m3_abs_err_bound(h.T, sht)
+    assert np.all(np.abs(out["P_hat"] - P) <= ep) and np.all(np.abs(out["Wt_hat"] - W.T) <= ew)
+    assert np.all(np.abs(out["Pt_hat"] - P.T) <= ept) and np.all(np.abs(out["ht_hat"] - h.T) <= eh)
+    # the exact backward of the oracle, from P in float32 (the quantised one's input)
+    dh_exact = P @ W.astype(np.float64)
+    dW_exact = P.T @ h.astype(np.float64)
+    assert np.allclose(dh_exact, ref["dh"], rtol=0, atol=1e-6 * np.max(np.abs(ref["dh"])))
+    bound_dh = ep @ np.abs(W.astype(np.float64)) + (np.abs(P) + ep) @ ew.T
+    bound_dW = ept @ np.abs(h.astype(np.float64)) + (np.abs(P.T) + ept) @ eh.T
+    assert np.all(np.abs(out["dh"] - dh_exact) <= bound_dh * (1 + 1e-9))
+    assert np.all(np.abs(out["dW"] - dW_exact) <= bound_dW * (1 + 1e-9))
+    # and quantisation did change something (the check is not vacuous)
+    assert np.max(np.abs(out["dh"] - dh_exact)) > 0
+
+
+def test_fp8_backward_zero_gradient():
+    rng = np.random.default_rng(73)
+    T, H, V = 9, 128, 20
+    h = rng.normal(0, 1, (T, H)).astype(np.float32)
+    W = rng.normal(0, 0.05, (V, H)).astype(np.float32)
+    hq, hs = Q.quantize(h, Q.BLOCK, Q.ACT)
+    wq, ws = Q.quantize(W, Q.BLOCK, Q.WEIGHT)
+    out = L.lm_head_backward_fp8(hq, hs, wq, ws, Q.BLOCK, rng.integers(0, V, T), np.zeros(T), h, W)
+    assert not np.any(out["dh"]) and not np.any(out["dW"])
+    # every block of P is zero: scale 1, codes +-0 (g * -p is -0.0)
+    assert np.all(out["p_scales"] == 1.0) and np.all((out["p_codes"] & 0x7F) == 0)
+    assert not np.any(out["P_hat"]) and not np.any(out["Pt_hat"])
