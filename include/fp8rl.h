@@ -413,31 +413,37 @@ fp8rl_status fp8rl_dlogits_rows(const uint8_t* h_codes, const float* h_scales,
                                 void* stream);
 
 /* Backward through the FP8 lm_head (the chain rule of a3/a4 past the logits;
- * the paper trains with FP8 forward and backward passes, §3 and the
+ * the paper trains with FP8 forward and backward GEMMs, §3 and the
  * performance appendix).  With g_t = grad_logp[t] (e.g. from
  * fp8rl_clipped_surrogate) and lse from fp8rl_token_logprobs:
  *   P[t][v] = g_t (1{v == y_t} - exp(z[t][v] - lse_t)),  z recomputed by the
- *             FP8 GEMM of fp8rl_token_logprobs and rounded to bf16 (P is
- *             written to the workspace in both orientations; the float32
- *             logits are never stored)
+ *             FP8 GEMM of fp8rl_token_logprobs, P in float32 (neither the
+ *             logits nor P in float32 are ever stored)
  *   dh[t][k] = sum_v P[t][v] W[v][k]        float32 [T][H]
  *   dW[v][k] = sum_t P[t][v] h[t][k]        float32 [V][H]
- * The quantisers pass the gradient straight through: the two contractions
- * run on tcgen05 in BF16 with float32 accumulation over the bf16 operands
- * h_bf16 [T][H] and w_bf16 [V][H] that the codes were quantised from.
- *   h_codes ... targets   as for fp8rl_token_logprobs (same granularity)
+ * The quantisers pass the gradient straight through, and both contractions
+ * run on the block-scaled FP8 tensor-core GEMM with every operand
+ * E4M3-quantised (Eq. 3) along its own K axis: P with 1x128 blocks along V
+ * (dh), P^T with 128 x 128 blocks (dW), and the transposed bf16 operands
+ * w_bf16^T [H][V] and h_bf16^T [H][T] with 128 x 128 blocks; float32
+ * accumulation.
+ *   h_codes ... targets   as for fp8rl_token_logprobs (any granularity)
  *   lse, grad_logp        float [T] DEVICE
+ *   h_bf16, w_bf16        bf16 [T][H], [V][H], the operands the codes came from
  *   dh, dW                float out, 16-byte aligned; either may be NULL to
  *                         skip that contraction (not both)
  *   accumulate_dw         nonzero: dW += (several token chunks, one dW)
- * T and V at most 2097120 (65535 x 32), else FP8RL_ESHAPE; misaligned h_bf16,
- * w_bf16, dh, dW or workspace give FP8RL_EALIGN.  The workspace holds P twice
- * and the transposed operands: 2 (T V' + V T' + H V' + H T') bytes, V' and T'
- * rounded up to multiples of 8 (about 11.3 GB at T 16384, H 4096, V 151936);
- * callers with less memory pass token chunks (granularity other than per
- * tensor, so the chunk's codes are the batch's) and accumulate dW.  Target
- * ids are not checked again here (fp8rl_token_logprobs flags them): an id
- * outside [0, V) adds no one-hot term to its row of P. */
+ * T and V below 2^31 - 256, else FP8RL_ESHAPE; misaligned h_bf16, w_bf16, dh,
+ * dW or workspace give FP8RL_EALIGN; a non-finite h_bf16 or w_bf16 sets
+ * FP8RL_EDEVICE.  The workspace holds the codes and scales of the four
+ * quantised operands: about (T + H) V' + (V + H) T' bytes with V', T' = V, T
+ * rounded up to multiples of 128 (5.72 GB at T 16384, H 4096, V 151936);
+ * callers with less memory pass token chunks whose length is a multiple of
+ * 128 (so the 128 x 128 blocks of P^T and h^T are those of the whole batch;
+ * granularity other than per tensor, so the chunk's codes are the batch's)
+ * and accumulate dW.  Target ids are not checked again here
+ * (fp8rl_token_logprobs flags them): an id outside [0, V) adds no one-hot
+ * term to its row of P. */
 size_t fp8rl_lm_head_backward_workspace_size(int64_t T, int64_t H, int64_t V);
 
 fp8rl_status fp8rl_lm_head_backward(const uint8_t* h_codes, const float* h_scales,

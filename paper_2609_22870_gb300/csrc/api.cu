@@ -439,7 +439,9 @@ fp8rl_status fp8rl_dlogits_rows(const uint8_t* hc, const float* hs, const uint8_
 }
 
 // ------------------------------------------------------------------ lm_head backward
-constexpr int64_t kMaxBwdRows = int64_t{65535} * 32;
+// The GEMMs index rows and K with 32-bit ints: T and V (and their 128-padded
+// K extents) must stay below 2^31.
+constexpr int64_t kMaxBwdRows = (int64_t{1} << 31) - 256;
 
 size_t fp8rl_lm_head_backward_workspace_size(int64_t T, int64_t H, int64_t V) {
   return (T < 1 || H < 1 || V < 1) ? 0 : bwd_layout(T, H, V).total;
@@ -453,7 +455,7 @@ fp8rl_status fp8rl_lm_head_backward(const uint8_t* hc, const float* hs, const ui
   fp8rl_status st = check_gemm_shape(hc, hs, wc, wsc, g, T, H, V);
   if (st != FP8RL_OK) return st;
   if (!targets || !lse || !grad || !h_bf16 || !w_bf16 || (!dh && !dW)) return FP8RL_EINVAL;
-  if (T > kMaxBwdRows || V > kMaxBwdRows) return FP8RL_ESHAPE;  // transpose grid: 65535 row tiles
+  if (T > kMaxBwdRows || V > kMaxBwdRows) return FP8RL_ESHAPE;
   if (!aligned16(h_bf16) || !aligned16(w_bf16) || (dh && !aligned16(dh)) || (dW && !aligned16(dW)))
     return FP8RL_EALIGN;
   if (!ws || ws_bytes < bwd_layout(T, H, V).total) return FP8RL_EWORKSPACE;

@@ -1,61 +1,115 @@
-// Backward through the FP8 lm_head: given g_t = dLoss/dlogp_t (the clipped
-// surrogate's gradient) and the forward pass's lse, the chain rule through the
-// log-softmax gives dLoss/dz[t][v] = g_t (1{v == y_t} - exp(z[t][v] - lse_t)),
-// and through z = h W^T the two contractions
-//   dh = P W  ([T][V] x [V][H]),     dW = P^T h  ([V][T] x [T][H]).
-// The quantisers pass the gradient straight through, so the contractions take
-// the bf16 operands.  Steps, all on the caller's stream:
-//   1. the FP8 GEMM recomputes z tile by tile and its epilogue writes P in
-//      bf16 twice, [T][V] and [V][T] (logits themselves are never stored);
-//   2. W and h are transposed to [H][V] and [H][T] (K-major B operands);
-//   3. the tcgen05 BF16 GEMM forms dh (K = V) and dW (K = T) into fp32.
+// Backward through the FP8 lm_head with FP8 contractions.  Given
+// g_t = dLoss/dlogp_t (the clipped surrogate's gradient) and the forward
+// pass's lse, the chain rule through the log-softmax gives
+// P[t][v] = dLoss/dz[t][v] = g_t (1{v == y_t} - exp(z[t][v] - lse_t)), and
+// through z = h W^T the two contractions
+//   dh = P W  ([T][V] x [V][H], K = V),     dW = P^T h  ([V][T] x [T][H], K = T).
+// The quantisers pass the gradient straight through; every operand of the two
+// contractions is E4M3-quantised along its own K axis (the paper trains with
+// FP8 GEMMs in the backward pass as well, §3 and the performance appendix):
+//   1. the FP8 GEMM recomputes z tile by tile and its epilogue writes the
+//      codes of P with 1x128 scales along V and the codes of P^T with
+//      128 x 128 scales (the float32 logits and P are never stored);
+//   2. W [V][H] and h [T][H] (bf16) are transposed and quantised to W^T
+//      [H][V'] and h^T [H][T'] with 128 x 128 scales (V', T' = V, T rounded
+//      up to 128; the padding holds zero codes);
+//   3. the block-scaled FP8 GEMM forms dh and dW into float32.
+#include <cuda_fp8.h>
+
 #include "common.cuh"
+#include "e4m3_encode.cuh"
 #include "internal.h"
 
 namespace fp8rl {
 namespace {
 
-constexpr int kTile = 32;
+__device__ uint32_t d_status;
 
-// out[c][r] = in[r][c] for a bf16 matrix [rows][cols]: 32 x 32 tiles through
-// shared memory (padded against bank conflicts), 32 x 8 threads, four
-// elements a thread each way.
-__global__ void __launch_bounds__(256) transpose_bf16_kernel(const uint16_t* __restrict__ in,
-                                                             int64_t rows, int64_t cols, int64_t ld_in,
-                                                             uint16_t* __restrict__ out, int64_t ld_out) {
-  __shared__ uint16_t tile[kTile][kTile + 2];
-  const int64_t c0 = static_cast<int64_t>(blockIdx.x) * kTile;
-  const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kTile;
-  const int tx = threadIdx.x, ty = threadIdx.y;
+constexpr int kQT = 128;  // edge of a quantisation block / transpose tile
+
+// codes[c][r] = Q_FP8(in[r][c] / S) for one 128 x 128 tile of the bf16 matrix
+// in[rows][cols]: S = fl32(amax / 448) over the tile (1 when it is all zero),
+// written to scales[c / 128][r / 128] (row stride ld_out / 128).  The tile goes
+// through shared memory (row pitch 136 bf16, so column reads by a warp hit
+// distinct banks); each thread encodes 64 codes of one output row.  Rows of
+// `in` past `rows` read as zero, so the padding columns of the codes are zero.
+__global__ void __launch_bounds__(256) transpose_quantize_kernel(const uint16_t* __restrict__ in, int64_t rows,
+                                                                 int64_t cols, int64_t ld_in,
+                                                                 uint8_t* __restrict__ codes,
+                                                                 float* __restrict__ scales, int64_t ld_out) {
+  constexpr int kPitch = kQT + 8;
+  __shared__ __align__(16) uint16_t tile[kQT][kPitch];
+  __shared__ uint32_t warp_max[8];
+  const int64_t r0 = static_cast<int64_t>(blockIdx.x) * kQT;
+  const int64_t c0 = static_cast<int64_t>(blockIdx.y) * kQT;
+  const int tid = threadIdx.x;
+  uint32_t m = 0;  // running max of |x| as packed bf16x2 (NaN-propagating)
+  // 128 rows x 16 groups of 8 bf16; cols % 8 == 0 and ld_in % 8 == 0, so a
+  // group is either wholly inside the matrix or wholly outside
 #pragma unroll
-  for (int k = 0; k < kTile; k += 8) {
-    const int64_t r = r0 + ty + k, c = c0 + tx;
-    if (r < rows && c < cols) tile[ty + k][tx] = in[r * ld_in + c];
+  for (int k = 0; k < 8; ++k) {
+    const int idx = tid + k * 256;
+    const int r = idx >> 4, gq = idx & 15;
+    const int64_t gr = r0 + r, gc = c0 + gq * 8;
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (gr < rows && gc < cols) v = __ldg(reinterpret_cast<const uint4*>(in + gr * ld_in + gc));
+    *reinterpret_cast<uint4*>(&tile[r][gq * 8]) = v;
+    m = amax_bf16x8(m, v);
   }
+  const float a = amax_of(m);
+  if (!(a <= 3.4e38f)) atomicOr(&d_status, kErrDevice);  // inf or NaN input
+  const uint32_t wm = __reduce_max_sync(0xffffffffu, __float_as_uint(a));
+  if ((tid & 31) == 0) warp_max[tid >> 5] = wm;
   __syncthreads();
+  uint32_t bm = warp_max[0];
 #pragma unroll
-  for (int k = 0; k < kTile; k += 8) {
-    const int64_t c = c0 + ty + k, r = r0 + tx;
-    if (c < cols && r < rows) out[c * ld_out + r] = tile[tx][ty + k];
+  for (int i = 1; i < 8; ++i) bm = max(bm, warp_max[i]);
+  const float s = e4m3_scale(__uint_as_float(bm), false);
+  const E4M3Enc e = e4m3_encoder(s);
+  // output row c = tid / 2 (column c of the tile), codes r = 64 (tid % 2) ..
+  const int c = tid >> 1, rh = (tid & 1) * 64;
+  if (c0 + c < cols) {
+    uint4* dst = reinterpret_cast<uint4*>(codes + (c0 + c) * ld_out + r0 + rh);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      uint2 w[2];
+#pragma unroll
+      for (int h8 = 0; h8 < 2; ++h8) {
+        const int rb = rh + q * 16 + h8 * 8;
+        uint4 v;
+        v.x = tile[rb + 0][c] | (static_cast<uint32_t>(tile[rb + 1][c]) << 16);
+        v.y = tile[rb + 2][c] | (static_cast<uint32_t>(tile[rb + 3][c]) << 16);
+        v.z = tile[rb + 4][c] | (static_cast<uint32_t>(tile[rb + 5][c]) << 16);
+        v.w = tile[rb + 6][c] | (static_cast<uint32_t>(tile[rb + 7][c]) << 16);
+        w[h8] = e4m3_encode8(v, e);
+      }
+      dst[q] = make_uint4(w[0].x, w[0].y, w[1].x, w[1].y);
+    }
   }
+  if (tid == 0) scales[(c0 / kQT) * (ld_out / kQT) + r0 / kQT] = s;
 }
 
 }  // namespace
 
 BwdLayout bwd_layout(int64_t T, int64_t H, int64_t V) {
   BwdLayout l;
-  l.vp = (V + 7) / 8 * 8;  // bf16 row strides must be multiples of 16 bytes (TMA)
-  l.tp = (T + 7) / 8 * 8;
+  l.vp = (V + kQT - 1) / kQT * kQT;
+  l.tp = (T + kQT - 1) / kQT * kQT;
+  const int64_t hb = (H + kQT - 1) / kQT;
   size_t off = 0;
   auto take = [&](size_t bytes) {
     const size_t at = off;
     off = align_up(off + bytes, 256);
     return at;
   };
-  l.p = take(static_cast<size_t>(T) * l.vp * 2);
-  l.pt = take(static_cast<size_t>(V) * l.tp * 2);
-  l.wt = take(static_cast<size_t>(H) * l.vp * 2);
-  l.ht = take(static_cast<size_t>(H) * l.tp * 2);
+  l.p = take(static_cast<size_t>(T) * l.vp);
+  l.ps = take(static_cast<size_t>(l.vp / kQT) * T * 4);
+  l.pt = take(static_cast<size_t>(V) * l.tp);
+  l.pts = take(static_cast<size_t>(l.tp / kQT) * V * 4);
+  l.wt = take(static_cast<size_t>(H) * l.vp);
+  l.wts = take(static_cast<size_t>(hb) * (l.vp / kQT) * 4);
+  l.ht = take(static_cast<size_t>(H) * l.tp);
+  l.hts = take(static_cast<size_t>(hb) * (l.tp / kQT) * 4);
   l.total = off;
   return l;
 }
@@ -67,11 +121,15 @@ cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const ui
                                     int accumulate_dw, void* ws, cudaStream_t s) {
   const BwdLayout l = bwd_layout(T, H, V);
   char* base = static_cast<char*>(ws);
-  uint16_t* P = reinterpret_cast<uint16_t*>(base + l.p);
-  uint16_t* Pt = reinterpret_cast<uint16_t*>(base + l.pt);
-  uint16_t* Wt = reinterpret_cast<uint16_t*>(base + l.wt);
-  uint16_t* Ht = reinterpret_cast<uint16_t*>(base + l.ht);
-  // 1. recompute z (FP8), write P = dLoss/dz in bf16, both orientations
+  uint8_t* Pq = reinterpret_cast<uint8_t*>(base + l.p);
+  float* Ps = reinterpret_cast<float*>(base + l.ps);
+  uint8_t* Ptq = reinterpret_cast<uint8_t*>(base + l.pt);
+  float* Pts = reinterpret_cast<float*>(base + l.pts);
+  uint8_t* Wtq = reinterpret_cast<uint8_t*>(base + l.wt);
+  float* Wts = reinterpret_cast<float*>(base + l.wts);
+  uint8_t* Htq = reinterpret_cast<uint8_t*>(base + l.ht);
+  float* Hts = reinterpret_cast<float*>(base + l.hts);
+  // 1. recompute z (FP8), quantise P = dLoss/dz in both orientations
   GemmArgs a{};
   a.a_codes = hc;
   a.a_scales = hs;
@@ -84,22 +142,26 @@ cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const ui
   a.targets = targets;
   a.lse = lse;
   a.grad = grad;
-  a.p_out = P;
-  a.pt_out = Pt;
-  a.ld_p = l.vp;
-  a.ld_pt = l.tp;
+  a.pq_out = Pq;
+  a.pq_scales = Ps;
+  a.ptq_out = Ptq;
+  a.ptq_scales = Pts;
+  a.ld_pq = l.vp;
+  a.ld_ptq = l.tp;
   cudaError_t e = launch_gemm_dense_dlogits(a, s);
   if (e != cudaSuccess) return e;
-  if (dh) {  // 2./3. dh[T][H] = P[T][V] . W[V][H]: B operand W^T [H][V]
-    e = launch_transpose_bf16(W, V, H, H, Wt, l.vp, s);
+  if (dh) {  // 2./3. dh[T][H] = P[T][V'] . (W^T[H][V'])^T
+    e = launch_transpose_quantize(W, V, H, H, Wtq, Wts, l.vp, s);
     if (e != cudaSuccess) return e;
     GemmArgs d{};
-    d.a_codes = P;
-    d.b_codes = Wt;
-    d.gran = kGemmBf16;
+    d.a_codes = Pq;
+    d.a_scales = Ps;
+    d.b_codes = Wtq;
+    d.b_scales = Wts;
+    d.gran = FP8RL_GRAN_BLOCK;
     d.M = T;
     d.N = H;
-    d.K = V;
+    d.K = l.vp;
     d.lda = l.vp;
     d.ldb = l.vp;
     d.c_out = dh;
@@ -107,16 +169,18 @@ cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const ui
     e = launch_gemm_store(d, s);
     if (e != cudaSuccess) return e;
   }
-  if (dW) {  // dW[V][H] = P^T[V][T] . h[T][H]: B operand h^T [H][T]
-    e = launch_transpose_bf16(h, T, H, H, Ht, l.tp, s);
+  if (dW) {  // dW[V][H] = P^T[V][T'] . (h^T[H][T'])^T
+    e = launch_transpose_quantize(h, T, H, H, Htq, Hts, l.tp, s);
     if (e != cudaSuccess) return e;
     GemmArgs d{};
-    d.a_codes = Pt;
-    d.b_codes = Ht;
-    d.gran = kGemmBf16;
+    d.a_codes = Ptq;
+    d.a_scales = Pts;
+    d.b_codes = Htq;
+    d.b_scales = Hts;
+    d.gran = FP8RL_GRAN_BLOCK;
     d.M = V;
     d.N = H;
-    d.K = T;
+    d.K = l.tp;
     d.lda = l.tp;
     d.ldb = l.tp;
     d.c_out = dW;
@@ -127,14 +191,22 @@ cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const ui
   return e;
 }
 
-cudaError_t launch_transpose_bf16(const uint16_t* in, int64_t rows, int64_t cols, int64_t ld_in,
-                                  uint16_t* out, int64_t ld_out, cudaStream_t s) {
+cudaError_t launch_transpose_quantize(const uint16_t* in, int64_t rows, int64_t cols, int64_t ld_in,
+                                      uint8_t* codes, float* scales, int64_t ld_out, cudaStream_t s) {
   if (rows == 0 || cols == 0) return cudaSuccess;
-  const int64_t gx = (cols + kTile - 1) / kTile, gy = (rows + kTile - 1) / kTile;
+  if (cols % 8 != 0 || ld_in % 8 != 0 || ld_out % kQT != 0 || ld_out < rows) return cudaErrorInvalidValue;
+  const int64_t gx = ld_out / kQT, gy = (cols + kQT - 1) / kQT;
   if (gx > 0x7FFFFFFF || gy > 65535) return cudaErrorInvalidValue;
-  transpose_bf16_kernel<<<dim3(static_cast<unsigned>(gx), static_cast<unsigned>(gy)), dim3(kTile, 8), 0, s>>>(
-      in, rows, cols, ld_in, out, ld_out);
+  transpose_quantize_kernel<<<dim3(static_cast<unsigned>(gx), static_cast<unsigned>(gy)), 256, 0, s>>>(
+      in, rows, cols, ld_in, codes, scales, ld_out);
   return cudaGetLastError();
+}
+
+uint32_t backward_status_take() {
+  uint32_t v = 0, z = 0;
+  if (cudaMemcpyFromSymbol(&v, d_status, sizeof(v)) != cudaSuccess) return 0;
+  cudaMemcpyToSymbol(d_status, &z, sizeof(z));
+  return v;
 }
 
 }  // namespace fp8rl

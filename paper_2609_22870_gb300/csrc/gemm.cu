@@ -34,6 +34,7 @@
 #include <cmath>
 
 #include "common.cuh"
+#include "e4m3_encode.cuh"
 #include "gemm_epi.cuh"
 #include "internal.h"
 
@@ -62,8 +63,99 @@ constexpr uint32_t SC_SLOT_FLOATS = SC_KB * SC_KB_FLOATS;
 constexpr uint32_t SC_BYTES = SC_SLOTS * SC_SLOT_FLOATS * 4;
 constexpr size_t SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + SC_BYTES + 512;
 constexpr uint64_t kDrainNs = 1000000000ull;
+// Exchange slots of the dense FP8 epilogue's 128 x 128 block maxima: an
+// epilogue warp runs at most two tiles ahead of another (tile i + 2 needs the
+// accumulator buffer that every warp released at tile i), so four slots are
+// never reused while a slower warp still reads one.
+constexpr int XSLOTS = 4;
 
 __device__ __forceinline__ void flag(uint32_t bits) { atomicOr(&d_status, bits); }
+
+// E4M3 codes Q_FP8(fl32(v_i / S)) of 128 floats, four per word (byte i % 4 of
+// word i / 4), in the packed arithmetic of the quantiser.
+__device__ __forceinline__ void encode128(const float* v, float s, uint32_t (&w)[32]) {
+  const E4M3Enc e = e4m3_encoder(s);
+  if (!e.divide) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const uint32_t a = cvt_e4m3x2(neg_quotient2(f32x2(v[4 * i], v[4 * i + 1]), e));
+      const uint32_t b = cvt_e4m3x2(neg_quotient2(f32x2(v[4 * i + 2], v[4 * i + 3]), e));
+      w[i] = (a | (b << 16)) ^ 0x80808080u;  // the quotients were negated
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const uint32_t a = static_cast<uint32_t>(__nv_cvt_float2_to_fp8x2(
+          make_float2(__fdiv_rn(v[4 * i], s), __fdiv_rn(v[4 * i + 1], s)), __NV_SATFINITE, __NV_E4M3));
+      const uint32_t b = static_cast<uint32_t>(__nv_cvt_float2_to_fp8x2(
+          make_float2(__fdiv_rn(v[4 * i + 2], s), __fdiv_rn(v[4 * i + 3], s)), __NV_SATFINITE, __NV_E4M3));
+      w[i] = a | (b << 16);
+    }
+  }
+}
+
+// S = fl32(amax / 448), 1 for an all-zero block (NaN amax gives NaN).
+__device__ __forceinline__ float scale_of(float amax) { return amax == 0.f ? 1.f : __fdiv_rn(amax, kE4M3Max); }
+
+// Dense dLoss/dz of one thread's 128 columns (row `row`, columns col0 ..
+// col0 + 127; z the scaled logits), quantised for the FP8 backward:
+//   P[t][v] = g_t (1{v == y_t} - exp(z[t][v] - lse_t))   (float32)
+//   codes of P with this row's 1x128 block scale        -> pq_out / pq_scales
+//   codes of P with the 128 x 128 block scale of the tile half (the max over
+//   the four warps holding its 128 rows, exchanged through shared memory
+//   with a bounded wait), stored transposed         -> ptq_out / ptq_scales
+// Rows past M and columns past N hold 0 (the K padding of the contractions).
+// Returns false if the exchange wait expired.
+__device__ __forceinline__ bool dense_fp8_epilogue(const Params& p, const EpiState& es, float* z, int row,
+                                                   int col0, int m_blk, int rit, int half, int quarter,
+                                                   int lane, int tcount, uint64_t* blk_bar, uint32_t* blk_max,
+                                                   uint64_t lim, const volatile int* abort_flag) {
+  const int ncol = min(CHUNK, p.N - col0);
+  const bool row_ok = row < p.M;
+  const float l = row_ok ? p.lse[row] : 0.f, g = row_ok ? p.grad[row] : 0.f;
+  float amax = 0.f;
+  bool nan = false;
+#pragma unroll
+  for (int i = 0; i < CHUNK; ++i) {
+    const float v = (row_ok && i < ncol) ? g * ((i == es.j ? 1.f : 0.f) - expf(z[i] - l)) : 0.f;
+    z[i] = v;
+    amax = fmaxf(amax, fabsf(v));
+    nan |= v != v;
+  }
+  if (nan) amax = __uint_as_float(0x7FC00000u);
+  uint32_t w[32];
+  if (row_ok && col0 < p.ld_pq) {  // the row's block along N (K of the dh contraction)
+    const float s = scale_of(amax);
+    encode128(z, s, w);
+    uint4* dst = reinterpret_cast<uint4*>(p.pq_out + static_cast<size_t>(row) * p.ld_pq + col0);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) dst[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+    p.pq_scales[static_cast<size_t>(col0 / CHUNK) * p.M + row] = s;
+  }
+  // 128 x 128 block maximum: non-negative floats (and NaN above them) order
+  // like their bit patterns
+  const uint32_t wmax = __reduce_max_sync(0xffffffffu, __float_as_uint(amax));
+  const int slot = tcount % XSLOTS;
+  const uint32_t par = static_cast<uint32_t>(tcount / XSLOTS) & 1u;
+  uint32_t* bm = blk_max + (slot * 2 + half) * 4;
+  const uint32_t bar = smem_u32(&blk_bar[slot * 2 + half]);
+  if (lane == 0) {
+    bm[quarter] = wmax;
+    mbar_arrive(bar);
+  }
+  if (!__all_sync(0xffffffffu, mbar_wait(bar, par, lim, abort_flag))) return false;
+  const uint32_t bmax = max(max(bm[0], bm[1]), max(bm[2], bm[3]));
+  if (ncol <= 0) return true;
+  const float sb = scale_of(__uint_as_float(bmax));
+  encode128(z, sb, w);
+  // lanes are consecutive tokens: each column of P^T gets 32 contiguous bytes
+  uint8_t* dst = p.ptq_out + static_cast<size_t>(col0) * p.ld_ptq + row;
+#pragma unroll
+  for (int i = 0; i < CHUNK; ++i)
+    if (i < ncol) dst[static_cast<size_t>(i) * p.ld_ptq] = static_cast<uint8_t>(w[i >> 2] >> (8 * (i & 3)));
+  if (rit < ncol) p.ptq_scales[static_cast<size_t>(m_blk) * p.N + col0 + rit] = sb;
+  return true;
+}
 
 template <int MODE, int EPI>
 __global__ void __launch_bounds__(THREADS, 1)
@@ -83,8 +175,10 @@ __global__ void __launch_bounds__(THREADS, 1)
   uint64_t* sc_full = acc_empty + 2;
   uint64_t* sc_empty = sc_full + SC_SLOTS;
   uint64_t* done = sc_empty + SC_SLOTS;
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(done + 1);
+  uint64_t* blk_bar = done + 1;  // dense FP8 epilogue: [XSLOTS][2 halves]
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(blk_bar + XSLOTS * 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+  uint32_t* blk_max = tmem_holder + 2;  // [XSLOTS][2 halves][4 warps] float bits
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -101,6 +195,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       mbar_init(smem_u32(&sc_empty[i]), EPI_WARPS);
     }
     mbar_init(smem_u32(done), 1);
+    for (int i = 0; i < XSLOTS * 2; ++i) mbar_init(smem_u32(&blk_bar[i]), 4);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -267,10 +362,10 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int half = ew >> 2;      // which 128 columns of the 256-wide tile
     const int rit = quarter * 32 + lane;
     const uint32_t t_row = static_cast<uint32_t>(quarter * 32) << 16;
-    int ab = 0, sslot = 0;
+    int ab = 0, sslot = 0, tcount = 0;
     uint32_t aphase = 0, sphase = 0;
     bool ok = true;
-    for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+    for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x, ++tcount) {
       int m_blk, n_blk;
       tile_coords(tile, p, m_blk, n_blk);
       const int row = m_blk * BM + rit;
@@ -332,9 +427,47 @@ __global__ void __launch_bounds__(THREADS, 1)
           if (ab == 0) aphase ^= 1;
         }
         if (!ok) break;
-        const float* z = reinterpret_cast<const float*>(z2);
+        float* z = reinterpret_cast<float*>(z2);
+        if (EPI == kEpiDenseFp8) {
+          ok = dense_fp8_epilogue(p, es, z, row, col0, m_blk, rit, half, quarter, lane, tcount, blk_bar, blk_max,
+                                  lim, abort_flag);
+          if (!ok) break;
+        } else {
 #pragma unroll
-        for (int c = 0; c < CHUNK / 32; ++c) epi_consume32<EPI>(p, es, z + c * 32, row, col0, c * 32);
+          for (int c = 0; c < CHUNK / 32; ++c) epi_consume32<EPI>(p, es, z + c * 32, row, col0, c * 32);
+        }
+      } else if (EPI == kEpiDenseFp8) {
+        // tensor / row scaling: all 128 scaled columns into registers, buffer
+        // released, then the quantised dense epilogue
+        ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&acc_full[ab]), aphase, lim, abort_flag));
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t taddr = tmem_base + t_row + static_cast<uint32_t>(ab * BN + half * CHUNK);
+        const float sa = (MODE == kTensor) ? __ldg(p.a_scales) : (row_ok ? __ldg(p.a_scales + row) : 0.f);
+        float zf[CHUNK];
+#pragma unroll
+        for (int c = 0; c < CHUNK / 32; ++c) {
+          float(&v)[32] = *reinterpret_cast<float(*)[32]>(zf + c * 32);
+          tmem_ld_32x32b_x32(taddr + c * 32, v);
+          if (MODE == kRow) {
+            const int colq = col0 + c * 32 + lane;
+            const float sbl = colq < p.N ? __ldg(p.b_scales + colq) : 0.f;
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] *= sa * __shfl_sync(0xffffffffu, sbl, i);
+          } else {
+            const float s0 = sa * __ldg(p.b_scales);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] *= s0;
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&acc_empty[ab]));
+        ab ^= 1;
+        if (ab == 0) aphase ^= 1;
+        ok = dense_fp8_epilogue(p, es, zf, row, col0, m_blk, rit, half, quarter, lane, tcount, blk_bar, blk_max,
+                                lim, abort_flag);
+        if (!ok) break;
       } else {
         ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&acc_full[ab]), aphase, lim, abort_flag));
         if (!ok) break;
@@ -513,10 +646,12 @@ cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s) {
   p.lse = a.lse;
   p.grad = a.grad;
   p.out = a.out;
-  p.p_out = a.p_out;
-  p.pt_out = a.pt_out;
-  p.ld_p = a.ld_p;
-  p.ld_pt = a.ld_pt;
+  p.pq_out = a.pq_out;
+  p.pq_scales = a.pq_scales;
+  p.ptq_out = a.ptq_out;
+  p.ptq_scales = a.ptq_scales;
+  p.ld_pq = a.ld_pq;
+  p.ld_ptq = a.ld_ptq;
   p.c_out = a.c_out;
   p.ld_c = a.ld_c;
   p.accumulate = a.accumulate;
@@ -532,9 +667,13 @@ cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s) {
   p.wait_limit_ns = wait_limit_ns();
   const int64_t tiles = static_cast<int64_t>(p.num_m) * p.num_n;
   const int grid = static_cast<int>(tiles < sm_count() ? tiles : sm_count());
-  if constexpr (EPI == kEpiStore) {  // the backward contractions: bf16 operands only
-    return a.gran == kBf16 ? launch_mode<kBf16, EPI>(ta, tb, p, grid, s) : cudaErrorInvalidValue;
-  } else if constexpr (EPI == kEpiDense) {  // recomputed FP8 logits only
+  if constexpr (EPI == kEpiStore) {  // plain fp32 store: block-scaled FP8 (backward) or BF16
+    switch (a.gran) {
+      case kBlock: return launch_mode<kBlock, EPI>(ta, tb, p, grid, s);
+      case kBf16: return launch_mode<kBf16, EPI>(ta, tb, p, grid, s);
+      default: return cudaErrorInvalidValue;
+    }
+  } else if constexpr (EPI == kEpiDenseFp8) {  // recomputed FP8 logits only
     switch (a.gran) {
       case kTensor: return launch_mode<kTensor, EPI>(ta, tb, p, grid, s);
       case kRow: return launch_mode<kRow, EPI>(ta, tb, p, grid, s);
@@ -567,7 +706,7 @@ cudaError_t launch_gemm_dlogits(const GemmArgs& a, cudaStream_t s) {
 }
 
 cudaError_t launch_gemm_dense_dlogits(const GemmArgs& a, cudaStream_t s) {
-  return launch_gemm<kEpiDense>(a, s);
+  return launch_gemm<kEpiDenseFp8>(a, s);
 }
 
 cudaError_t launch_gemm_store(const GemmArgs& a, cudaStream_t s) { return launch_gemm<kEpiStore>(a, s); }

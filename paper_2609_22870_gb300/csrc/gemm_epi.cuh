@@ -16,10 +16,10 @@ constexpr float kLog2e = 1.4426950408889634f;
 enum { kTensor = FP8RL_GRAN_TENSOR, kRow = FP8RL_GRAN_ROWWISE, kBlock = FP8RL_GRAN_BLOCK, kBf16 = 3 };
 static_assert(kBf16 == kGemmBf16, "BF16 mode id shared with the host interface");
 // Epilogues: streaming LSE partials + target logit; dense dlogits rows (fp32);
-// dlogits of every token in bf16, both [M][N] and transposed [N][M] (the
-// operands of the two backward contractions); plain store of the fp32
+// dlogits of every token E4M3-quantised in both orientations, the A operands
+// of the two FP8 backward contractions (gemm.cu); plain store of the fp32
 // accumulators (optionally added to what is there).
-enum { kEpiLse = 0, kEpiDlogits = 1, kEpiDense = 2, kEpiStore = 3 };
+enum { kEpiLse = 0, kEpiDlogits = 1, kEpiDenseFp8 = 2, kEpiStore = 3 };
 
 struct Params {
   const float* a_scales;
@@ -30,9 +30,11 @@ struct Params {
   const float* lse;
   const float* grad;
   float* out;
-  uint16_t* p_out;   // kEpiDense: bf16 [M][ld_p]
-  uint16_t* pt_out;  // kEpiDense: bf16 [N][ld_pt]
-  int64_t ld_p, ld_pt;
+  uint8_t* pq_out;   // kEpiDenseFp8: P codes [M][ld_pq], 1x128 blocks along N
+  float* pq_scales;  //   [ld_pq / 128][M]
+  uint8_t* ptq_out;  //   P^T codes [N][ld_ptq], 128 x 128 blocks
+  float* ptq_scales; //   [ld_ptq / 128][N] (each block's scale on its 128 rows)
+  int64_t ld_pq, ld_ptq;
   float* c_out;      // kEpiStore: fp32 [M][ld_c]
   int64_t ld_c;
   int accumulate;
@@ -113,35 +115,6 @@ __device__ __forceinline__ void epi_consume32(const Params& p, EpiState& e, cons
 #pragma unroll
     for (int i = 0; i < 32; ++i)
       if (i < ncol) o[i] = g * ((i == jj ? 1.f : 0.f) - expf(z[i] - l));
-  } else if (EPI == kEpiDense) {
-    const float l = p.lse[row], g = p.grad[row];
-    const int jj = e.j - base;
-    const int c = col0 + base;
-    uint32_t w[16];  // bf16 pairs, column order
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      const float v0 = g * ((2 * i == jj ? 1.f : 0.f) - expf(z[2 * i] - l));
-      const float v1 = g * ((2 * i + 1 == jj ? 1.f : 0.f) - expf(z[2 * i + 1] - l));
-      w[i] = pack_bf16x2(v0, v1);
-    }
-    uint16_t* pr = p.p_out + static_cast<size_t>(row) * p.ld_p + c;  // 64-byte aligned
-    uint16_t* pt = p.pt_out + static_cast<size_t>(c) * p.ld_pt + row;
-    if (ncol >= 32) {
-#pragma unroll
-      for (int q = 0; q < 4; ++q)
-        reinterpret_cast<uint4*>(pr)[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
-#pragma unroll
-      for (int i = 0; i < 32; ++i)  // lanes are consecutive rows: 64 contiguous bytes per column
-        pt[static_cast<size_t>(i) * p.ld_pt] = static_cast<uint16_t>(w[i >> 1] >> (16 * (i & 1)));
-    } else {
-#pragma unroll
-      for (int i = 0; i < 32; ++i)
-        if (i < ncol) {
-          const uint16_t b = static_cast<uint16_t>(w[i >> 1] >> (16 * (i & 1)));
-          pr[i] = b;
-          pt[static_cast<size_t>(i) * p.ld_pt] = b;
-        }
-    }
   } else {  // kEpiStore
     float* cr = p.c_out + static_cast<size_t>(row) * p.ld_c + col0 + base;  // 16-byte aligned
     if (ncol >= 32) {

@@ -38,10 +38,12 @@ struct GemmArgs {
   const float* lse;         // [M]
   const float* grad;        // [M]
   float* out;               // [M][N]
-  // dense dlogits epilogue (bf16, both orientations)
-  uint16_t* p_out;          // [M][ld_p]
-  uint16_t* pt_out;         // [N][ld_pt]
-  int64_t ld_p, ld_pt;
+  // dense dlogits epilogue (E4M3 codes and scales, both orientations)
+  uint8_t* pq_out;          // [M][ld_pq], 1x128 blocks along N
+  float* pq_scales;         // [ld_pq / 128][M]
+  uint8_t* ptq_out;         // [N][ld_ptq], 128 x 128 blocks
+  float* ptq_scales;        // [ld_ptq / 128][N]
+  int64_t ld_pq, ld_ptq;
   // store epilogue (fp32 accumulators)
   float* c_out;             // [M][ld_c], 16-byte aligned, ld_c % 4 == 0
   int64_t ld_c;
@@ -57,8 +59,10 @@ cudaError_t launch_gemm_dlogits(const GemmArgs& a, cudaStream_t s);
 cudaError_t launch_gemm_dense_dlogits(const GemmArgs& a, cudaStream_t s);
 cudaError_t launch_gemm_store(const GemmArgs& a, cudaStream_t s);
 struct BwdLayout {
-  int64_t vp, tp;             // padded row lengths of P [T][vp] and P^T, h^T [.][tp]
-  size_t p, pt, wt, ht, total;  // byte offsets in the workspace
+  int64_t vp, tp;  // V and T rounded up to multiples of 128 (the K extents)
+  // byte offsets in the workspace: codes and scales of P [T][vp], P^T [V][tp],
+  // W^T [H][vp], h^T [H][tp]
+  size_t p, ps, pt, pts, wt, wts, ht, hts, total;
 };
 BwdLayout bwd_layout(int64_t T, int64_t H, int64_t V);
 cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const uint8_t* wc,
@@ -66,8 +70,12 @@ cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const ui
                                     const int32_t* targets, const float* lse, const float* grad,
                                     const uint16_t* h, const uint16_t* W, float* dh, float* dW,
                                     int accumulate_dw, void* ws, cudaStream_t s);
-cudaError_t launch_transpose_bf16(const uint16_t* in, int64_t rows, int64_t cols, int64_t ld_in,
-                                  uint16_t* out, int64_t ld_out, cudaStream_t s);
+// codes [cols][ld_out] of the transposed bf16 matrix in [rows][ld_in] with
+// 128 x 128 E4M3 blocks, scales [ceil(cols/128)][ld_out/128]; columns
+// rows .. ld_out-1 of the codes are zero (ld_out a multiple of 128, >= rows)
+cudaError_t launch_transpose_quantize(const uint16_t* in, int64_t rows, int64_t cols, int64_t ld_in,
+                                      uint8_t* codes, float* scales, int64_t ld_out, cudaStream_t s);
+uint32_t backward_status_take();
 cudaError_t launch_combine(const float2* partials, const float* zy, const int32_t* targets,
                            const float* logp_old, float* logp, float* lse, float* ratio,
                            int64_t M, int64_t N, cudaStream_t s);

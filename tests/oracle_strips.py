@@ -30,3 +30,15 @@ def bf16_strip(args):
     """z[:, v0:v1] of the BF16 shadow pass: float64 products of the bf16 values."""
     h_rows, w_strip = args
     return OL.bf16_logits(h_rows, w_strip)
+
+
+def bwd_dh_strip(args):
+    """Partial dh of the FP8 backward over one vocabulary strip: the oracle
+    quantises the strip of W with 128 x 128 blocks (the blocks of W^T), and
+    returns (P_hat[:, strip] @ W_hat_strip, |P_hat[:, strip]| @ |W_hat_strip|,
+    slack[:, strip] @ |W_hat_strip|) in float64."""
+    p_hat, slack, w_strip = args
+    wq, ws = OQ.quantize(w_strip, OQ.BLOCK, OQ.WEIGHT)
+    wd = OQ.dequantize(wq, ws, OQ.BLOCK, OQ.WEIGHT)
+    aw = np.abs(wd)
+    return p_hat @ wd, np.abs(p_hat) @ aw, slack @ aw

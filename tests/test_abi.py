@@ -106,7 +106,7 @@ int main(void) {
   CHECK(fp8rl_scales_count(151936, 4096, FP8RL_GRAN_ROWWISE, FP8RL_ROLE_WEIGHT) == 151936);
   CHECK(fp8rl_scales_count(7, 4096, FP8RL_GRAN_TENSOR, FP8RL_ROLE_ACT) == 1);
   CHECK(fp8rl_token_logprobs_workspace_size(16384, 4096, 151936, FP8RL_GRAN_BLOCK) > 0);
-  CHECK(fp8rl_lm_head_backward_workspace_size(16384, 4096, 151936) > (size_t)11e9);
+  CHECK(fp8rl_lm_head_backward_workspace_size(16384, 4096, 151936) > (size_t)5.7e9);
   /* argument checks: null pointers, bad enums and shapes are refused on the host */
   CHECK(fp8rl_quantize(NULL, 4, 128, 128, FP8RL_GRAN_ROWWISE, FP8RL_ROLE_ACT, NULL, NULL, NULL, 0, NULL)
         == FP8RL_EINVAL);
