@@ -45,11 +45,20 @@ typedef enum fp8rl_status {
 /* Scaling granularity of Eq. 3 (§2.2): one scale per tensor, per row, or per
  * block.  For the lm_head operands "row" means one scale per token of h[T][H]
  * and one per vocabulary row (output channel) of W[V][H]; "block" means 1x128
- * blocks of h and 128x128 blocks of W. */
+ * blocks of h and 128x128 blocks of W.
+ * FP8RL_GRAN_BLOCK_UE8M0 is the block layout with power-of-two scales (the
+ * codes and scales of fp8rl_quantize_ue8m0 at FP8RL_GRAN_BLOCK), a variant
+ * outside the paper: the scoring calls then apply the scales in the tensor
+ * cores' block-scaled MMA (E8M0 scale factors) instead of promoting each
+ * 128-wide K block in registers.  Accepted by the scoring calls
+ * (fp8rl_token_logprobs and its halves, the no-alloc variant, dlogits rows,
+ * the lm_head backward) and by fp8rl_scales_count; the quantisers take
+ * FP8RL_GRAN_BLOCK. */
 typedef enum fp8rl_gran {
   FP8RL_GRAN_TENSOR = 0,
   FP8RL_GRAN_ROWWISE = 1,
-  FP8RL_GRAN_BLOCK = 2
+  FP8RL_GRAN_BLOCK = 2,
+  FP8RL_GRAN_BLOCK_UE8M0 = 3
 } fp8rl_gran;
 
 /* Operand role, which fixes the block shape and scale layout in block mode. */
@@ -138,7 +147,12 @@ fp8rl_status fp8rl_quantize_ue8m0(const void* x, int64_t rows, int64_t cols, int
  *   lse               float [T] out, or NULL
  *   ratio             float [T] out, or NULL (needs logp_old)
  * Requires T >= 1, V >= 1, H >= 16, H % 16 == 0 (H % 128 == 0 in block mode),
- * code pointers 16-byte aligned.  Temperature 1. */
+ * code pointers 16-byte aligned.  Temperature 1.
+ * With FP8RL_GRAN_BLOCK_UE8M0 the workspace also holds the E8M0 scale-factor
+ * images the block-scaled MMA reads (one byte per token, or per vocabulary
+ * row block, and K block, laid out for the tensor memory; about (T + V)*H/128
+ * bytes), and a scale that is not a power of two in E8M0's range
+ * (2^-127 .. 2^127) sets FP8RL_EDEVICE. */
 size_t fp8rl_token_logprobs_workspace_size(int64_t T, int64_t H, int64_t V, fp8rl_gran gran);
 
 fp8rl_status fp8rl_token_logprobs(const uint8_t* h_codes, const float* h_scales,

@@ -20,6 +20,8 @@ lib = ctypes.CDLL(_LIB_PATH)
 
 OK, EINVAL, ESHAPE, EALIGN, EWORKSPACE, ECUDA, EDEVICE, ETIMEOUT = range(8)
 GRAN_TENSOR, GRAN_ROWWISE, GRAN_BLOCK = 0, 1, 2
+# block layout with power-of-two scales, applied by the block-scaled MMA (scoring calls only)
+GRAN_BLOCK_UE8M0 = 3
 ROLE_ACT, ROLE_WEIGHT = 0, 1
 CALIB_EXACT, CALIB_GRID = 0, 1
 CLIP_HI, CLIP_LO = 1, 2

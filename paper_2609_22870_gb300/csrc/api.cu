@@ -23,6 +23,9 @@ fp8rl_status cuda_fail(cudaError_t e) {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 bool valid_gran(int g) { return g == FP8RL_GRAN_TENSOR || g == FP8RL_GRAN_ROWWISE || g == FP8RL_GRAN_BLOCK; }
+// the scoring calls also take the block layout with power-of-two scales
+bool valid_score_gran(int g) { return valid_gran(g) || g == FP8RL_GRAN_BLOCK_UE8M0; }
+bool block_layout(int g) { return g == FP8RL_GRAN_BLOCK || g == FP8RL_GRAN_BLOCK_UE8M0; }
 
 // Workspace layout of fp8rl_token_logprobs: per-token LSE partials
 // [gemm_partials_per_token(V)][T] float2, then z_y [T] float.
@@ -35,9 +38,9 @@ size_t logprob_ws(int64_t T, int64_t V) {
 
 fp8rl_status check_gemm_shape(const uint8_t* hc, const float* hs, const uint8_t* wc, const float* wsc,
                               fp8rl_gran g, int64_t T, int64_t H, int64_t V) {
-  if (!hc || !hs || !wc || !wsc || !valid_gran(g)) return FP8RL_EINVAL;
+  if (!hc || !hs || !wc || !wsc || !valid_score_gran(g)) return FP8RL_EINVAL;
   if (T < 1 || V < 1 || H < 16) return FP8RL_ESHAPE;
-  if (H % 16 != 0 || (g == FP8RL_GRAN_BLOCK && H % 128 != 0)) return FP8RL_ESHAPE;
+  if (H % 16 != 0 || (block_layout(g) && H % 128 != 0)) return FP8RL_ESHAPE;
   if (T > 0x7FFFFFFF || V > 0x7FFFFFFF || H > 0x7FFFFFFF) return FP8RL_ESHAPE;
   if (!aligned16(hc) || !aligned16(wc)) return FP8RL_EALIGN;
   return FP8RL_OK;
@@ -120,7 +123,7 @@ fp8rl_status fp8rl_wait_selftest(uint64_t limit_ns, void* stream) {
 
 // ------------------------------------------------------------------ quantize
 int64_t fp8rl_scales_count(int64_t rows, int64_t cols, fp8rl_gran g, fp8rl_role role) {
-  if (rows < 0 || cols < 0 || !valid_gran(g)) return 0;
+  if (rows < 0 || cols < 0 || !valid_score_gran(g)) return 0;
   if (g == FP8RL_GRAN_TENSOR) return 1;
   if (g == FP8RL_GRAN_ROWWISE) return rows;
   if (cols % 128 != 0) return 0;
@@ -162,9 +165,10 @@ fp8rl_status fp8rl_quantize_ue8m0(const void* x, int64_t rows, int64_t cols, int
 }
 
 // ------------------------------------------------------------------ scoring
-size_t fp8rl_token_logprobs_workspace_size(int64_t T, int64_t, int64_t V, fp8rl_gran) {
-  if (T < 0 || V < 0) return 0;
-  return logprob_ws(T, V);
+size_t fp8rl_token_logprobs_workspace_size(int64_t T, int64_t H, int64_t V, fp8rl_gran g) {
+  if (T < 0 || V < 0 || H < 0) return 0;
+  // the UE8M0 mode adds the scale-factor images of the block-scaled MMA
+  return logprob_ws(T, V) + (g == FP8RL_GRAN_BLOCK_UE8M0 ? gemm_ue8m0_image_bytes(T, V, H) : 0);
 }
 
 fp8rl_status fp8rl_logit_partials(const uint8_t* hc, const float* hs, const uint8_t* wc,
@@ -173,7 +177,8 @@ fp8rl_status fp8rl_logit_partials(const uint8_t* hc, const float* hs, const uint
   fp8rl_status st = check_gemm_shape(hc, hs, wc, wsc, g, T, H, V);
   if (st != FP8RL_OK) return st;
   if (!targets) return FP8RL_EINVAL;
-  if (!ws || ws_bytes < logprob_ws(T, V)) return FP8RL_EWORKSPACE;
+  if (!ws || ws_bytes < fp8rl_token_logprobs_workspace_size(T, H, V, g)) return FP8RL_EWORKSPACE;
+  if (g == FP8RL_GRAN_BLOCK_UE8M0 && !aligned16(ws)) return FP8RL_EALIGN;
   GemmArgs a{};
   a.a_codes = hc;
   a.a_scales = hs;
@@ -186,6 +191,7 @@ fp8rl_status fp8rl_logit_partials(const uint8_t* hc, const float* hs, const uint
   a.targets = targets;
   a.partials = static_cast<float2*>(ws);
   a.zy = reinterpret_cast<float*>(static_cast<char*>(ws) + partials_bytes(T, V));
+  if (g == FP8RL_GRAN_BLOCK_UE8M0) a.sf_images = static_cast<uint8_t*>(ws) + logprob_ws(T, V);
   cudaError_t e = launch_gemm_lse(a, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? FP8RL_OK : cuda_fail(e);
 }
@@ -194,7 +200,7 @@ fp8rl_status fp8rl_combine_logprobs(int64_t T, int64_t, int64_t V, fp8rl_gran g,
                                     const int32_t* targets, const float* logp_old, float* logp,
                                     float* lse, float* ratio, void* ws, size_t ws_bytes,
                                     void* stream) {
-  if (!targets || !logp || !valid_gran(g) || (ratio && !logp_old)) return FP8RL_EINVAL;
+  if (!targets || !logp || !valid_score_gran(g) || (ratio && !logp_old)) return FP8RL_EINVAL;
   if (T < 1 || V < 1) return FP8RL_ESHAPE;
   if (!ws || ws_bytes < logprob_ws(T, V)) return FP8RL_EWORKSPACE;
   const float2* partials = static_cast<const float2*>(ws);
@@ -391,9 +397,10 @@ static size_t dl_scales_bytes(int64_t n, int64_t H) {
 }
 static size_t dl_vec_bytes(int64_t n) { return align_up(static_cast<size_t>(n > 0 ? n : 1) * 4, 256); }
 
-size_t fp8rl_dlogits_workspace_size(int64_t n, int64_t H, int64_t, fp8rl_gran) {
-  if (n < 0 || H < 0) return 0;
-  return dl_codes_bytes(n, H) + dl_scales_bytes(n, H) + 3 * dl_vec_bytes(n);
+size_t fp8rl_dlogits_workspace_size(int64_t n, int64_t H, int64_t V, fp8rl_gran g) {
+  if (n < 0 || H < 0 || V < 0) return 0;
+  return dl_codes_bytes(n, H) + dl_scales_bytes(n, H) + 3 * dl_vec_bytes(n) +
+         (g == FP8RL_GRAN_BLOCK_UE8M0 ? gemm_ue8m0_image_bytes(n, V, H) : 0);
 }
 
 fp8rl_status fp8rl_dlogits_rows(const uint8_t* hc, const float* hs, const uint8_t* wc,
@@ -407,6 +414,7 @@ fp8rl_status fp8rl_dlogits_rows(const uint8_t* hc, const float* hs, const uint8_
   if (n_rows < 0 || n_rows > 0x7FFFFFFF) return FP8RL_ESHAPE;
   if (n_rows == 0) return FP8RL_OK;
   if (!ws || ws_bytes < fp8rl_dlogits_workspace_size(n_rows, H, V, g)) return FP8RL_EWORKSPACE;
+  if (!aligned16(ws)) return FP8RL_EALIGN;
   char* p = static_cast<char*>(ws);
   uint8_t* g_codes = reinterpret_cast<uint8_t*>(p);
   p += dl_codes_bytes(n_rows, H);
@@ -417,6 +425,7 @@ fp8rl_status fp8rl_dlogits_rows(const uint8_t* hc, const float* hs, const uint8_
   float* g_lse = reinterpret_cast<float*>(p);
   p += dl_vec_bytes(n_rows);
   float* g_grad = reinterpret_cast<float*>(p);
+  p += dl_vec_bytes(n_rows);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e = launch_gather_rows(hc, hs, g, T, H, targets, lse, grad, rows, n_rows, g_codes,
                                      g_scales, g_t, g_lse, g_grad, s);
@@ -434,6 +443,7 @@ fp8rl_status fp8rl_dlogits_rows(const uint8_t* hc, const float* hs, const uint8_
   a.lse = g_lse;
   a.grad = g_grad;
   a.out = out;
+  if (g == FP8RL_GRAN_BLOCK_UE8M0) a.sf_images = reinterpret_cast<uint8_t*>(p);
   e = launch_gemm_dlogits(a, s);
   return e == cudaSuccess ? FP8RL_OK : cuda_fail(e);
 }

@@ -110,6 +110,7 @@ BwdLayout bwd_layout(int64_t T, int64_t H, int64_t V) {
   l.wts = take(static_cast<size_t>(hb) * (l.vp / kQT) * 4);
   l.ht = take(static_cast<size_t>(H) * l.tp);
   l.hts = take(static_cast<size_t>(hb) * (l.tp / kQT) * 4);
+  l.sf = take(gemm_ue8m0_image_bytes(T, V, H));  // UE8M0 recompute only
   l.total = off;
   return l;
 }
@@ -148,6 +149,7 @@ cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const ui
   a.ptq_scales = Pts;
   a.ld_pq = l.vp;
   a.ld_ptq = l.tp;
+  a.sf_images = reinterpret_cast<uint8_t*>(base + l.sf);
   cudaError_t e = launch_gemm_dense_dlogits(a, s);
   if (e != cudaSuccess) return e;
   if (dh) {  // 2./3. dh[T][H] = P[T][V'] . (W^T[H][V'])^T

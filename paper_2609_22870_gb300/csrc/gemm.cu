@@ -61,7 +61,28 @@ constexpr int SC_KB = 4;                          // K blocks per slot
 constexpr uint32_t SC_KB_FLOATS = BM + 4;         // 128 activation + 2 weight (+2 pad)
 constexpr uint32_t SC_SLOT_FLOATS = SC_KB * SC_KB_FLOATS;
 constexpr uint32_t SC_BYTES = SC_SLOTS * SC_SLOT_FLOATS * 4;
-constexpr size_t SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + SC_BYTES + 512;
+// UE8M0 (hardware block scaling) mode: the E8M0 scale factors come as images
+// in global memory (ue8m0_pack_kernel), one per group of four K blocks and
+// 128-row token block or 256-row vocabulary tile, and the producer loads a
+// group's images with the stage of its first K block.  An image is 32 lanes x
+// 16 bytes: row i of the block in lane i % 32, word i / 32, and byte q of the
+// word the scale of K block 4g + q.  One image covers the 128 token rows, two
+// the 256 vocabulary rows.
+constexpr int SF_KB = 4;                          // K blocks per image group
+constexpr uint32_t SF_IMG_BYTES = 512;
+constexpr uint32_t SF_GROUP_BYTES = 3 * SF_IMG_BYTES;
+constexpr uint32_t SF_BYTES = STAGES * SF_GROUP_BYTES;
+// In TMEM the mode keeps one 256-column accumulator (columns 0..255) and a
+// ring of scale factors from column 256: per group 4 columns for the rows of A
+// and 8 for those of B (entry i in lane i % 32 of every lane quarter, column
+// i / 32), 16 groups deep.
+constexpr uint32_t SF_TCOL0 = 256;
+constexpr uint32_t SF_TCOLS = 12;
+constexpr int SF_TRING = 16;
+template <int MODE>
+constexpr uint32_t ring_bytes() { return MODE == kUe8m0 ? SF_BYTES : SC_BYTES; }
+template <int MODE>
+constexpr size_t smem_bytes() { return 1024 + STAGES * STAGE_BYTES + ring_bytes<MODE>() + 512; }
 constexpr uint64_t kDrainNs = 1000000000ull;
 // Exchange slots of the dense FP8 epilogue's 128 x 128 block maxima: an
 // epilogue warp runs at most two tiles ahead of another (tile i + 2 needs the
@@ -70,6 +91,75 @@ constexpr uint64_t kDrainNs = 1000000000ull;
 constexpr int XSLOTS = 4;
 
 __device__ __forceinline__ void flag(uint32_t bits) { atomicOr(&d_status, bits); }
+
+// E8M0 byte of a power-of-two float32 scale (its biased exponent; 2^-127,
+// a subnormal float32, is byte 0).  A scale that is not a positive power of
+// two in E8M0's range is bad input: NaN byte 0xFF, status flagged.
+__device__ __forceinline__ uint32_t e8m0_byte(float s) {
+  const uint32_t b = __float_as_uint(s);
+  if (b == 0x00400000u) return 0;
+  const uint32_t e = b >> 23;
+  if ((b & 0x807FFFFFu) != 0 || e == 0 || e >= 255) {
+    flag(kErrDevice);
+    return 0xFFu;
+  }
+  return e;
+}
+
+// Bulk copy global -> shared of `bytes` (a multiple of 16, both addresses
+// 16-byte aligned), completing as transaction bytes on mbarrier `bar`.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+      "l"(src), "r"(bytes), "r"(bar)
+      : "memory");
+}
+
+// Shared-memory descriptor of a 32-row x 16-byte image without swizzle
+// (8-row x 16-byte core matrices, 128 bytes apart), the source of a
+// 32x128b tcgen05.cp.
+__device__ __forceinline__ uint64_t smem_desc_plain(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>(128u >> 4) << 16;
+  d |= static_cast<uint64_t>(128u >> 4) << 32;
+  d |= static_cast<uint64_t>(1u) << 46;
+  return d;
+}
+
+// Copies a 32-row x 128-bit image from shared memory to TMEM columns
+// [taddr, taddr + 4) of lanes 0..31, repeated in every lane quarter; issued by
+// one elected lane of a converged warp, in order with its MMAs.
+__device__ __forceinline__ void tmem_cp_32x128b_x4_elect(uint32_t taddr, uint64_t sdesc) {
+  asm volatile(
+      "{\n\t.reg .pred e;\n\t"
+      "elect.sync _|e, 0xffffffff;\n\t"
+      "@e tcgen05.cp.cta_group::1.32x128b.warpx4 [%0], %1;\n\t}" ::"r"(taddr),
+      "l"(sdesc)
+      : "memory");
+}
+
+// D (+)= (A x SFA) * (B x SFB)^T with E8M0 scale factors per 32-wide K step
+// (kind::mxf8f6f4, E4M3 operands): sfa / sfb are TMEM addresses of the scale
+// vectors, idesc selects the byte of each word; warp-converged.
+__device__ __forceinline__ void mma_mx_e4m3_elect(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                                  uint32_t idesc, uint32_t sfa, uint32_t sfb,
+                                                  uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p, e;\n\t"
+      "setp.ne.b32 p, %6, 0;\n\t"
+      "elect.sync _|e, 0xffffffff;\n\t"
+      "@e tcgen05.mma.cta_group::1.kind::mxf8f6f4.block_scale.scale_vec::1X [%0], %1, %2, %3, [%4], [%5], p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(sfa), "r"(sfb), "r"(accumulate)
+      : "memory");
+}
+
+// Instruction descriptor of the block-scaled MMA: E4M3 A and B, K-major,
+// E8M0 scale factors (bit 23), N >> 3 at bit 17, M >> 7 at bit 27; the scale
+// byte of B at bits 4-5 and of A at bits 29-30.
+__host__ __device__ constexpr uint32_t idesc_mx_e4m3(uint32_t M, uint32_t N) {
+  return ((N >> 3) << 17) | (1u << 23) | ((M >> 7) << 27);
+}
 
 // E4M3 codes Q_FP8(fl32(v_i / S)) of 128 floats, four per word (byte i % 4 of
 // word i / 4), in the packed arithmetic of the quantiser.
@@ -167,7 +257,8 @@ __global__ void __launch_bounds__(THREADS, 1)
   uint8_t* smA = smem;
   uint8_t* smB = smem + STAGES * A_BYTES;
   float* sc_ring = reinterpret_cast<float*>(smB + STAGES * B_BYTES);  // [SC_SLOTS][132]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smB + STAGES * B_BYTES + SC_BYTES);
+  uint8_t* sf_img = smB + STAGES * B_BYTES;  // UE8M0 mode: [STAGES][3 images]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smB + STAGES * B_BYTES + ring_bytes<MODE>());
   uint64_t* full = bars;
   uint64_t* empty = bars + STAGES;
   uint64_t* acc_full = bars + 2 * STAGES;
@@ -232,11 +323,22 @@ __global__ void __launch_bounds__(THREADS, 1)
         ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&empty[stage]), phase ^ 1, lim, abort_flag));
         if (!ok) break;
         if (elect_one()) {
-          mbar_arrive_expect_tx(smem_u32(&full[stage]), STAGE_BYTES);
+          // UE8M0 mode: the first K block of each group also brings the
+          // group's scale-factor images
+          const bool sf = MODE == kUe8m0 && kb % SF_KB == 0;
+          mbar_arrive_expect_tx(smem_u32(&full[stage]), STAGE_BYTES + (sf ? SF_GROUP_BYTES : 0u));
           // K coordinate in elements: 128 E4M3 or 64 BF16 per 128-byte row
           const int kx = kb * ((MODE == kBf16) ? BK / 2 : BK);
           tma_load_2d(smem_u32(smA + stage * A_BYTES), &tmA, smem_u32(&full[stage]), kx, m0);
           tma_load_2d(smem_u32(smB + stage * B_BYTES), &tmB, smem_u32(&full[stage]), kx, n0);
+          if (sf) {
+            const size_t g = static_cast<size_t>(kb / SF_KB);
+            const uint32_t dst = smem_u32(sf_img + stage * SF_GROUP_BYTES);
+            bulk_load(dst, p.sf_a + (static_cast<size_t>(m_blk) * p.num_kg + g) * SF_IMG_BYTES, SF_IMG_BYTES,
+                      smem_u32(&full[stage]));
+            bulk_load(dst + SF_IMG_BYTES, p.sf_b + (static_cast<size_t>(n_blk) * p.num_kg + g) * 2 * SF_IMG_BYTES,
+                      2 * SF_IMG_BYTES, smem_u32(&full[stage]));
+          }
         }
         __syncwarp();
         armed |= 1u << stage;
@@ -296,6 +398,57 @@ __global__ void __launch_bounds__(THREADS, 1)
       flag(kErrTimeout);
     }
     asm volatile("cp.async.wait_all;" ::: "memory");  // no copy in flight at exit
+   } else if (warp == 1 && MODE == kUe8m0) {
+    // ------------------------------------------------------------ MMA issuer (UE8M0)
+    // one accumulator over all of K; at the first K block of each group the
+    // group's scale images are copied from the stage into the TMEM ring (in
+    // order with the MMAs that read them, so the stage's release covers the
+    // copy too), and each K block's four block-scaled MMAs select byte
+    // kb % 4 of the scale words
+    int stage = 0, gcount = 0;
+    uint32_t phase = 0, aphase = 0;
+    uint32_t sf = tmem_base + SF_TCOL0;
+    constexpr uint32_t idesc = idesc_mx_e4m3(BM, BN);
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+      ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&acc_empty[0]), aphase ^ 1, lim, abort_flag));
+      if (!ok) break;
+      tc_fence_after();
+      for (int kb = 0; kb < p.num_kb; ++kb) {
+        ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&full[stage]), phase, lim, abort_flag));
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t q = static_cast<uint32_t>(kb % SF_KB);
+        if (q == 0) {
+          sf = tmem_base + SF_TCOL0 + static_cast<uint32_t>(gcount % SF_TRING) * SF_TCOLS;
+          ++gcount;
+          const uint32_t img = smem_u32(sf_img + stage * SF_GROUP_BYTES);
+          tmem_cp_32x128b_x4_elect(sf, smem_desc_plain(img));
+          tmem_cp_32x128b_x4_elect(sf + 4, smem_desc_plain(img + SF_IMG_BYTES));
+          tmem_cp_32x128b_x4_elect(sf + 8, smem_desc_plain(img + 2 * SF_IMG_BYTES));
+        }
+        const uint64_t adesc = smem_desc_sw128(smem_u32(smA + stage * A_BYTES));
+        const uint64_t bdesc = smem_desc_sw128(smem_u32(smB + stage * B_BYTES));
+        const uint32_t id = idesc | (q << 29) | (q << 4);
+#pragma unroll
+        for (int k = 0; k < BK / 32; ++k)
+          mma_mx_e4m3_elect(tmem_base, adesc + 2 * k, bdesc + 2 * k, id, sf, sf + 4, kb > 0 || k > 0);
+        mma_commit_elect(smem_u32(&empty[stage]));
+        if (++stage == STAGES) {
+          stage = 0;
+          phase ^= 1;
+        }
+      }
+      if (!ok) break;
+      mma_commit_elect(smem_u32(&acc_full[0]));
+      aphase ^= 1;
+    }
+    if (!ok && lane == 0) {
+      *abort_flag = 1;
+      flag(kErrTimeout);
+    }
+    mma_commit_elect(smem_u32(done));
+    mbar_wait(smem_u32(done), 0, kDrainNs, nullptr);
    } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     // whole warp converged; elect.sync picks the lane that issues each
@@ -436,6 +589,29 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
           for (int c = 0; c < CHUNK / 32; ++c) epi_consume32<EPI>(p, es, z + c * 32, row, col0, c * 32);
         }
+      } else if (MODE == kUe8m0) {
+        // scales already applied by the MMA: all 128 columns into registers,
+        // the single accumulator released at once, then the epilogue
+        ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&acc_full[0]), aphase, lim, abort_flag));
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t taddr = tmem_base + t_row + static_cast<uint32_t>(half * CHUNK);
+        float zf[CHUNK];
+#pragma unroll
+        for (int c = 0; c < CHUNK / 32; ++c)
+          tmem_ld_32x32b_x32(taddr + c * 32, *reinterpret_cast<float(*)[32]>(zf + c * 32));
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&acc_empty[0]));
+        aphase ^= 1;
+        if (EPI == kEpiDenseFp8) {
+          ok = dense_fp8_epilogue(p, es, zf, row, col0, m_blk, rit, half, quarter, lane, tcount, blk_bar, blk_max,
+                                  lim, abort_flag);
+          if (!ok) break;
+        } else {
+#pragma unroll
+          for (int c = 0; c < CHUNK / 32; ++c) epi_consume32<EPI>(p, es, zf + c * 32, row, col0, c * 32);
+        }
       } else if (EPI == kEpiDenseFp8) {
         // tensor / row scaling: all 128 scaled columns into registers, buffer
         // released, then the quantised dense epilogue
@@ -522,6 +698,51 @@ __global__ void ratios_kernel(const float* __restrict__ a, const float* __restri
     r[t] = expf(a[t] - b[t]);
 }
 
+// E8M0 scale-factor images of the UE8M0 mode (layout at SF_IMG_BYTES) from
+// the power-of-two float32 scales: activations [num_kb][M] (1x128 blocks),
+// weights [n_chunks][num_kb] (128x128 blocks).  One warp per image group:
+// first the num_m x num_kg groups of A, then the num_n x num_kg of B.  Rows
+// past M or N and K blocks past num_kb get scale 1 (byte 127).
+__global__ void ue8m0_pack_kernel(const float* __restrict__ a_scales, const float* __restrict__ b_scales,
+                                  int M, int num_kb, int n_chunks, int num_m, int num_n, int num_kg,
+                                  uint8_t* __restrict__ sf_a, uint8_t* __restrict__ sf_b) {
+  const int64_t w = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  const int64_t na = static_cast<int64_t>(num_m) * num_kg, nb = static_cast<int64_t>(num_n) * num_kg;
+  if (w < na) {
+    const int m_blk = static_cast<int>(w / num_kg), g = static_cast<int>(w % num_kg);
+    uint32_t word[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int row = m_blk * BM + j * 32 + lane;
+      uint32_t v = 0;
+#pragma unroll
+      for (int q = 0; q < SF_KB; ++q) {
+        const int kb = g * SF_KB + q;
+        const float sc = (row < M && kb < num_kb) ? a_scales[static_cast<size_t>(kb) * M + row] : 1.f;
+        v |= e8m0_byte(sc) << (8 * q);
+      }
+      word[j] = v;
+    }
+    reinterpret_cast<uint4*>(sf_a + w * SF_IMG_BYTES)[lane] = make_uint4(word[0], word[1], word[2], word[3]);
+  } else if (w < na + nb) {
+    const int64_t wb = w - na;
+    const int n_blk = static_cast<int>(wb / num_kg), g = static_cast<int>(wb % num_kg);
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int chunk = 2 * n_blk + h;
+      uint32_t v = 0;
+#pragma unroll
+      for (int q = 0; q < SF_KB; ++q) {
+        const int kb = g * SF_KB + q;
+        const float sc = (chunk < n_chunks && kb < num_kb) ? b_scales[static_cast<size_t>(chunk) * num_kb + kb] : 1.f;
+        v |= e8m0_byte(sc) << (8 * q);
+      }
+      reinterpret_cast<uint4*>(sf_b + (wb * 2 + h) * SF_IMG_BYTES)[lane] = make_uint4(v, v, v, v);
+    }
+  }
+}
+
 // Rows selected for dense dlogits are gathered (codes, scales, targets, lse,
 // grad) into a contiguous operand for the same GEMM kernel.
 __global__ void gather_rows_kernel(const uint8_t* __restrict__ h_codes,
@@ -553,7 +774,7 @@ __global__ void gather_rows_kernel(const uint8_t* __restrict__ h_codes,
       g_scales[i] = h_scales[t];
     }
   }
-  if (gran == kBlock) {
+  if (gran == kBlock || gran == kUe8m0) {
     const int64_t nkb = H / 128;
     for (int64_t kb = threadIdx.x; kb < nkb; kb += blockDim.x) g_scales[kb * n_rows + i] = h_scales[kb * T + t];
   }
@@ -621,11 +842,11 @@ cudaError_t launch_mode(const CUtensorMap& ta, const CUtensorMap& tb, const Para
         attr.numRegs * THREADS < 128 * CTRL_REGS + EPI_WARPS * 32 * EPI_REGS)
       return cudaErrorInvalidConfiguration;
     e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(SMEM_BYTES));
+                             static_cast<int>(smem_bytes<MODE>()));
     if (e != cudaSuccess) return e;
     configured_device = dev;
   }
-  kern<<<grid, THREADS, SMEM_BYTES, s>>>(ta, tb, p);
+  kern<<<grid, THREADS, smem_bytes<MODE>(), s>>>(ta, tb, p);
   return cudaGetLastError();
 }
 
@@ -665,6 +886,20 @@ cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s) {
   p.num_kb = static_cast<int>((a.K + bk_elems - 1) / bk_elems);
   p.n_chunks = static_cast<int>((a.N + CHUNK - 1) / CHUNK);
   p.wait_limit_ns = wait_limit_ns();
+  if (a.gran == kUe8m0) {
+    if (a.sf_images == nullptr || (reinterpret_cast<uintptr_t>(a.sf_images) & 15u) != 0)
+      return cudaErrorInvalidValue;
+    p.num_kg = (p.num_kb + SF_KB - 1) / SF_KB;
+    uint8_t* sf_a = a.sf_images;
+    uint8_t* sf_b = sf_a + static_cast<size_t>(p.num_m) * p.num_kg * SF_IMG_BYTES;
+    p.sf_a = sf_a;
+    p.sf_b = sf_b;
+    const int64_t warps = (static_cast<int64_t>(p.num_m) + p.num_n) * p.num_kg;
+    ue8m0_pack_kernel<<<static_cast<unsigned>((warps + 7) / 8), 256, 0, s>>>(
+        a.a_scales, a.b_scales, p.M, p.num_kb, p.n_chunks, p.num_m, p.num_n, p.num_kg, sf_a, sf_b);
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
   const int64_t tiles = static_cast<int64_t>(p.num_m) * p.num_n;
   const int grid = static_cast<int>(tiles < sm_count() ? tiles : sm_count());
   if constexpr (EPI == kEpiStore) {  // plain fp32 store: block-scaled FP8 (backward) or BF16
@@ -678,6 +913,7 @@ cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s) {
       case kTensor: return launch_mode<kTensor, EPI>(ta, tb, p, grid, s);
       case kRow: return launch_mode<kRow, EPI>(ta, tb, p, grid, s);
       case kBlock: return launch_mode<kBlock, EPI>(ta, tb, p, grid, s);
+      case kUe8m0: return launch_mode<kUe8m0, EPI>(ta, tb, p, grid, s);
       default: return cudaErrorInvalidValue;
     }
   } else {
@@ -685,6 +921,7 @@ cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s) {
       case kTensor: return launch_mode<kTensor, EPI>(ta, tb, p, grid, s);
       case kRow: return launch_mode<kRow, EPI>(ta, tb, p, grid, s);
       case kBf16: return launch_mode<kBf16, EPI>(ta, tb, p, grid, s);
+      case kUe8m0: return launch_mode<kUe8m0, EPI>(ta, tb, p, grid, s);
       default: return launch_mode<kBlock, EPI>(ta, tb, p, grid, s);
     }
   }
@@ -698,6 +935,13 @@ int blocks_for(int64_t n, int threads) {
 }  // namespace
 
 int64_t gemm_partials_per_token(int64_t N) { return (N + CHUNK - 1) / CHUNK; }
+
+size_t gemm_ue8m0_image_bytes(int64_t M, int64_t N, int64_t K) {
+  if (M < 1 || N < 1 || K < 1) return 0;
+  const int64_t num_m = (M + BM - 1) / BM, num_n = (N + BN - 1) / BN;
+  const int64_t num_kg = ((K + BK - 1) / BK + SF_KB - 1) / SF_KB;
+  return align_up(static_cast<size_t>((num_m + 2 * num_n) * num_kg) * SF_IMG_BYTES, 256);
+}
 
 cudaError_t launch_gemm_lse(const GemmArgs& a, cudaStream_t s) { return launch_gemm<kEpiLse>(a, s); }
 

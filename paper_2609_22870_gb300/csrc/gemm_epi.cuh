@@ -13,7 +13,13 @@ namespace {
 constexpr int CHUNK = 128;        // vocabulary columns per LSE partial
 constexpr float kLog2e = 1.4426950408889634f;
 
-enum { kTensor = FP8RL_GRAN_TENSOR, kRow = FP8RL_GRAN_ROWWISE, kBlock = FP8RL_GRAN_BLOCK, kBf16 = 3 };
+enum {
+  kTensor = FP8RL_GRAN_TENSOR,
+  kRow = FP8RL_GRAN_ROWWISE,
+  kBlock = FP8RL_GRAN_BLOCK,
+  kUe8m0 = FP8RL_GRAN_BLOCK_UE8M0,  // block layout, power-of-two scales applied by the MMA
+  kBf16 = 16
+};
 static_assert(kBf16 == kGemmBf16, "BF16 mode id shared with the host interface");
 // Epilogues: streaming LSE partials + target logit; dense dlogits rows (fp32);
 // dlogits of every token E4M3-quantised in both orientations, the A operands
@@ -42,6 +48,9 @@ struct Params {
   int num_m, num_n, num_kb;
   int band_m;  // row blocks per band of the tile order
   int n_chunks;
+  const uint8_t* sf_a;  // UE8M0 mode: E8M0 scale images [num_m][num_kg][512 B]
+  const uint8_t* sf_b;  //   [num_n][num_kg][1024 B]
+  int num_kg;           //   groups of four K blocks
   uint64_t wait_limit_ns;
 };
 

@@ -48,12 +48,18 @@ struct GemmArgs {
   float* c_out;             // [M][ld_c], 16-byte aligned, ld_c % 4 == 0
   int64_t ld_c;
   int accumulate;           // add to c_out instead of overwriting it
+  // FP8RL_GRAN_BLOCK_UE8M0: device scratch of gemm_ue8m0_image_bytes(M, N, K)
+  // bytes (16-byte aligned) for the E8M0 scale-factor images
+  uint8_t* sf_images;
 };
-constexpr int kGemmBf16 = 3;
+constexpr int kGemmBf16 = 16;  // internal mode id, outside fp8rl_gran
 
 // LSE partials the GEMM leaves per token (one per column slot of each
 // 256-wide vocabulary tile).
 int64_t gemm_partials_per_token(int64_t N);
+// Scratch the GEMM needs for the E8M0 scale-factor images of the UE8M0 mode
+// (a multiple of 256 bytes).
+size_t gemm_ue8m0_image_bytes(int64_t M, int64_t N, int64_t K);
 cudaError_t launch_gemm_lse(const GemmArgs& a, cudaStream_t s);
 cudaError_t launch_gemm_dlogits(const GemmArgs& a, cudaStream_t s);
 cudaError_t launch_gemm_dense_dlogits(const GemmArgs& a, cudaStream_t s);
@@ -61,8 +67,8 @@ cudaError_t launch_gemm_store(const GemmArgs& a, cudaStream_t s);
 struct BwdLayout {
   int64_t vp, tp;  // V and T rounded up to multiples of 128 (the K extents)
   // byte offsets in the workspace: codes and scales of P [T][vp], P^T [V][tp],
-  // W^T [H][vp], h^T [H][tp]
-  size_t p, ps, pt, pts, wt, wts, ht, hts, total;
+  // W^T [H][vp], h^T [H][tp]; E8M0 scale images of the UE8M0 recompute
+  size_t p, ps, pt, pts, wt, wts, ht, hts, sf, total;
 };
 BwdLayout bwd_layout(int64_t T, int64_t H, int64_t V);
 cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const uint8_t* wc,
