@@ -586,8 +586,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                                   lim, abort_flag);
           if (!ok) break;
         } else {
-#pragma unroll
-          for (int c = 0; c < CHUNK / 32; ++c) epi_consume32<EPI>(p, es, z + c * 32, row, col0, c * 32);
+          epi_consume128<EPI>(p, es, z, row, col0);
         }
       } else if (MODE == kUe8m0) {
         // scales already applied by the MMA: all 128 columns into registers,
@@ -609,8 +608,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                                   lim, abort_flag);
           if (!ok) break;
         } else {
-#pragma unroll
-          for (int c = 0; c < CHUNK / 32; ++c) epi_consume32<EPI>(p, es, zf + c * 32, row, col0, c * 32);
+          epi_consume128<EPI>(p, es, zf, row, col0);
         }
       } else if (EPI == kEpiDenseFp8) {
         // tensor / row scaling: all 128 scaled columns into registers, buffer

@@ -147,6 +147,39 @@ __device__ __forceinline__ void epi_consume32(const Params& p, EpiState& e, cons
   }
 }
 
+// All 128 columns of a thread at once (block and UE8M0 scaling, which hold the
+// whole row of the tile half in registers): the same (max, sum exp) and z_y as
+// four epi_consume32 calls, with one maximum and one rescale instead of four
+// and no per-column bounds tests when the whole chunk lies inside [0, N).
+template <int EPI>
+__device__ __forceinline__ void epi_consume128(const Params& p, EpiState& e, const float* z, int row, int col0) {
+  if (EPI != kEpiLse || p.N - col0 < CHUNK || row >= p.M) {
+#pragma unroll
+    for (int c = 0; c < CHUNK / 32; ++c) epi_consume32<EPI>(p, e, z + c * 32, row, col0, c * 32);
+    return;
+  }
+  float m4[4] = {z[0], z[1], z[2], z[3]};
+#pragma unroll
+  for (int i = 4; i < CHUNK; i += 4) {
+    m4[0] = fmaxf(m4[0], z[i]);
+    m4[1] = fmaxf(m4[1], z[i + 1]);
+    m4[2] = fmaxf(m4[2], z[i + 2]);
+    m4[3] = fmaxf(m4[3], z[i + 3]);
+  }
+  const float mn = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+  const float mb = mn * kLog2e;
+  float a4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int i = 0; i < CHUNK; ++i) a4[i & 3] += exp2f(fmaf(z[i], kLog2e, -mb));
+  e.s = (a4[0] + a4[1]) + (a4[2] + a4[3]);
+  e.m = mn;
+  if (e.j >= 0 && e.j < CHUNK) {
+#pragma unroll
+    for (int i = 0; i < CHUNK; ++i)
+      if (i == e.j) e.zy = z[i];
+  }
+}
+
 template <int EPI>
 __device__ __forceinline__ void epi_finish(const Params& p, const EpiState& e, int row, int chunk) {
   if (EPI != kEpiLse || row >= p.M || chunk >= p.n_chunks) return;
