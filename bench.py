@@ -276,30 +276,34 @@ def run_ours(args, rank, world, local_rank):
 
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(7)]
 
-    def step(record=False):
-        if record:
-            ev[0].record(stream)
-        api.quantize(h, gran, api.ROLE_ACT, b.h_codes, b.h_scales, b.q_ws)
-        if record:
-            ev[1].record(stream)
-        api.quantize(W, gran, api.ROLE_WEIGHT, b.w_codes, b.w_scales, b.q_ws)
-        if record:
-            ev[2].record(stream)
-        api.logit_partials(b.h_codes, b.h_scales, b.w_codes, b.w_scales, gran, y, b.lp_ws)
-        if record:
-            ev[3].record(stream)
-        api.combine_logprobs(T, H, V, gran, y, b.lp_ws, logp_old, b.logp, b.lse, b.ratio)
-        if record:
-            ev[4].record(stream)
-        api.calibrate_clip_bounds(b.ratio, r_bf16, adv_d, mask_d, coef, w.eps_low, w.eps_high, opts,
-                                  b.cal_res, b.cal_ws)
-        if record:
-            ev[5].record(stream)
-        api.clipped_surrogate(b.ratio, adv_d, mask_d, None, bounds=api.bounds_view(b.cal_res),
-                              stats=b.stats, workspace=b.sur_ws,
-                              out={"grad": b.grad, "clip_mask": b.clip_mask})
-        if record:
-            ev[6].record(stream)
+    def make_step(g, bb):
+        def step(record=False):
+            if record:
+                ev[0].record(stream)
+            api.quantize(h, g, api.ROLE_ACT, bb.h_codes, bb.h_scales, bb.q_ws)
+            if record:
+                ev[1].record(stream)
+            api.quantize(W, g, api.ROLE_WEIGHT, bb.w_codes, bb.w_scales, bb.q_ws)
+            if record:
+                ev[2].record(stream)
+            api.logit_partials(bb.h_codes, bb.h_scales, bb.w_codes, bb.w_scales, g, y, bb.lp_ws)
+            if record:
+                ev[3].record(stream)
+            api.combine_logprobs(T, H, V, g, y, bb.lp_ws, logp_old, bb.logp, bb.lse, bb.ratio)
+            if record:
+                ev[4].record(stream)
+            api.calibrate_clip_bounds(bb.ratio, r_bf16, adv_d, mask_d, coef, w.eps_low, w.eps_high, opts,
+                                      bb.cal_res, bb.cal_ws)
+            if record:
+                ev[5].record(stream)
+            api.clipped_surrogate(bb.ratio, adv_d, mask_d, None, bounds=api.bounds_view(bb.cal_res),
+                                  stats=bb.stats, workspace=bb.sur_ws,
+                                  out={"grad": bb.grad, "clip_mask": bb.clip_mask})
+            if record:
+                ev[6].record(stream)
+        return step
+
+    step = make_step(gran, b)
 
     for _ in range(args.warmup):
         step()
@@ -336,6 +340,35 @@ def run_ours(args, rank, world, local_rank):
         for _ in range(n_more):
             step()
         torch.cuda.synchronize()
+
+    # the same step with power-of-two block scales applied by the tensor
+    # cores' block-scaled MMA (a variant outside the paper; block layout only)
+    ue = None
+    if gran == api.GRAN_BLOCK and not args.no_variants:
+        b3 = api.StepBuffers(T, H, V, api.GRAN_BLOCK_UE8M0, dev)
+        step3 = make_step(api.GRAN_BLOCK_UE8M0, b3)
+        for _ in range(args.warmup):
+            step3()
+        torch.cuda.synchronize()
+        u0 = torch.cuda.Event(enable_timing=True)
+        u1 = torch.cuda.Event(enable_timing=True)
+        ue_events = []
+        with clocks.active():
+            u0.record(stream)
+            for _ in range(args.steps):
+                ev[:] = [torch.cuda.Event(enable_timing=True) for _ in range(7)]
+                step3(record=True)
+                ue_events.append(list(ev))
+            u1.record(stream)
+            torch.cuda.synchronize()
+        api.check()
+        ue_stage = np.zeros(6)
+        for evs in ue_events:
+            ue_stage += [evs[i].elapsed_time(evs[i + 1]) for i in range(6)]
+        ue_stage /= args.steps
+        ue = {"ms_per_step": u0.elapsed_time(u1) / args.steps, "gemm_ms": ue_stage[2],
+              "quantize_ms": ue_stage[0] + ue_stage[1]}
+        del b3
 
     # the BF16 shadow pass on its own (same inputs; the paper reruns it every
     # 20 steps, so it is reported separately and amortised)
@@ -498,6 +531,15 @@ def run_ours(args, rank, world, local_rank):
                                              "clipped_hi_fp8", "clipped_lo_bf16", "clipped_hi_bf16",
                                              "nmae_prob", "nmae_ratio")},
     }
+    if ue is not None:
+        ue_tf = flops / (ue["gemm_ms"] * 1e-3) / 1e12
+        line["ue8m0_mma_variant"] = {
+            "value": whole_job_rate(T, 1, ue["ms_per_step"]), "unit": "tokens/s",
+            "ms_per_step": ue["ms_per_step"], "gemm_ms": ue["gemm_ms"], "quantize_ms": ue["quantize_ms"],
+            "gemm_tflops": ue_tf, "gemm_frac_of_fp8_peak": ue_tf / fp8_peak,
+            "note": "the same step with power-of-two block scales (fp8rl_quantize_ue8m0, 1x128 / 128x128) "
+                    "applied by tcgen05.mma kind::mxf8f6f4 with E8M0 scale factors in tensor memory; a "
+                    "variant outside the paper (its scales are amax / 448), so not the headline value"}
     if bwd is not None:
         ideal_ms = 3 * flops / (fp8_peak * 1e12) * 1e3
         bwd.update({"tflop_per_call": 3 * flops / 1e12, "tflops": 3 * flops / (bwd["ms"] * 1e-3) / 1e12,
@@ -789,6 +831,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-backward", action="store_true", help="skip timing the lm_head backward")
     ap.add_argument("--no-fp8-peak", action="store_true", help="skip measuring the vendor FP8 GEMM rate")
+    ap.add_argument("--no-variants", action="store_true",
+                    help="skip timing the step with power-of-two scales on the block-scaled MMA")
     ap.add_argument("--kernels", action="store_true",
                     help="print HBM rooflines of the memory-bound kernels at stress sizes instead")
     ap.add_argument("--stress-scale", type=float, default=1.0,

@@ -184,6 +184,8 @@ def quantize(x, gran, role=ROLE_ACT, codes=None, scales=None, workspace=None, st
     with ``ue8m0`` fp8rl_quantize_ue8m0 (power-of-two scales)."""
     if x.dim() != 2 or x.dtype != torch.bfloat16 or not x.is_cuda or x.stride(1) != 1:
         raise ValueError("x: expected a 2-D CUDA bf16 tensor with unit column stride")
+    if gran == GRAN_BLOCK_UE8M0:  # the block layout with power-of-two scales
+        gran, ue8m0 = GRAN_BLOCK, True
     rows, cols = x.shape
     n = scales_count(rows, cols, gran, role)
     codes = torch.empty(rows, cols, dtype=torch.uint8, device=x.device) if codes is None else codes

@@ -118,3 +118,24 @@ def test_ue8m0_mma_rejects_scales_that_are_not_powers_of_two(cuda_lib):
     api.token_logprobs(hc, hs, wc, ws, UE, y)
     assert api.check_status() == api.EDEVICE
     api.check()
+
+
+def test_ue8m0_mma_step_through_the_binding(cuda_lib):
+    """score_calibrate_loss with the UE8M0 granularity: the binding quantises
+    with power-of-two block scales and the scoring runs on the block-scaled
+    MMA; log-probs against the oracle's power-of-two path."""
+    api = cuda_lib
+    T, H, V = 640, 512, 3000
+    h, W, y = _data(T, H, V, 97)
+    g = torch.Generator().manual_seed(98)
+    logp_old = (torch.randn(T, generator=g) * 0.01 - 8.0).float().cuda()
+    r_bf16 = torch.exp(torch.randn(T, generator=g) * 0.01).float().cuda()
+    adv = torch.randn(T, generator=g).float().cuda()
+    mask = torch.ones(T, dtype=torch.uint8, device="cuda")
+    coef = torch.ones(T, dtype=torch.float32, device="cuda")
+    b = api.score_calibrate_loss(h, W, y, logp_old, r_bf16, adv, mask, coef, UE, 0.2, 0.2)
+    api.check()
+    ref_lp, _, _ = oracle_logprobs_rows(h, W, OQ.BLOCK, y, np.arange(T), pow2=True)
+    assert np.max(np.abs(b.logp.cpu().numpy() - ref_lp)) <= TOL
+    hc, hs = api.quantize(h, api.GRAN_BLOCK, api.ROLE_ACT, ue8m0=True)
+    assert torch.equal(b.h_codes, hc) and torch.equal(b.h_scales[:hs.numel()], hs)
