@@ -300,19 +300,6 @@ __device__ __forceinline__ void tmem_ld_32x32b_x64(uint32_t taddr, float (&v)[64
   for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-// (a0, a1) = (x0, x1) * s + (a0, a1): one packed two-lane FMA.
-__device__ __forceinline__ void ffma2(float& a0, float& a1, float x0, float x1, float s) {
-  asm(
-      "{\n\t.reg .b64 x, c, sc, d;\n\t"
-      "mov.b64 x, {%2, %3};\n\t"
-      "mov.b64 c, {%0, %1};\n\t"
-      "mov.b64 sc, {%4, %4};\n\t"
-      "fma.rn.f32x2 d, x, sc, c;\n\t"
-      "mov.b64 {%0, %1}, d;\n\t}"
-      : "+f"(a0), "+f"(a1)
-      : "f"(x0), "f"(x1), "f"(s));
-}
-
 // Register budget of a warpgroup (all four warps execute it together).
 template <uint32_t N>
 __device__ __forceinline__ void warpgroup_reg_dealloc() {

@@ -26,8 +26,12 @@
 // stage, so the shared-memory layout is the FP8 one) and no scales.  Block scales (1x128 for h,
 // 128x128 for W) change every 128-wide K block: the MMA writes each K block's
 // partial product into one of the two TMEM buffers and the epilogue promotes
-// it, acc += S_h[t][kb] S_W[vb][kb] * partial, into registers (packed f32x2
-// FMAs) while the MMA fills the other buffer.
+// it, acc += S_h[t][kb] S_W[vb][kb] * partial, into registers while the MMA
+// fills the other buffer.
+// Power-of-two block scales (the UE8M0 variant) go to the tensor cores instead:
+// tcgen05.mma kind::mxf8f6f4 multiplies each 32-wide K step by E8M0 scale
+// factors it reads from TMEM, so one accumulator runs over the whole K and the
+// epilogue only reads it once per tile.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -187,9 +191,17 @@ __device__ __forceinline__ void encode128(const float* v, float s, uint32_t (&w)
 // S = fl32(amax / 448), 1 for an all-zero block (NaN amax gives NaN).
 __device__ __forceinline__ float scale_of(float amax) { return amax == 0.f ? 1.f : __fdiv_rn(amax, kE4M3Max); }
 
+// max that propagates NaN (a NaN block maximum marks the block's scale NaN).
+__device__ __forceinline__ float fmax_nan(float a, float b) {
+  float r;
+  asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
+  return r;
+}
+
 // Dense dLoss/dz of one thread's 128 columns (row `row`, columns col0 ..
 // col0 + 127; z the scaled logits), quantised for the FP8 backward:
-//   P[t][v] = g_t (1{v == y_t} - exp(z[t][v] - lse_t))   (float32)
+//   P[t][v] = g_t (1{v == y_t} - exp(z[t][v] - lse_t))   (float32, the
+//   exponential as exp2(z log2(e) - lse log2(e)) with one fused multiply-add)
 //   codes of P with this row's 1x128 block scale        -> pq_out / pq_scales
 //   codes of P with the 128 x 128 block scale of the tile half (the max over
 //   the four warps holding its 128 rows, exchanged through shared memory
@@ -202,17 +214,27 @@ __device__ __forceinline__ bool dense_fp8_epilogue(const Params& p, const EpiSta
                                                    uint64_t lim, const volatile int* abort_flag) {
   const int ncol = min(CHUNK, p.N - col0);
   const bool row_ok = row < p.M;
-  const float l = row_ok ? p.lse[row] : 0.f, g = row_ok ? p.grad[row] : 0.f;
+  const float g = es.g;
+  const float lb = es.l * kLog2e;
   float amax = 0.f;
-  bool nan = false;
+  const bool here = es.j >= 0 && es.j < CHUNK;
+  if (__all_sync(0xffffffffu, row_ok && !here) && ncol == CHUNK) {
+    // the common case: every row of the warp valid, no target column here
+    const float ng = -g;
 #pragma unroll
-  for (int i = 0; i < CHUNK; ++i) {
-    const float v = (row_ok && i < ncol) ? g * ((i == es.j ? 1.f : 0.f) - expf(z[i] - l)) : 0.f;
-    z[i] = v;
-    amax = fmaxf(amax, fabsf(v));
-    nan |= v != v;
+    for (int i = 0; i < CHUNK; ++i) {
+      const float v = ng * exp2f(fmaf(z[i], kLog2e, -lb));
+      z[i] = v;
+      amax = fmax_nan(amax, fabsf(v));
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < CHUNK; ++i) {
+      const float v = (row_ok && i < ncol) ? g * ((i == es.j ? 1.f : 0.f) - exp2f(fmaf(z[i], kLog2e, -lb))) : 0.f;
+      z[i] = v;
+      amax = fmax_nan(amax, fabsf(v));
+    }
   }
-  if (nan) amax = __uint_as_float(0x7FC00000u);
   uint32_t w[32];
   if (row_ok && col0 < p.ld_pq) {  // the row's block along N (K of the dh contraction)
     const float s = scale_of(amax);
@@ -238,11 +260,24 @@ __device__ __forceinline__ bool dense_fp8_epilogue(const Params& p, const EpiSta
   if (ncol <= 0) return true;
   const float sb = scale_of(__uint_as_float(bmax));
   encode128(z, sb, w);
-  // lanes are consecutive tokens: each column of P^T gets 32 contiguous bytes
-  uint8_t* dst = p.ptq_out + static_cast<size_t>(col0) * p.ld_ptq + row;
+  // lanes are consecutive tokens; a 4 x 4 byte transpose within each group of
+  // four lanes (two exchanges) leaves lane 4a + j with column 4k + j of rows
+  // 4a .. 4a + 3, so each store writes four bytes and each column of P^T gets
+  // 32 contiguous bytes per warp
+  const int j = lane & 3;
+  const size_t ld = static_cast<size_t>(p.ld_ptq);
+  uint8_t* dst = p.ptq_out + static_cast<size_t>(col0 + j) * ld + (row - j);
 #pragma unroll
-  for (int i = 0; i < CHUNK; ++i)
-    if (i < ncol) dst[static_cast<size_t>(i) * p.ld_ptq] = static_cast<uint8_t>(w[i >> 2] >> (8 * (i & 3)));
+  for (int k = 0; k < CHUNK / 4; ++k) {
+    // round 1 (lanes j, j ^ 1): even lanes keep bytes 0, 2 and take the
+    // partner's; odd lanes keep 1, 3
+    const uint32_t o1 = __shfl_xor_sync(0xffffffffu, w[k], 1);
+    const uint32_t r1 = (j & 1) ? __byte_perm(o1, w[k], 0x7351) : __byte_perm(w[k], o1, 0x6240);
+    // round 2 (lanes j, j ^ 2): lanes 0, 1 keep their low halves
+    const uint32_t o2 = __shfl_xor_sync(0xffffffffu, r1, 2);
+    const uint32_t t = (j & 2) ? __byte_perm(o2, r1, 0x7632) : __byte_perm(r1, o2, 0x5410);
+    if (4 * k + j < ncol) *reinterpret_cast<uint32_t*>(dst + static_cast<size_t>(4 * k) * ld) = t;
+  }
   if (rit < ncol) p.ptq_scales[static_cast<size_t>(m_blk) * p.N + col0 + rit] = sb;
   return true;
 }
@@ -572,8 +607,11 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
 #pragma unroll
             for (int i = 0; i < 16; ++i)
-              ffma2(z2[c * 16 + i].x, z2[c * 16 + i].y, __uint_as_float(cur[2 * i]),
-                    __uint_as_float(cur[2 * i + 1]), sc);
+            {
+              // scalar FMAs: the packed f32x2 form measured no faster here
+              z2[c * 16 + i].x = fmaf(__uint_as_float(cur[2 * i]), sc, z2[c * 16 + i].x);
+              z2[c * 16 + i].y = fmaf(__uint_as_float(cur[2 * i + 1]), sc, z2[c * 16 + i].y);
+            }
             if (c + 1 < CHUNK / 32) tmem_wait_ld(nxt);
           }
           ab ^= 1;

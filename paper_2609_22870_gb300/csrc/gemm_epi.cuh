@@ -77,7 +77,8 @@ __device__ __forceinline__ void tile_coords(int tile, const Params& p, int& m_bl
 // [col0, col0 + 128) consumed 32 at a time (values already scaled).
 struct EpiState {
   float m, s, zy;
-  int j;  // target column relative to col0 (outside [0, 128): not here)
+  int j;     // target column relative to col0 (outside [0, 128): not here)
+  float l, g;  // dense dlogits epilogue: lse and dLoss/dlogp of the row
 };
 
 template <int EPI>
@@ -86,9 +87,16 @@ __device__ __forceinline__ void epi_begin(const Params& p, EpiState& e, int row,
   e.s = 0.f;
   e.zy = 0.f;
   e.j = -1;
+  e.l = 0.f;
+  e.g = 0.f;
   if (EPI != kEpiStore && row < p.M) {
     const int y = p.targets[row];
     if (y >= 0 && y < p.N) e.j = y - col0;
+  }
+  // loaded when the tile starts, so their latency hides behind its K loop
+  if (EPI == kEpiDenseFp8 && row < p.M) {
+    e.l = p.lse[row];
+    e.g = p.grad[row];
   }
 }
 
