@@ -74,7 +74,17 @@ __global__ void __launch_bounds__(kThreads) count_valid_kernel(const uint8_t* __
   uint32_t n = 0;
   const bool vec = (reinterpret_cast<uintptr_t>(mask) & 15) == 0;
   const int64_t T16 = vec ? T / 16 : 0;
-  for (int64_t i = tid; i < T16; i += stride) {
+  int64_t i = tid;
+  // four 16-byte loads in flight per thread, then the remainder one at a time
+  for (; i + 3 * stride < T16; i += 4 * stride) {
+    uint4 v[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) v[u] = __ldg(reinterpret_cast<const uint4*>(mask) + i + u * stride);
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+      n += nonzero_bytes(v[u].x) + nonzero_bytes(v[u].y) + nonzero_bytes(v[u].z) + nonzero_bytes(v[u].w);
+  }
+  for (; i < T16; i += stride) {
     const uint4 v = __ldg(reinterpret_cast<const uint4*>(mask) + i);
     n += nonzero_bytes(v.x) + nonzero_bytes(v.y) + nonzero_bytes(v.z) + nonzero_bytes(v.w);
   }
@@ -420,38 +430,8 @@ __global__ void __launch_bounds__(kThreads) seq_accum_kernel(
     acc_q = 0;
     acc_n = 0;
   };
-  for (int64_t base = beg; base < end; base += 128) {
-    const int64_t t0 = base + 4 * lane;
-    int id[4];
-    float lp[4], lo[4];
-    bool on[4];
-    if (VEC && t0 + 3 < end) {
-      const int4 iv = __ldg(reinterpret_cast<const int4*>(sid + t0));
-      const uint32_t mv = mask ? __ldg(reinterpret_cast<const uint32_t*>(mask + t0)) : 0x01010101u;
-      id[0] = iv.x, id[1] = iv.y, id[2] = iv.z, id[3] = iv.w;
-      if (SUMS) {
-        const float4 a = __ldg(reinterpret_cast<const float4*>(logp + t0));
-        const float4 b = __ldg(reinterpret_cast<const float4*>(logp_old + t0));
-        lp[0] = a.x, lp[1] = a.y, lp[2] = a.z, lp[3] = a.w;
-        lo[0] = b.x, lo[1] = b.y, lo[2] = b.z, lo[3] = b.w;
-      } else {
-#pragma unroll
-        for (int k = 0; k < 4; ++k) lp[k] = lo[k] = 0.f;
-      }
-#pragma unroll
-      for (int k = 0; k < 4; ++k) on[k] = ((mv >> (8 * k)) & 0xFFu) != 0;
-    } else {
-#pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const int64_t t = t0 + k;
-        const bool in = t < end;
-        id[k] = in ? __ldg(sid + t) : 0;
-        lp[k] = SUMS && in ? __ldg(logp + t) : 0.f;
-        lo[k] = SUMS && in ? __ldg(logp_old + t) : 0.f;
-        on[k] = in && (!mask || __ldg(mask + t) != 0);
-        if (!in) id[k] = cur;  // past the end: nothing to add
-      }
-    }
+  // one 128-token step (four consecutive tokens a lane), after its loads
+  auto step = [&](const int (&id)[4], const float (&lp)[4], const float (&lo)[4], const bool (&on)[4], int64_t t0) {
     long long q[4];
     bool v[4];
     bool match = true;
@@ -476,7 +456,7 @@ __global__ void __launch_bounds__(kThreads) seq_accum_kernel(
         acc_q += q[k];
         acc_n += v[k];
       }
-      continue;
+      return;
     }
     // a boundary: finish the current sequence with this step's tokens of it
 #pragma unroll
@@ -508,6 +488,56 @@ __global__ void __launch_bounds__(kThreads) seq_accum_kernel(
         s_new += atomicAdd(&cnt[id[k]], 1u) == 0u;
         if (SUMS) atomicAdd(&qsum[id[k]], static_cast<unsigned long long>(q[k]));
       }
+  };
+  auto load_vec = [&](int64_t t0, int (&id)[4], float (&lp)[4], float (&lo)[4], bool (&on)[4]) {
+    const int4 iv = __ldg(reinterpret_cast<const int4*>(sid + t0));
+    const uint32_t mv = mask ? __ldg(reinterpret_cast<const uint32_t*>(mask + t0)) : 0x01010101u;
+    id[0] = iv.x, id[1] = iv.y, id[2] = iv.z, id[3] = iv.w;
+    if (SUMS) {
+      const float4 a = __ldg(reinterpret_cast<const float4*>(logp + t0));
+      const float4 b = __ldg(reinterpret_cast<const float4*>(logp_old + t0));
+      lp[0] = a.x, lp[1] = a.y, lp[2] = a.z, lp[3] = a.w;
+      lo[0] = b.x, lo[1] = b.y, lo[2] = b.z, lo[3] = b.w;
+    } else {
+#pragma unroll
+      for (int k = 0; k < 4; ++k) lp[k] = lo[k] = 0.f;
+    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k) on[k] = ((mv >> (8 * k)) & 0xFFu) != 0;
+  };
+  int64_t base = beg;
+  // two full steps' loads in flight before either is processed
+  if (VEC) {
+    for (; base + 255 < end; base += 256) {
+      int idA[4], idB[4];
+      float lpA[4], loA[4], lpB[4], loB[4];
+      bool onA[4], onB[4];
+      load_vec(base + 4 * lane, idA, lpA, loA, onA);
+      load_vec(base + 128 + 4 * lane, idB, lpB, loB, onB);
+      step(idA, lpA, loA, onA, base + 4 * lane);
+      step(idB, lpB, loB, onB, base + 128 + 4 * lane);
+    }
+  }
+  for (; base < end; base += 128) {
+    const int64_t t0 = base + 4 * lane;
+    int id[4];
+    float lp[4], lo[4];
+    bool on[4];
+    if (VEC && t0 + 3 < end) {
+      load_vec(t0, id, lp, lo, on);
+    } else {
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int64_t t = t0 + k;
+        const bool in = t < end;
+        id[k] = in ? __ldg(sid + t) : 0;
+        lp[k] = SUMS && in ? __ldg(logp + t) : 0.f;
+        lo[k] = SUMS && in ? __ldg(logp_old + t) : 0.f;
+        on[k] = in && (!mask || __ldg(mask + t) != 0);
+        if (!in) id[k] = cur;  // past the end: nothing to add
+      }
+    }
+    step(id, lp, lo, on, t0);
   }
   flush();
   if (__any_sync(0xffffffffu, bad) && lane == 0) atomicOr(&d_status, kErrDevice);

@@ -51,17 +51,37 @@ __device__ __forceinline__ void bar_sync(uint32_t id, uint32_t n) {
 }
 
 // ---------------------------------------------------------------- tensor
+// The per-tensor kernels walk the tensor as vectors of 8 bf16 (16 bytes):
+// vector i sits at row i / vpr, column (i % vpr) * 8.  A contiguous tensor
+// (ld == cols) is one linear array, read without that division; otherwise
+// each thread carries its (row, column) and steps it by the grid stride.
+// Four vectors per thread and step keep 64 bytes in flight per thread.
+struct VecWalk {
+  const uint16_t* x;
+  int64_t vpr, ld;
+  __device__ __forceinline__ int64_t offset(int64_t i) const {
+    if (ld == vpr * 8) return i * 8;
+    const int64_t r = i / vpr;
+    return r * ld + (i - r * vpr) * 8;
+  }
+};
+
 // Global amax over the tensor, as float bits (atomicMax on the bits).
 __global__ void amax_kernel(const uint16_t* __restrict__ x, int64_t rows, int64_t cols, int64_t ld,
                             unsigned int* __restrict__ amax) {
-  const int64_t vpr = cols / 8;
-  const int64_t nvec = rows * vpr;
+  const VecWalk vw{x, cols / 8, ld};
+  const int64_t nvec = rows * vw.vpr;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   uint32_t m = 0;
-  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < nvec;
-       i += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t r = i / vpr, c = (i - r * vpr) * 8;
-    m = amax_bf16x8(m, __ldg(reinterpret_cast<const uint4*>(x + r * ld + c)));
+  int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
+  for (; i + 3 * stride < nvec; i += 4 * stride) {
+    uint4 v[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) v[u] = __ldg(reinterpret_cast<const uint4*>(x + vw.offset(i + u * stride)));
+#pragma unroll
+    for (int u = 0; u < 4; ++u) m = amax_bf16x8(m, v[u]);
   }
+  for (; i < nvec; i += stride) m = amax_bf16x8(m, __ldg(reinterpret_cast<const uint4*>(x + vw.offset(i))));
   const uint32_t b = __reduce_max_sync(0xffffffffu, amax_bits(m));
   if ((threadIdx.x & 31) == 0) {
     if (b >= kInfBits) flag_bad();
@@ -76,14 +96,20 @@ __global__ void quant_tensor_kernel(const uint16_t* __restrict__ x, int64_t rows
   const float s = e4m3_scale(__uint_as_float(*amax), pow2);
   const E4M3Enc e = e4m3_encoder(s);
   if (blockIdx.x == 0 && threadIdx.x == 0) scales[0] = s;
-  const int64_t vpr = cols / 8;
-  const int64_t nvec = rows * vpr;
-  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < nvec;
-       i += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t r = i / vpr, c = (i - r * vpr) * 8;
-    const uint4 v = __ldg(reinterpret_cast<const uint4*>(x + r * ld + c));
-    *reinterpret_cast<uint2*>(codes + r * cols + c) = e4m3_encode8(v, e);
+  const VecWalk vw{x, cols / 8, ld};
+  const int64_t nvec = rows * vw.vpr;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
+  // codes are [rows][cols] contiguous: vector i's codes start at byte i * 8
+  for (; i + 3 * stride < nvec; i += 4 * stride) {
+    uint4 v[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) v[u] = __ldg(reinterpret_cast<const uint4*>(x + vw.offset(i + u * stride)));
+#pragma unroll
+    for (int u = 0; u < 4; ++u) *reinterpret_cast<uint2*>(codes + (i + u * stride) * 8) = e4m3_encode8(v[u], e);
   }
+  for (; i < nvec; i += stride)
+    *reinterpret_cast<uint2*>(codes + i * 8) = e4m3_encode8(__ldg(reinterpret_cast<const uint4*>(x + vw.offset(i))), e);
 }
 
 // ---------------------------------------------------------------- row
