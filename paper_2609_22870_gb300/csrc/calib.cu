@@ -61,6 +61,13 @@ struct State {
   unsigned int nb_mpiece;  // L: min{key > key(lo_min)}   H: min{key >= key(hi_min), q > 0}
   unsigned int nb_Mpiece1; // L: 1 + max{key <= key(lo_max)}   H: 1 + max{key < key(hi_max), q > 0}
   unsigned int pad0;
+  // EXACT mode selects only among the ratios inside the search interval (the
+  // others cannot move a bound inside it): the radix histograms count A<0
+  // tokens with lo_min <= r_fp8 <= lo_max and weigh A>0 tokens with
+  // hi_min <= r_fp8 < hi_max; what lies below enters the select as `below`
+  unsigned long long l_below;  // #{A<0 : r_fp8 < lo_min}
+  unsigned long long l_in;     // #{A<0 : lo_min <= r_fp8 <= lo_max}
+  unsigned long long h_below;  // sum_{A>0, r_fp8 < hi_min} q_fp8 (int64 two's complement)
   // written by decide steps
   int shift;
   int found;
@@ -261,6 +268,8 @@ struct PassAcc {
   unsigned long long n_neg, n_pos, k_bf, k_fp;
   long long s_pos_bf, s_neg_bf, s_neg_fp, s_pos_fp;
   unsigned emax, bad, nb_below1, nb_above, nb_m, nb_M1;
+  unsigned l_below, l_in;  // per-thread counts: T / grid threads each at most
+  long long h_below;
 };
 
 // Constants of one pass.
@@ -273,12 +282,13 @@ struct PassCtx {
 
 // One token of a pass: updates the thread's scalars and returns the
 // histogram bin the token adds `w` to (-1: none).
+template <int STAGE>
 __device__ __forceinline__ int pass_token(const Args& a, const PassCtx& x, const float* sh_cand,
                                           bool valid, float A, float rf, float rb, float c,
                                           PassAcc& acc, long long& w) {
   w = 0;
   const bool neg = valid && A < 0.f, pos = valid && A > 0.f;
-  if (x.stage == kPrep) {
+  if (STAGE == kPrep) {
     if (!(isfinite(A) && isfinite(rf) && isfinite(rb) && isfinite(c)) || rf < 0.f || rb < 0.f ||
         c < 0.f)
       acc.bad = 1;
@@ -295,9 +305,17 @@ __device__ __forceinline__ int pass_token(const Args& a, const PassCtx& x, const
     }
     if (!neg) return -1;
     w = 1;
-    return x.grid_mode ? first_cand(sh_cand, a.n_lcand, rf, false) : static_cast<int>(digit_of(key_of(rf), 0));
+    if (x.grid_mode) return first_cand(sh_cand, a.n_lcand, rf, false);
+    const unsigned key = key_of(rf);
+    if (key < x.key_lm) {
+      ++acc.l_below;
+      return -1;
+    }
+    if (key > x.key_lM) return -1;
+    ++acc.l_in;
+    return static_cast<int>(digit_of(key, 0));
   }
-  if (x.stage == kSums) {
+  if (STAGE == kSums) {
     if (!(neg || pos)) return -1;
     const long long qb = fixed_term(c, rb, A, x.shift);
     if (pos && rb < a.c_hi) acc.s_pos_bf += qb;
@@ -312,15 +330,15 @@ __device__ __forceinline__ int pass_token(const Args& a, const PassCtx& x, const
     }
     if (!neg) return -1;
     const unsigned key = key_of(rf);
-    if (!digit_match(key, 1, x.prefix)) return -1;
+    if (key < x.key_lm || key > x.key_lM || !digit_match(key, 1, x.prefix)) return -1;
     w = 1;
     return static_cast<int>(digit_of(key, 1));
   }
-  if (x.stage == kL2 || x.stage == kLNb) {
+  if (STAGE == kL2 || STAGE == kLNb) {
     if (!neg) return -1;
     const unsigned key = key_of(rf);
-    if (x.stage == kL2) {
-      if (!digit_match(key, 2, x.prefix)) return -1;
+    if (STAGE == kL2) {
+      if (key < x.key_lm || key > x.key_lM || !digit_match(key, 2, x.prefix)) return -1;
       w = 1;
       return static_cast<int>(digit_of(key, 2));
     }
@@ -332,7 +350,7 @@ __device__ __forceinline__ int pass_token(const Args& a, const PassCtx& x, const
   }
   // H stages: Pos set, weights q_fp8.  kH0 needs q_fp8 for both signs: one
   // evaluation for every signed token keeps the warp on one path.
-  if (x.stage == kH0) {
+  if (STAGE == kH0) {
     if (!(neg || pos)) return -1;
     const long long qf = fixed_term(c, rf, A, x.shift);
     if (neg) {
@@ -340,16 +358,22 @@ __device__ __forceinline__ int pass_token(const Args& a, const PassCtx& x, const
       else ++acc.k_fp;
       return -1;
     }
+    const unsigned key = key_of(rf);
+    if (key < x.key_hm) {
+      acc.h_below += qf;
+      return -1;
+    }
+    if (key >= x.key_hM) return -1;
     w = qf;
-    return static_cast<int>(digit_of(key_of(rf), 0));
+    return static_cast<int>(digit_of(key, 0));
   }
   if (!pos) return -1;
   const unsigned key = key_of(rf);
-  if (x.stage == kPFin) {
+  if (STAGE == kPFin) {
     if (rf < x.hi_star) acc.s_pos_fp += fixed_term(c, rf, A, x.shift);
     return -1;
   }
-  if (x.stage == kHNb) {
+  if (STAGE == kHNb) {
     if (fixed_nonzero(c, rf, A, x.shift)) {
       if (key < x.u) acc.nb_below1 = max(acc.nb_below1, key + 1);
       if (key > x.u) acc.nb_above = min(acc.nb_above, key);
@@ -358,7 +382,7 @@ __device__ __forceinline__ int pass_token(const Args& a, const PassCtx& x, const
     }
     return -1;
   }
-  if (!digit_match(key, x.digit, x.prefix)) return -1;
+  if (key < x.key_hm || key >= x.key_hM || !digit_match(key, x.digit, x.prefix)) return -1;
   w = fixed_term(c, rf, A, x.shift);
   return static_cast<int>(digit_of(key, x.digit));
 }
@@ -416,8 +440,9 @@ __device__ __forceinline__ void hist_add_lane(ShHist& sh, int d, long long w) {
 // One pass over the tokens by the whole grid (or by one block in the fused
 // small-T kernel).  Passes read G tokens per lane and step: 16-byte loads when
 // G = 4.  sh_cand holds the stage's grid candidates in GRID mode.
-template <int G>
-__device__ void pass_body(const Args& a, int stage, ShHist& sh, float* sh_cand) {
+template <int G, int STAGE>
+__device__ void pass_body(const Args& a, ShHist& sh, float* sh_cand) {
+  constexpr int stage = STAGE;
   State* st = a.st;
   if ((stage == kH1 || stage == kH2 || stage == kHNb) && !st->h_active) return;
   if (stage == kPFin && st->p_known) return;
@@ -460,7 +485,7 @@ __device__ void pass_body(const Args& a, int stage, ShHist& sh, float* sh_cand) 
   x.key_lM = key_lM;
   x.key_hm = key_hm;
   x.key_hM = key_hM;
-  PassAcc acc{0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, kNone, kNone, 0};
+  PassAcc acc{0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, kNone, kNone, 0, 0, 0, 0};
   // histogram update: 0 none, 1 warp-aggregated counts, 2 warp-aggregated
   // weights (leading digit, grid candidates), 3 per lane (later digits)
   int hist_mode = 0;
@@ -518,7 +543,7 @@ __device__ void pass_body(const Args& a, int stage, ShHist& sh, float* sh_cand) 
 #pragma unroll
     for (int j = 0; j < G; ++j) {
       long long w;
-      const int d = pass_token(a, x, sh_cand, valid[j], A[j], rf[j], rb[j], c[j], acc, w);
+      const int d = pass_token<STAGE>(a, x, sh_cand, valid[j], A[j], rf[j], rb[j], c[j], acc, w);
       if (hist_mode == 1) hist_add_warp<true>(sh, d, w);
       else if (hist_mode == 2) hist_add_warp<false>(sh, d, w);
       else if (hist_mode == 3) hist_add_lane(sh, d, w);
@@ -533,7 +558,7 @@ __device__ void pass_body(const Args& a, int stage, ShHist& sh, float* sh_cand) 
     const float c = in && need_c ? a.coef[t] : 1.f;
     const bool valid = in && (a.mask ? a.mask[t] != 0 : true);
     long long w;
-    const int d = pass_token(a, x, sh_cand, valid, A, rf, rb, c, acc, w);
+    const int d = pass_token<STAGE>(a, x, sh_cand, valid, A, rf, rb, c, acc, w);
     if (hist_mode == 1) hist_add_warp<true>(sh, d, w);
     else if (hist_mode == 2) hist_add_warp<false>(sh, d, w);
     else if (hist_mode == 3) hist_add_lane(sh, d, w);
@@ -543,6 +568,8 @@ __device__ void pass_body(const Args& a, int stage, ShHist& sh, float* sh_cand) 
             s_pos_fp = acc.s_pos_fp;
   unsigned emax = acc.emax, bad = acc.bad;
   unsigned nb_below1 = acc.nb_below1, nb_above = acc.nb_above, nb_m = acc.nb_m, nb_M1 = acc.nb_M1;
+  unsigned long long l_below = acc.l_below, l_in = acc.l_in;  // widened for the warp sum
+  long long h_below = acc.h_below;
 
   // ---- flush: warp-aggregated scalars, then the block histogram
   n_neg = warp_sum(n_neg);
@@ -559,7 +586,13 @@ __device__ void pass_body(const Args& a, int stage, ShHist& sh, float* sh_cand) 
   nb_above = __reduce_min_sync(0xffffffffu, nb_above);
   nb_m = __reduce_min_sync(0xffffffffu, nb_m);
   nb_M1 = __reduce_max_sync(0xffffffffu, nb_M1);
+  l_below = warp_sum(l_below);
+  l_in = warp_sum(l_in);
+  h_below = warp_sum(h_below);
   if (lane == 0) {
+    if (l_below) atomicAdd(&st->l_below, l_below);
+    if (l_in) atomicAdd(&st->l_in, l_in);
+    if (h_below) atomicAdd(&st->h_below, static_cast<unsigned long long>(h_below));
     if (n_neg) atomicAdd(&st->n_neg, n_neg);
     if (n_pos) atomicAdd(&st->n_pos, n_pos);
     if (k_bf) atomicAdd(&st->k_bf16, k_bf);
@@ -589,11 +622,42 @@ __device__ void pass_body(const Args& a, int stage, ShHist& sh, float* sh_cand) 
   }
 }
 
+// One pass, compiled per stage so that each holds only its own state.
 template <int G>
-__global__ void __launch_bounds__(256) pass_kernel(Args a, int stage) {
+__device__ void pass_any(const Args& a, int stage, ShHist& sh, float* sh_cand) {
+  switch (stage) {
+    case kPrep: pass_body<G, kPrep>(a, sh, sh_cand); break;
+    case kSums: pass_body<G, kSums>(a, sh, sh_cand); break;
+    case kL2: pass_body<G, kL2>(a, sh, sh_cand); break;
+    case kLNb: pass_body<G, kLNb>(a, sh, sh_cand); break;
+    case kH0: pass_body<G, kH0>(a, sh, sh_cand); break;
+    case kH1: pass_body<G, kH1>(a, sh, sh_cand); break;
+    case kH2: pass_body<G, kH2>(a, sh, sh_cand); break;
+    case kHNb: pass_body<G, kHNb>(a, sh, sh_cand); break;
+    default: pass_body<G, kPFin>(a, sh, sh_cand); break;
+  }
+}
+
+template <int G, int STAGE>
+__global__ void __launch_bounds__(256) pass_kernel(Args a) {
   __shared__ ShHist sh;
   __shared__ float sh_cand[kBuckets];
-  pass_body<G>(a, stage, sh, sh_cand);
+  pass_body<G, STAGE>(a, sh, sh_cand);
+}
+
+template <int G>
+void launch_pass(const Args& a, int stage, int grid, cudaStream_t s) {
+  switch (stage) {
+    case kPrep: pass_kernel<G, kPrep><<<grid, 256, 0, s>>>(a); break;
+    case kSums: pass_kernel<G, kSums><<<grid, 256, 0, s>>>(a); break;
+    case kL2: pass_kernel<G, kL2><<<grid, 256, 0, s>>>(a); break;
+    case kLNb: pass_kernel<G, kLNb><<<grid, 256, 0, s>>>(a); break;
+    case kH0: pass_kernel<G, kH0><<<grid, 256, 0, s>>>(a); break;
+    case kH1: pass_kernel<G, kH1><<<grid, 256, 0, s>>>(a); break;
+    case kH2: pass_kernel<G, kH2><<<grid, 256, 0, s>>>(a); break;
+    case kHNb: pass_kernel<G, kHNb><<<grid, 256, 0, s>>>(a); break;
+    default: pass_kernel<G, kPFin><<<grid, 256, 0, s>>>(a); break;
+  }
 }
 
 // ------------------------------------------------------------------ 128-bit
@@ -810,7 +874,7 @@ __device__ void decide_body(const Args& a, int stage, long long* scratch) {
       st->tgt_hi = 0;
       st->tgt_lo = st->k_bf16;
       st->dmul = 1;
-      st->below = 0;
+      st->below = static_cast<long long>(st->l_below);  // A<0 tokens under I_L (0 in GRID mode)
       st->prefix = 0;
       st->found = 1;
       sh_go = st->n_neg > 0;
@@ -881,9 +945,18 @@ __device__ void decide_body(const Args& a, int stage, long long* scratch) {
 
   if (stage == kLNb) {
     if (tid == 0) {
-      if (st->n_neg > 0) {
-        // minimisers of |C(L) - k|, C(L) = #{A<0 : r_fp8 <= L}, around u = r_(k)
-        const long long k = static_cast<long long>(st->k_bf16);
+      const long long k = static_cast<long long>(st->k_bf16);
+      const long long lb = static_cast<long long>(st->l_below), lin = static_cast<long long>(st->l_in);
+      if (st->n_neg > 0 && k <= lb) {
+        // C(lo_min) >= k already: |C - k| grows across I_L, so the bound is in
+        // the piece that contains lo_min
+        st->lo_star = lower_from_interval(a, st, -INFINITY, next_down(a.lo_min));
+      } else if (st->n_neg > 0 && k > lb + lin) {
+        // C(lo_max) < k: |C - k| shrinks across I_L, the piece containing lo_max
+        st->lo_star = lower_from_interval(a, st, next_up(a.lo_max), INFINITY);
+      } else if (st->n_neg > 0) {
+        // minimisers of |C(L) - k|, C(L) = #{A<0 : r_fp8 <= L}, around u = r_(k),
+        // which the select found inside I_L
         const float fu = __uint_as_float(st->u_key);
         const long long w_above = st->p_le - k, w_below = k - st->p_lt;
         const float z = st->nb_below1 ? __uint_as_float(st->nb_below1 - 1) : -INFINITY;
@@ -912,7 +985,10 @@ __device__ void decide_body(const Args& a, int stage, long long* scratch) {
   }
 
   if (stage == kH0) {
-    if (tid == 0) sh_go = begin_upper(a, st);
+    if (tid == 0) {
+      sh_go = begin_upper(a, st);
+      st->below = static_cast<long long>(st->h_below);  // P(hi_min): A>0 weight under I_H
+    }
     __syncthreads();
     if (sh_go) select_step(st, 11, false, scratch);
     return;
@@ -938,7 +1014,12 @@ __device__ void decide_body(const Args& a, int stage, long long* scratch) {
       const float z = st->nb_below1 ? __uint_as_float(st->nb_below1 - 1) : -INFINITY;
       const float w = st->nb_above != kNone ? __uint_as_float(st->nb_above) : INFINITY;
       float lo, hi;
-      if (!st->found) {  // even all of P stays below the target
+      if (ge128(mul_u64(static_cast<unsigned long long>(st->h_below), D), X)) {
+        // P(hi_min) D >= X already: the objective grows across I_H, so the
+        // bound is in the piece that contains hi_min (P(H*) by the last pass)
+        lo = -INFINITY;
+        hi = next_down(a.hi_min);
+      } else if (!st->found) {  // even all of P stays below the target
         lo = next_up(z);
         hi = INFINITY;
       } else {
@@ -1033,7 +1114,7 @@ __global__ void __launch_bounds__(kCoopThreads) coop_kernel(Args a, StageList li
   __shared__ float sh_cand[kBuckets];
   __shared__ int sh_ok;
   for (int i = 0; i < list.n; ++i) {
-    pass_body<G>(a, list.s[i], sh, sh_cand);
+    pass_any<G>(a, list.s[i], sh, sh_cand);
     if (!grid_barrier(a.st, limit_ns, &sh_ok)) return;
     if (blockIdx.x == 0) decide_body(a, list.s[i], reinterpret_cast<long long*>(&sh));
     if (!grid_barrier(a.st, limit_ns, &sh_ok)) return;
@@ -1099,8 +1180,8 @@ cudaError_t launch_calibrate(const float* r_fp8, const float* r_bf16, const floa
     return cudaLaunchCooperativeKernel(fn, dim3(static_cast<unsigned>(nb)), dim3(kCoopThreads), args, 0, s);
   }
   for (int i = 0; i < n; ++i) {
-    if (vec) pass_kernel<4><<<grid, 256, 0, s>>>(a, stages[i]);
-    else pass_kernel<1><<<grid, 256, 0, s>>>(a, stages[i]);
+    if (vec) launch_pass<4>(a, stages[i], grid, s);
+    else launch_pass<1>(a, stages[i], grid, s);
     decide_kernel<<<1, 1024, 0, s>>>(a, stages[i]);
   }
   return cudaGetLastError();
