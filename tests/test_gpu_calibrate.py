@@ -145,3 +145,44 @@ def test_calibrate_unaligned_inputs(cuda_lib, mode):
     cuda_lib.check()
     host = [None if t is None else t[1:] for t in args]
     _compare(cuda_lib.read_calib_result(buf), _ref(*host, 0.2, 0.28, mode=mode))
+
+
+def _interval_case(case, T, seed):
+    """Inputs that put the selection on a given side of the search intervals
+    I_L = [0.5, 0.9], I_H = [1.2, 2.0]: Algorithm 1 minimises over the pieces
+    inside the interval, so a crossing below or above it must come back as the
+    piece at that end, and ratios lying exactly on an end must count on the
+    right side of it (r <= L for the lower CDF, r < H for P(H))."""
+    r_fp, r_bf, adv, mask, coef = _inputs(T, seed)
+    g = torch.Generator().manual_seed(seed + 7)
+    neg, pos = adv < 0, adv > 0
+    if case == "lower_crossing_above_interval":  # C(lo_max) < k: many A<0 with r_bf <= c_lo, none in I_L
+        r_bf[neg] = 0.7
+        r_fp[neg] = 0.95 + 0.01 * torch.rand(int(neg.sum()), generator=g)
+    elif case == "lower_crossing_below_interval":  # k <= C(lo_min^-): most A<0 ratios under lo_min
+        r_fp[neg] = 0.3 + 0.1 * torch.rand(int(neg.sum()), generator=g)
+    elif case == "upper_target_below_interval":  # P(hi_min) D_bf >= N_bf D_fp8
+        r_bf[pos] = 1.1
+        r_fp[pos] = 1.15
+    elif case == "upper_target_above_interval":  # every A>0 ratio at or above hi_max
+        r_fp[pos] = 2.0 + torch.rand(int(pos.sum()), generator=g)
+    elif case == "ratios_on_interval_ends":
+        ends = torch.tensor([0.5, 0.9, 1.2, 2.0], dtype=torch.float32)
+        pick = torch.randint(0, 4, (T,), generator=g)
+        on = torch.rand(T, generator=g) < 0.3
+        r_fp[on] = ends[pick[on]]
+        r_bf[on & (torch.rand(T, generator=g) < 0.5)] = 0.8
+    return r_fp, r_bf, adv, mask, coef
+
+
+@pytest.mark.parametrize("mode", MODES)
+@pytest.mark.parametrize("T", [5000, 300000])
+@pytest.mark.parametrize("case", ["lower_crossing_above_interval", "lower_crossing_below_interval",
+                                  "upper_target_below_interval", "upper_target_above_interval",
+                                  "ratios_on_interval_ends"])
+def test_calibrate_crossings_outside_the_interval(cuda_lib, mode, T, case):
+    """Both launch paths (one cooperative launch up to 2^18 tokens, stage
+    launches above), every side a crossing can fall on, and ratios on the
+    interval ends; bit-exact against the oracle."""
+    args = _interval_case(case, T, 400 + T % 97)
+    _compare(_run(cuda_lib, *args, 0.2, 0.2, mode=mode), _ref(*args, 0.2, 0.2, mode=mode))
