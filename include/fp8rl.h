@@ -278,6 +278,9 @@ typedef struct fp8rl_calib_result {
 
 void fp8rl_default_calib_opts(fp8rl_calib_opts* opts);
 
+/* The workspace holds the search state (33 KB) and, for EXACT mode, lists of
+ * the tokens whose ratios fall inside I_L and I_H: 16 bytes per token of
+ * capacity (T entries each, so any input fits). */
 size_t fp8rl_calibrate_workspace_size(int64_t T);
 
 /* Algorithm 1.  Inputs, float [T] unless noted:

@@ -68,6 +68,21 @@ struct State {
   unsigned long long l_below;  // #{A<0 : r_fp8 < lo_min}
   unsigned long long l_in;     // #{A<0 : lo_min <= r_fp8 <= lo_max}
   unsigned long long h_below;  // sum_{A>0, r_fp8 < hi_min} q_fp8 (int64 two's complement)
+  // The tokens inside the intervals are also written to two lists (keys of
+  // I_L's A<0 tokens from the first pass; keys and q_fp8 of I_H's A>0 tokens
+  // from the H digit-0 pass), and the later selection passes read only the
+  // lists.  What they would have met outside the intervals is kept here
+  // (u32 maxima; a minimum is kept as the maximum of ~key, 0 = none):
+  unsigned int l_nb_below1;     // 1 + max{key : A<0, r < lo_min}
+  unsigned int l_nb_above_inv;  // ~min{key : A<0, r > lo_max}
+  unsigned int l_mp_inv;        // ~min{key in I_L : key > key(lo_min)}
+  unsigned int l_Mp1;           // 1 + max{key in I_L}
+  unsigned int h_nb_below1;     // 1 + max{key : A>0, r < hi_min, q != 0}
+  unsigned int h_nb_above_inv;  // ~min{key : A>0, r >= hi_max, q != 0}
+  unsigned int h_top1;          // 1 + max{key : A>0, r >= hi_max, q != 0}
+  unsigned int h_mp_inv;        // ~min{key in I_H : q != 0}
+  unsigned int h_Mp1;           // 1 + max{key in I_H : q != 0}
+  unsigned int pad2;
   // written by decide steps
   int shift;
   int found;
@@ -103,6 +118,15 @@ struct Args {
   int n_lcand, n_hcand;
   State* st;
   fp8rl_calib_result* out;
+  // Interval lists (EXACT mode), one segment per warp of the full passes
+  // (nseg segments of seg_cap entries, each warp's tokens fit its segment, so
+  // no list entry needs an atomic), with the segment's fill in *_cnt[seg]:
+  unsigned* l_keys;   // keys of the A<0 tokens inside I_L
+  unsigned* l_cnt;
+  unsigned* h_keys;   // keys of the A>0 tokens inside I_H
+  long long* h_q;     // their q_fp8
+  unsigned* h_cnt;
+  unsigned nseg, seg_cap;
 };
 
 __device__ __forceinline__ void flag(uint32_t bits) { atomicOr(&d_status, bits); }
@@ -225,18 +249,6 @@ __device__ __forceinline__ int approx_exponent(float c, float r, float a) {
   return static_cast<int>(ex) - 126 + kEBias;
 }
 
-// q = RNE(fl64(fl64(c r) a) 2^s) != 0, decided from the float32 product when
-// it is clearly above 1/2 or below 1/4 after scaling, exactly otherwise.
-__device__ __forceinline__ bool fixed_nonzero(float c, float r, float a, int s) {
-  const int ea = approx_exponent(c, r, a);
-  if (ea >= 0) {
-    const int e = ea - kEBias + s;  // product 2^s in [2^(e-1), 2^e)
-    if (e - 1 >= 1) return true;    // >= 2
-    if (e <= -2) return false;      // < 1/4
-  }
-  return fixed_term(c, r, a, s) != 0;
-}
-
 // Candidate i of an Algorithm 1 grid, fl32(x0 + i * step) in float64.
 __device__ __forceinline__ float cand_at(double x0, double step, int i) {
   return static_cast<float>(x0 + static_cast<double>(i) * step);
@@ -270,6 +282,8 @@ struct PassAcc {
   unsigned emax, bad, nb_below1, nb_above, nb_m, nb_M1;
   unsigned l_below, l_in;  // per-thread counts: T / grid threads each at most
   long long h_below;
+  unsigned l_nb_below1, l_nb_above_inv, l_mp_inv, l_Mp1;
+  unsigned h_nb_below1, h_nb_above_inv, h_top1, h_mp_inv, h_Mp1;
 };
 
 // Constants of one pass.
@@ -285,8 +299,9 @@ struct PassCtx {
 template <int STAGE>
 __device__ __forceinline__ int pass_token(const Args& a, const PassCtx& x, const float* sh_cand,
                                           bool valid, float A, float rf, float rb, float c,
-                                          PassAcc& acc, long long& w) {
+                                          PassAcc& acc, long long& w, unsigned& cand) {
   w = 0;
+  cand = kNone;  // the token's key when it goes to a list
   const bool neg = valid && A < 0.f, pos = valid && A > 0.f;
   if (STAGE == kPrep) {
     if (!(isfinite(A) && isfinite(rf) && isfinite(rb) && isfinite(c)) || rf < 0.f || rb < 0.f ||
@@ -309,10 +324,17 @@ __device__ __forceinline__ int pass_token(const Args& a, const PassCtx& x, const
     const unsigned key = key_of(rf);
     if (key < x.key_lm) {
       ++acc.l_below;
+      acc.l_nb_below1 = max(acc.l_nb_below1, key + 1);
       return -1;
     }
-    if (key > x.key_lM) return -1;
+    if (key > x.key_lM) {
+      acc.l_nb_above_inv = max(acc.l_nb_above_inv, ~key);
+      return -1;
+    }
     ++acc.l_in;
+    if (key > x.key_lm) acc.l_mp_inv = max(acc.l_mp_inv, ~key);
+    acc.l_Mp1 = max(acc.l_Mp1, key + 1);
+    cand = key;
     return static_cast<int>(digit_of(key, 0));
   }
   if (STAGE == kSums) {
@@ -334,20 +356,6 @@ __device__ __forceinline__ int pass_token(const Args& a, const PassCtx& x, const
     w = 1;
     return static_cast<int>(digit_of(key, 1));
   }
-  if (STAGE == kL2 || STAGE == kLNb) {
-    if (!neg) return -1;
-    const unsigned key = key_of(rf);
-    if (STAGE == kL2) {
-      if (key < x.key_lm || key > x.key_lM || !digit_match(key, 2, x.prefix)) return -1;
-      w = 1;
-      return static_cast<int>(digit_of(key, 2));
-    }
-    if (key < x.u) acc.nb_below1 = max(acc.nb_below1, key + 1);
-    if (key > x.u) acc.nb_above = min(acc.nb_above, key);
-    if (key > x.key_lm) acc.nb_m = min(acc.nb_m, key);
-    if (key <= x.key_lM) acc.nb_M1 = max(acc.nb_M1, key + 1);
-    return -1;
-  }
   // H stages: Pos set, weights q_fp8.  kH0 needs q_fp8 for both signs: one
   // evaluation for every signed token keeps the warp on one path.
   if (STAGE == kH0) {
@@ -361,30 +369,31 @@ __device__ __forceinline__ int pass_token(const Args& a, const PassCtx& x, const
     const unsigned key = key_of(rf);
     if (key < x.key_hm) {
       acc.h_below += qf;
+      if (qf != 0) acc.h_nb_below1 = max(acc.h_nb_below1, key + 1);
       return -1;
     }
-    if (key >= x.key_hM) return -1;
+    if (key >= x.key_hM) {
+      if (qf != 0) {
+        acc.h_nb_above_inv = max(acc.h_nb_above_inv, ~key);
+        acc.h_top1 = max(acc.h_top1, key + 1);
+      }
+      return -1;
+    }
+    if (qf != 0) {
+      acc.h_mp_inv = max(acc.h_mp_inv, ~key);
+      acc.h_Mp1 = max(acc.h_Mp1, key + 1);
+    }
+    cand = key;
     w = qf;
     return static_cast<int>(digit_of(key, 0));
   }
+  // GRID mode's P(H*) pass (EXACT mode takes P(H*) from the I_H list)
   if (!pos) return -1;
-  const unsigned key = key_of(rf);
   if (STAGE == kPFin) {
     if (rf < x.hi_star) acc.s_pos_fp += fixed_term(c, rf, A, x.shift);
     return -1;
   }
-  if (STAGE == kHNb) {
-    if (fixed_nonzero(c, rf, A, x.shift)) {
-      if (key < x.u) acc.nb_below1 = max(acc.nb_below1, key + 1);
-      if (key > x.u) acc.nb_above = min(acc.nb_above, key);
-      if (key >= x.key_hm) acc.nb_m = min(acc.nb_m, key);
-      if (key < x.key_hM) acc.nb_M1 = max(acc.nb_M1, key + 1);
-    }
-    return -1;
-  }
-  if (key < x.key_hm || key >= x.key_hM || !digit_match(key, x.digit, x.prefix)) return -1;
-  w = fixed_term(c, rf, A, x.shift);
-  return static_cast<int>(digit_of(key, x.digit));
+  return -1;
 }
 
 // Block histogram in shared memory with native 32-bit atomics only: counts
@@ -442,14 +451,13 @@ __device__ __forceinline__ void hist_add_lane(ShHist& sh, int d, long long w) {
 // G = 4.  sh_cand holds the stage's grid candidates in GRID mode.
 template <int G, int STAGE>
 __device__ void pass_body(const Args& a, ShHist& sh, float* sh_cand) {
+  // full passes over the tokens: kPrep, kSums, kH0 and GRID mode's kPFin
   constexpr int stage = STAGE;
   State* st = a.st;
-  if ((stage == kH1 || stage == kH2 || stage == kHNb) && !st->h_active) return;
   if (stage == kPFin && st->p_known) return;
   const bool grid_mode = a.grid_mode != 0;
   const bool want_hist = grid_mode ? (stage == kPrep || stage == kSums)
-                                   : (stage == kPrep || stage == kSums || stage == kL2 ||
-                                      stage == kH0 || stage == kH1 || stage == kH2);
+                                   : (stage == kPrep || stage == kSums || stage == kH0);
   if (want_hist) {
     for (int i = threadIdx.x; i < kBuckets; i += blockDim.x) {
       sh.cnt[i] = 0;
@@ -466,9 +474,7 @@ __device__ void pass_body(const Args& a, ShHist& sh, float* sh_cand) {
   const int shift = st->shift;
   const float lo_star = st->lo_star, hi_star = st->hi_star;
   const unsigned prefix = st->prefix, u = st->u_key;
-  int digit = 0;
-  if (stage == kSums || stage == kH1) digit = 1;
-  if (stage == kL2 || stage == kH2) digit = 2;
+  const int digit = stage == kSums ? 1 : 0;
   const unsigned key_lm = key_of(a.lo_min), key_lM = key_of(a.lo_max);
   const unsigned key_hm = key_of(a.hi_min), key_hM = key_of(a.hi_max);
 
@@ -485,7 +491,15 @@ __device__ void pass_body(const Args& a, ShHist& sh, float* sh_cand) {
   x.key_lM = key_lM;
   x.key_hm = key_hm;
   x.key_hM = key_hM;
-  PassAcc acc{0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, kNone, kNone, 0, 0, 0, 0};
+  PassAcc acc{0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, kNone, kNone, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0};
+  // EXACT mode writes the tokens inside the interval to its list: I_L from
+  // the first pass, I_H (with q_fp8) from the H digit-0 pass, each warp into
+  // its own segment
+  const bool to_list = !grid_mode && (stage == kPrep || stage == kH0);
+  const unsigned seg = static_cast<unsigned>((blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+  const size_t seg0 = static_cast<size_t>(seg) * a.seg_cap;
+  unsigned* list_keys = stage == kPrep ? a.l_keys : a.h_keys;
+  unsigned seg_fill = 0;
   // histogram update: 0 none, 1 warp-aggregated counts, 2 warp-aggregated
   // weights (leading digit, grid candidates), 3 per lane (later digits)
   int hist_mode = 0;
@@ -495,8 +509,19 @@ __device__ void pass_body(const Args& a, ShHist& sh, float* sh_cand) {
     else hist_mode = 3;
   }
   const bool need_rb = stage == kPrep || stage == kSums;
-  const bool need_c = a.coef != nullptr && !(stage == kL2 || stage == kLNb);
+  const bool need_c = a.coef != nullptr;
   const int lane = threadIdx.x & 31;
+  // append to the warp's segment (warp-uniform fill)
+  auto append = [&](unsigned cand, long long q) {
+    const unsigned want = __ballot_sync(0xffffffffu, cand != kNone);
+    if (!want) return;
+    if (cand != kNone) {
+      const size_t i = seg0 + seg_fill + __popc(want & ((1u << lane) - 1u));
+      list_keys[i] = cand;
+      if (stage == kH0) a.h_q[i] = q;
+    }
+    seg_fill += __popc(want);
+  };
   const int64_t ng = a.T / G;
   const int64_t warp_id = (blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x) >> 5;
   const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
@@ -543,7 +568,9 @@ __device__ void pass_body(const Args& a, ShHist& sh, float* sh_cand) {
 #pragma unroll
     for (int j = 0; j < G; ++j) {
       long long w;
-      const int d = pass_token<STAGE>(a, x, sh_cand, valid[j], A[j], rf[j], rb[j], c[j], acc, w);
+      unsigned cand;
+      const int d = pass_token<STAGE>(a, x, sh_cand, valid[j], A[j], rf[j], rb[j], c[j], acc, w, cand);
+      if (to_list) append(cand, w);
       if (hist_mode == 1) hist_add_warp<true>(sh, d, w);
       else if (hist_mode == 2) hist_add_warp<false>(sh, d, w);
       else if (hist_mode == 3) hist_add_lane(sh, d, w);
@@ -558,11 +585,14 @@ __device__ void pass_body(const Args& a, ShHist& sh, float* sh_cand) {
     const float c = in && need_c ? a.coef[t] : 1.f;
     const bool valid = in && (a.mask ? a.mask[t] != 0 : true);
     long long w;
-    const int d = pass_token<STAGE>(a, x, sh_cand, valid, A, rf, rb, c, acc, w);
+    unsigned cand;
+    const int d = pass_token<STAGE>(a, x, sh_cand, valid, A, rf, rb, c, acc, w, cand);
+    if (to_list) append(cand, w);
     if (hist_mode == 1) hist_add_warp<true>(sh, d, w);
     else if (hist_mode == 2) hist_add_warp<false>(sh, d, w);
     else if (hist_mode == 3) hist_add_lane(sh, d, w);
   }
+  if (to_list && lane == 0) (stage == kPrep ? a.l_cnt : a.h_cnt)[seg] = seg_fill;
   unsigned long long n_neg = acc.n_neg, n_pos = acc.n_pos, k_bf = acc.k_bf, k_fp = acc.k_fp;
   long long s_pos_bf = acc.s_pos_bf, s_neg_bf = acc.s_neg_bf, s_neg_fp = acc.s_neg_fp,
             s_pos_fp = acc.s_pos_fp;
@@ -589,7 +619,16 @@ __device__ void pass_body(const Args& a, ShHist& sh, float* sh_cand) {
   l_below = warp_sum(l_below);
   l_in = warp_sum(l_in);
   h_below = warp_sum(h_below);
+  unsigned ext[9] = {acc.l_nb_below1, acc.l_nb_above_inv, acc.l_mp_inv, acc.l_Mp1, acc.h_nb_below1,
+                     acc.h_nb_above_inv, acc.h_top1, acc.h_mp_inv, acc.h_Mp1};
+  unsigned* ext_st[9] = {&st->l_nb_below1, &st->l_nb_above_inv, &st->l_mp_inv, &st->l_Mp1, &st->h_nb_below1,
+                         &st->h_nb_above_inv, &st->h_top1, &st->h_mp_inv, &st->h_Mp1};
+#pragma unroll
+  for (int i = 0; i < 9; ++i) ext[i] = __reduce_max_sync(0xffffffffu, ext[i]);
   if (lane == 0) {
+#pragma unroll
+    for (int i = 0; i < 9; ++i)
+      if (ext[i]) atomicMax(ext_st[i], ext[i]);
     if (l_below) atomicAdd(&st->l_below, l_below);
     if (l_in) atomicAdd(&st->l_in, l_in);
     if (h_below) atomicAdd(&st->h_below, static_cast<unsigned long long>(h_below));
@@ -622,19 +661,95 @@ __device__ void pass_body(const Args& a, ShHist& sh, float* sh_cand) {
   }
 }
 
+// EXACT mode's later selection passes read the interval lists only:
+//   kL2   L digit 2 of the I_L keys (counts)
+//   kLNb  the I_L keys next to u (the ones outside I_L were kept by kPrep)
+//   kH1, kH2  H digits 1 and 2 of the I_H keys, weighted by q_fp8
+//   kHNb  the q != 0 keys of I_H next to u
+//   kPFin P(H*) = P(hi_min) + the q of I_H keys below H*
+template <int STAGE>
+__device__ void list_body(const Args& a, ShHist& sh) {
+  State* st = a.st;
+  if ((STAGE == kH1 || STAGE == kH2 || STAGE == kHNb) && !st->h_active) return;
+  if (STAGE == kPFin && st->p_known) return;
+  constexpr bool lower = STAGE == kL2 || STAGE == kLNb;
+  constexpr bool want_hist = STAGE == kL2 || STAGE == kH1 || STAGE == kH2;
+  constexpr int digit = STAGE == kH1 ? 1 : 2;
+  if (want_hist) {
+    for (int i = threadIdx.x; i < kBuckets; i += blockDim.x) {
+      sh.cnt[i] = 0;
+      sh.wlo[i] = 0;
+      sh.whi[i] = 0;
+    }
+    __syncthreads();
+  }
+  const unsigned prefix = st->prefix, u = st->u_key, key_h = key_of(st->hi_star);
+  const unsigned* cnt = lower ? a.l_cnt : a.h_cnt;
+  const int lane = threadIdx.x & 31;
+  const unsigned nwarps = (gridDim.x * blockDim.x) >> 5;
+  unsigned nb_below1 = 0, nb_above = kNone;
+  long long p = 0;
+  for (unsigned sg = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; sg < a.nseg; sg += nwarps) {
+    const unsigned fill = cnt[sg];
+    for (unsigned j = lane; j < fill; j += 32) {
+      const size_t i = static_cast<size_t>(sg) * a.seg_cap + j;
+      const unsigned key = lower ? a.l_keys[i] : a.h_keys[i];
+      if (STAGE == kL2) {
+        if (digit_match(key, 2, prefix)) hist_add_lane(sh, static_cast<int>(digit_of(key, 2)), 1);
+      } else if (STAGE == kLNb) {
+        if (key < u) nb_below1 = max(nb_below1, key + 1);
+        if (key > u) nb_above = min(nb_above, key);
+      } else {
+        const long long q = a.h_q[i];
+        if (STAGE == kH1 || STAGE == kH2) {
+          if (digit_match(key, digit, prefix)) hist_add_lane(sh, static_cast<int>(digit_of(key, digit)), q);
+        } else if (STAGE == kHNb) {
+          if (q != 0) {
+            if (key < u) nb_below1 = max(nb_below1, key + 1);
+            if (key > u) nb_above = min(nb_above, key);
+          }
+        } else if (key < key_h) {  // kPFin: r < H*
+          p += q;
+        }
+      }
+    }
+  }
+  if (STAGE == kPFin && blockIdx.x == 0 && threadIdx.x == 0) p += static_cast<long long>(st->h_below);
+  nb_below1 = __reduce_max_sync(0xffffffffu, nb_below1);
+  nb_above = __reduce_min_sync(0xffffffffu, nb_above);
+  p = warp_sum(p);
+  if (lane == 0) {
+    if (nb_below1) atomicMax(&st->nb_below1, nb_below1);
+    if (nb_above != kNone) atomicMin(&st->nb_above, nb_above);
+    if (p) atomicAdd(&st->s_pos_fp, static_cast<unsigned long long>(p));
+  }
+  if (want_hist) {
+    __syncthreads();
+    for (int i = threadIdx.x; i < kBuckets; i += blockDim.x) {
+      if (sh.cnt[i]) {
+        atomicAdd(&st->h_cnt[i], static_cast<unsigned long long>(sh.cnt[i]));
+        atomicAdd(&st->h_w[i], (static_cast<unsigned long long>(sh.whi[i]) << 32) | sh.wlo[i]);
+      }
+    }
+  }
+}
+
 // One pass, compiled per stage so that each holds only its own state.
 template <int G>
 __device__ void pass_any(const Args& a, int stage, ShHist& sh, float* sh_cand) {
   switch (stage) {
     case kPrep: pass_body<G, kPrep>(a, sh, sh_cand); break;
     case kSums: pass_body<G, kSums>(a, sh, sh_cand); break;
-    case kL2: pass_body<G, kL2>(a, sh, sh_cand); break;
-    case kLNb: pass_body<G, kLNb>(a, sh, sh_cand); break;
+    case kL2: list_body<kL2>(a, sh); break;
+    case kLNb: list_body<kLNb>(a, sh); break;
     case kH0: pass_body<G, kH0>(a, sh, sh_cand); break;
-    case kH1: pass_body<G, kH1>(a, sh, sh_cand); break;
-    case kH2: pass_body<G, kH2>(a, sh, sh_cand); break;
-    case kHNb: pass_body<G, kHNb>(a, sh, sh_cand); break;
-    default: pass_body<G, kPFin>(a, sh, sh_cand); break;
+    case kH1: list_body<kH1>(a, sh); break;
+    case kH2: list_body<kH2>(a, sh); break;
+    case kHNb: list_body<kHNb>(a, sh); break;
+    default:
+      if (a.grid_mode) pass_body<G, kPFin>(a, sh, sh_cand);
+      else list_body<kPFin>(a, sh);
+      break;
   }
 }
 
@@ -645,18 +760,27 @@ __global__ void __launch_bounds__(256) pass_kernel(Args a) {
   pass_body<G, STAGE>(a, sh, sh_cand);
 }
 
+template <int STAGE>
+__global__ void __launch_bounds__(256) list_kernel(Args a) {
+  __shared__ ShHist sh;
+  list_body<STAGE>(a, sh);
+}
+
 template <int G>
 void launch_pass(const Args& a, int stage, int grid, cudaStream_t s) {
   switch (stage) {
     case kPrep: pass_kernel<G, kPrep><<<grid, 256, 0, s>>>(a); break;
     case kSums: pass_kernel<G, kSums><<<grid, 256, 0, s>>>(a); break;
-    case kL2: pass_kernel<G, kL2><<<grid, 256, 0, s>>>(a); break;
-    case kLNb: pass_kernel<G, kLNb><<<grid, 256, 0, s>>>(a); break;
+    case kL2: list_kernel<kL2><<<grid, 256, 0, s>>>(a); break;
+    case kLNb: list_kernel<kLNb><<<grid, 256, 0, s>>>(a); break;
     case kH0: pass_kernel<G, kH0><<<grid, 256, 0, s>>>(a); break;
-    case kH1: pass_kernel<G, kH1><<<grid, 256, 0, s>>>(a); break;
-    case kH2: pass_kernel<G, kH2><<<grid, 256, 0, s>>>(a); break;
-    case kHNb: pass_kernel<G, kHNb><<<grid, 256, 0, s>>>(a); break;
-    default: pass_kernel<G, kPFin><<<grid, 256, 0, s>>>(a); break;
+    case kH1: list_kernel<kH1><<<grid, 256, 0, s>>>(a); break;
+    case kH2: list_kernel<kH2><<<grid, 256, 0, s>>>(a); break;
+    case kHNb: list_kernel<kHNb><<<grid, 256, 0, s>>>(a); break;
+    default:
+      if (a.grid_mode) pass_kernel<G, kPFin><<<grid, 256, 0, s>>>(a);
+      else list_kernel<kPFin><<<grid, 256, 0, s>>>(a);
+      break;
   }
 }
 
@@ -945,6 +1069,15 @@ __device__ void decide_body(const Args& a, int stage, long long* scratch) {
 
   if (stage == kLNb) {
     if (tid == 0) {
+      // the list pass met only I_L's keys; the first pass kept the nearest
+      // keys outside I_L, which lie below or above every key of I_L
+      st->nb_below1 = max(st->nb_below1, st->l_nb_below1);
+      if (st->l_nb_above_inv) st->nb_above = min(st->nb_above, ~st->l_nb_above_inv);
+      // pieces at the ends of I_L: min{key > key(lo_min)}, 1 + max{key <= key(lo_max)}
+      unsigned mp = st->l_mp_inv ? ~st->l_mp_inv : kNone;
+      if (st->l_nb_above_inv) mp = min(mp, ~st->l_nb_above_inv);
+      st->nb_mpiece = mp;
+      st->nb_Mpiece1 = max(st->l_Mp1, st->l_nb_below1);
       const long long k = static_cast<long long>(st->k_bf16);
       const long long lb = static_cast<long long>(st->l_below), lin = static_cast<long long>(st->l_in);
       if (st->n_neg > 0 && k <= lb) {
@@ -1011,6 +1144,21 @@ __device__ void decide_body(const Args& a, int stage, long long* scratch) {
       // float interval of H, from u and its positive-weight neighbours
       const U128 X{st->tgt_hi, st->tgt_lo};
       const unsigned long long D = static_cast<unsigned long long>(st->dmul);
+      // the list pass met only I_H's keys; H0 kept the nearest q != 0 keys
+      // outside I_H.  With u in I_H those below lie under u and those above
+      // over it; with no u (P stays below the target) every key lies under it.
+      if (st->found) {
+        st->nb_below1 = max(st->nb_below1, st->h_nb_below1);
+        if (st->h_nb_above_inv) st->nb_above = min(st->nb_above, ~st->h_nb_above_inv);
+      } else {
+        st->nb_below1 = max(st->nb_below1, max(st->h_nb_below1, st->h_top1));
+      }
+      // pieces at the ends of I_H: min{key >= key(hi_min), q > 0},
+      // 1 + max{key < key(hi_max), q > 0}
+      unsigned mp = st->h_mp_inv ? ~st->h_mp_inv : kNone;
+      if (st->h_nb_above_inv) mp = min(mp, ~st->h_nb_above_inv);
+      st->nb_mpiece = mp;
+      st->nb_Mpiece1 = max(st->h_Mp1, st->h_nb_below1);
       const float z = st->nb_below1 ? __uint_as_float(st->nb_below1 - 1) : -INFINITY;
       const float w = st->nb_above != kNone ? __uint_as_float(st->nb_above) : INFINITY;
       float lo, hi;
@@ -1123,7 +1271,72 @@ __global__ void __launch_bounds__(kCoopThreads) coop_kernel(Args a, StageList li
 
 }  // namespace
 
-size_t calib_workspace_bytes(int64_t) { return align_up(sizeof(State), 256); }
+// Launch shape of a call: one cooperative launch up to kCoopMaxT tokens, else
+// pass / decide launches on up to four blocks of 256 per SM.  The interval
+// lists get one segment per warp of the full passes, as long as the tokens
+// that warp visits (its grid-stride steps of 32 lanes x G tokens, plus the
+// T mod 4 tail that warp 0 takes).
+struct CalibShape {
+  bool coop;
+  int blocks, threads;
+  unsigned nseg, seg_cap;
+};
+
+CalibShape calib_shape(int64_t T, int G) {
+  CalibShape c{};
+  c.coop = T <= kCoopMaxT;
+  if (c.coop) {
+    int64_t nb = (T + kCoopTokensPerBlock - 1) / kCoopTokensPerBlock;
+    nb = nb < 1 ? 1 : (nb > kCoopMaxBlocks ? kCoopMaxBlocks : nb);
+    if (nb > sm_count()) nb = sm_count();
+    c.blocks = static_cast<int>(nb);
+    c.threads = kCoopThreads;
+  } else {
+    const int64_t want = (T + 4095) / 4096;
+    const int64_t cap = static_cast<int64_t>(sm_count()) * 4;
+    c.blocks = static_cast<int>(want < 1 ? 1 : (want > cap ? cap : want));
+    c.threads = 256;
+  }
+  c.nseg = static_cast<unsigned>(c.blocks) * static_cast<unsigned>(c.threads / 32);
+  const int64_t ng = (T > 0 ? T : 0) / G;
+  const int64_t per = static_cast<int64_t>(c.nseg) * 32;
+  const int64_t steps = (ng + per - 1) / per;
+  c.seg_cap = static_cast<unsigned>(steps * 32 * G + 32);
+  return c;
+}
+
+size_t calib_state_bytes() { return align_up(sizeof(State), 256); }
+
+// Workspace: the State, then (EXACT mode's interval lists) I_L keys, I_L
+// segment fills, I_H keys, I_H q, I_H segment fills, for the larger of the
+// two token groupings (4 tokens a lane with aligned inputs, else 1).
+struct CalibLayout {
+  size_t l_keys, l_cnt, h_keys, h_q, h_cnt, total;
+  unsigned seg_cap;
+};
+
+CalibLayout calib_layout(int64_t T) {
+  const CalibShape s1 = calib_shape(T, 1), s4 = calib_shape(T, 4);
+  const unsigned cap = s1.seg_cap > s4.seg_cap ? s1.seg_cap : s4.seg_cap;
+  const size_t n = static_cast<size_t>(s1.nseg) * cap;
+  CalibLayout l{};
+  size_t off = calib_state_bytes();
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off = align_up(off + bytes, 256);
+    return at;
+  };
+  l.l_keys = take(n * 4);
+  l.l_cnt = take(static_cast<size_t>(s1.nseg) * 4);
+  l.h_keys = take(n * 4);
+  l.h_q = take(n * 8);
+  l.h_cnt = take(static_cast<size_t>(s1.nseg) * 4);
+  l.total = off;
+  l.seg_cap = cap;
+  return l;
+}
+
+size_t calib_workspace_bytes(int64_t T) { return calib_layout(T).total; }
 
 cudaError_t launch_calibrate(const float* r_fp8, const float* r_bf16, const float* adv,
                              const uint8_t* mask, const float* coef, int64_t T, float eps_low,
@@ -1154,34 +1367,38 @@ cudaError_t launch_calibrate(const float* r_fp8, const float* r_bf16, const floa
   a.n_hcand = a.grid_mode ? static_cast<int>(std::llround((o.hi_max - o.hi_min) / o.step)) + 1 : 0;
   a.st = static_cast<State*>(ws);
   a.out = result;
+  const CalibLayout lay = calib_layout(T);
+  char* base = static_cast<char*>(ws);
+  a.l_keys = reinterpret_cast<unsigned*>(base + lay.l_keys);
+  a.l_cnt = reinterpret_cast<unsigned*>(base + lay.l_cnt);
+  a.h_keys = reinterpret_cast<unsigned*>(base + lay.h_keys);
+  a.h_q = reinterpret_cast<long long*>(base + lay.h_q);
+  a.h_cnt = reinterpret_cast<unsigned*>(base + lay.h_cnt);
+  a.seg_cap = lay.seg_cap;
 
   cudaError_t e = cudaMemsetAsync(ws, 0, sizeof(State), s);
   if (e != cudaSuccess) return e;
   auto al = [](const void* p, uintptr_t n) { return (reinterpret_cast<uintptr_t>(p) & (n - 1)) == 0; };
   const bool vec = al(r_fp8, 16) && al(r_bf16, 16) && al(adv, 16) && al(coef, 16) && al(mask, 4);
-  int64_t want = (T + 4095) / 4096;
-  const int64_t cap = static_cast<int64_t>(sm_count()) * 4;
-  const int grid = static_cast<int>(want < 1 ? 1 : (want > cap ? cap : want));
+  const CalibShape sh = calib_shape(T, vec ? 4 : 1);
+  a.nseg = sh.nseg;  // the layout's segment capacity covers either grouping
   const int stages_exact[] = {kPrep, kSums, kL2, kLNb, kH0, kH1, kH2, kHNb, kPFin};
   const int stages_grid[] = {kPrep, kSums, kPFin};
   const int* stages = a.grid_mode ? stages_grid : stages_exact;
   const int n = a.grid_mode ? 3 : 9;
-  if (T <= kCoopMaxT) {
+  if (sh.coop) {
     StageList list{};
     list.n = n;
     for (int i = 0; i < n; ++i) list.s[i] = stages[i];
-    int64_t nb = (T + kCoopTokensPerBlock - 1) / kCoopTokensPerBlock;
-    nb = nb < 1 ? 1 : (nb > kCoopMaxBlocks ? kCoopMaxBlocks : nb);
-    if (nb > sm_count()) nb = sm_count();
     uint64_t limit = wait_limit_ns();
     void* args[] = {&a, &list, &limit};
     const void* fn = vec ? reinterpret_cast<const void*>(&coop_kernel<4>)
                          : reinterpret_cast<const void*>(&coop_kernel<1>);
-    return cudaLaunchCooperativeKernel(fn, dim3(static_cast<unsigned>(nb)), dim3(kCoopThreads), args, 0, s);
+    return cudaLaunchCooperativeKernel(fn, dim3(static_cast<unsigned>(sh.blocks)), dim3(sh.threads), args, 0, s);
   }
   for (int i = 0; i < n; ++i) {
-    if (vec) launch_pass<4>(a, stages[i], grid, s);
-    else launch_pass<1>(a, stages[i], grid, s);
+    if (vec) launch_pass<4>(a, stages[i], sh.blocks, s);
+    else launch_pass<1>(a, stages[i], sh.blocks, s);
     decide_kernel<<<1, 1024, 0, s>>>(a, stages[i]);
   }
   return cudaGetLastError();
