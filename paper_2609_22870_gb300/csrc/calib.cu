@@ -235,18 +235,21 @@ __device__ __forceinline__ unsigned digit_of(unsigned key, int digit) {
   return key & 0x3FFu;
 }
 
-// frexp exponent of fl32(fl32(|c r|) |a|) plus kEBias, or -1 when that
-// product or c r is not a normal float32 (zero, subnormal, overflow).  For a normal
-// product the exact |fl64(fl64(c r) a)| lies within a factor 1 +- 2^-22 of
-// it, so its exponent differs by at most one.
-__device__ __forceinline__ int approx_exponent(float c, float r, float a) {
+// frexp exponent of |fl64(fl64(c r) a)| plus kEBias (0 for a zero product),
+// from the float32 product wherever that settles it: the two float32
+// roundings leave it within a factor 1 +- 2^-22 of the exact product, so when
+// its significand lies at least 8 ulps (2^-20) from both ends of its binade
+// the exact product shares its exponent.  Otherwise (about 2^-19 of the
+// products, or any zero, subnormal or overflowing one) the integer
+// evaluation decides, so the warp almost never takes that path.
+__device__ __forceinline__ unsigned term_exponent_fast(float c, float r, float a) {
   const float cr = fabsf(c * r);
-  const unsigned ecr = __float_as_uint(cr) >> 23;
-  if (ecr == 0 || ecr >= 255) return -1;  // c r itself must be normal
   const float p = cr * fabsf(a);
-  const unsigned ex = __float_as_uint(p) >> 23;
-  if (ex == 0 || ex >= 255) return -1;
-  return static_cast<int>(ex) - 126 + kEBias;
+  const unsigned bcr = __float_as_uint(cr), bp = __float_as_uint(p);
+  const unsigned ecr = bcr >> 23, ex = bp >> 23, m = bp & 0x7FFFFFu;
+  if (ecr != 0 && ecr < 255 && ex != 0 && ex < 255 && m >= 8u && m <= 0x7FFFF7u)
+    return ex - 126u + static_cast<unsigned>(kEBias);
+  return term_exponent(c, r, a);
 }
 
 // Candidate i of an Algorithm 1 grid, fl32(x0 + i * step) in float64.
@@ -313,10 +316,7 @@ __device__ __forceinline__ int pass_token(const Args& a, const PassCtx& x, const
     }
     if (pos) ++acc.n_pos;
     if (neg || pos) {
-      // the exact exponent only where it can raise the running maximum
-      const int eb = approx_exponent(c, rb, A), ef = approx_exponent(c, rf, A);
-      if (eb < 0 || eb + 1 > static_cast<int>(acc.emax)) acc.emax = max(acc.emax, term_exponent(c, rb, A));
-      if (ef < 0 || ef + 1 > static_cast<int>(acc.emax)) acc.emax = max(acc.emax, term_exponent(c, rf, A));
+      acc.emax = max(acc.emax, max(term_exponent_fast(c, rb, A), term_exponent_fast(c, rf, A)));
     }
     if (!neg) return -1;
     w = 1;
