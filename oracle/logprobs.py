@@ -49,6 +49,11 @@ transposed bf16 weight W^T and hidden states h^T (the B operands; the weight
 granularity of the forward pass).  P is taken in float32 (the value the
 hardware holds) before it is quantised; V and T are padded with zeros to
 multiples of 128 along K.
+
+With power-of-two (UE8M0) forward scales the backward keeps that scale format
+for its own four operands (the scales of the hardware's block-scaled MMA):
+each S is the smallest power of two not below fl32(amax / 448), raised to
+2^-127 where it falls below E8M0's range.
 """
 
 import numpy as np
@@ -149,25 +154,28 @@ def _pad_cols(x, mult=128):
     return out
 
 
-def lm_head_backward_fp8(h_codes, h_scales, w_codes, w_scales, gran, targets, g, h, W):
+def lm_head_backward_fp8(h_codes, h_scales, w_codes, w_scales, gran, targets, g, h, W, pow2=False):
     """dLoss/dh and dLoss/dW with both contractions on E4M3 operands.
 
     P (float64 from the FP8 logits) is rounded to float32 and quantised twice:
     P [T][V] with 1x128 blocks along V (A operand of dh = P W), P^T [V][T]
     with 128 x 128 blocks (A operand of dW = P^T h); W^T [H][V] and h^T [H][T]
     are quantised from the bf16 values with 128 x 128 blocks (B operands).
-    The products of the dequantised operands are summed in float64.  Returns
-    the quantised operands too (codes and scales in natural shape)."""
+    ``pow2``: the four take power-of-two scales floored at 2^-127 (the
+    backward of the UE8M0 variant).  The products of the dequantised operands
+    are summed in float64.  Returns the quantised operands too (codes and
+    scales in natural shape)."""
     y = np.asarray(targets, np.int64)
     gg = np.asarray(g, np.float64)
     z = logits(h_codes, h_scales, w_codes, w_scales, gran)
     _, lse = log_softmax_gather(z, y)
     P32 = dlogits(z, y, lse, gg).astype(np.float32)
     T, V = P32.shape
-    pq, ps = Q.quantize(_pad_cols(P32), Q.BLOCK, Q.ACT)              # (T, V') codes, (T, V'/128)
-    ptq, pts = Q.quantize(_pad_cols(P32.T), Q.BLOCK, Q.WEIGHT)       # (V, T'),  (ceil(V/128), T'/128)
-    wtq, wts = Q.quantize(_pad_cols(np.asarray(W, np.float32).T), Q.BLOCK, Q.WEIGHT)   # (H, V')
-    htq, hts = Q.quantize(_pad_cols(np.asarray(h, np.float32).T), Q.BLOCK, Q.WEIGHT)   # (H, T')
+    kw = {"pow2": True, "scale_floor": Q.E8M0_MIN} if pow2 else {}
+    pq, ps = Q.quantize(_pad_cols(P32), Q.BLOCK, Q.ACT, **kw)              # (T, V') codes, (T, V'/128)
+    ptq, pts = Q.quantize(_pad_cols(P32.T), Q.BLOCK, Q.WEIGHT, **kw)       # (V, T'),  (ceil(V/128), T'/128)
+    wtq, wts = Q.quantize(_pad_cols(np.asarray(W, np.float32).T), Q.BLOCK, Q.WEIGHT, **kw)   # (H, V')
+    htq, hts = Q.quantize(_pad_cols(np.asarray(h, np.float32).T), Q.BLOCK, Q.WEIGHT, **kw)   # (H, T')
     P_hat = Q.dequantize(pq, ps, Q.BLOCK, Q.ACT)
     Pt_hat = Q.dequantize(ptq, pts, Q.BLOCK, Q.WEIGHT)
     Wt_hat = Q.dequantize(wtq, wts, Q.BLOCK, Q.WEIGHT)

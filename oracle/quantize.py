@@ -26,7 +26,11 @@ Readings taken where the paper is silent:
 Power-of-two (UE8M0) variant, outside the paper (its S is amax / 448): the
 scale format that the hardware's block-scaled MMA takes.  S is rounded up to
 the smallest power of two not below fl32(amax / 448), so |x / S| <= 448 still
-holds and x / S is exact; amax == 0 gives S = 1.
+holds and x / S is exact; amax == 0 gives S = 1.  Where the scales are formed
+by the FP8 backward itself (not given as input), a floor keeps them inside
+E8M0's range: S = max(that power of two, 2^-127), so a block of tiny values
+(e.g. a row of dLoss/dlogits whose probabilities underflow) still has a scale
+the MMA takes; x / S stays exact.
 
 Scales are returned in their natural shapes:
   tensor: (1,);  row: (rows,);  act block: (rows, cols/128);
@@ -39,6 +43,7 @@ from . import e4m3
 
 TENSOR, ROWWISE, BLOCK = 0, 1, 2
 ACT, WEIGHT = 0, 1
+E8M0_MIN = 2.0 ** -127  # the smallest E8M0 scale (biased exponent 0)
 BLOCK_K = 128  # block edge along the hidden (reduction) dimension
 BLOCK_W = 128  # block edge of the weight along the vocabulary dimension
 
@@ -64,13 +69,18 @@ def _encode_block(x, s):
     return e4m3.encode(q)
 
 
-def quantize(x, gran, role=ACT, pow2=False):
+def quantize(x, gran, role=ACT, pow2=False, scale_floor=0.0):
     """Quantise a 2-D float32 array (bf16-valued) at the given granularity.
 
     Returns (codes uint8 [rows][cols], scales float32 in natural shape).
-    ``pow2`` selects the power-of-two (UE8M0) scales.
+    ``pow2`` selects the power-of-two (UE8M0) scales; ``scale_floor`` raises
+    every scale below it to it (E8M0_MIN for the backward's own scales).
     """
-    scale_from = pow2_scale_from_amax if pow2 else scale_from_amax
+    base = pow2_scale_from_amax if pow2 else scale_from_amax
+
+    def scale_from(amax):
+        return np.maximum(base(amax), np.float32(scale_floor)).astype(np.float32)
+
     x = np.asarray(x, dtype=np.float32)
     if x.ndim != 2:
         raise ValueError("quantize: 2-D input expected")

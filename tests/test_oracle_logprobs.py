@@ -305,22 +305,24 @@ def _e4m3_abs_err_bound(x, scale_of):
     return np.maximum(2.0 ** -4 * np.abs(x), 2.0 ** -10 * scale_of)
 
 
-@pytest.mark.parametrize("gran", [Q.TENSOR, Q.ROWWISE, Q.BLOCK])
-def test_fp8_backward_within_quantisation_error_of_exact_backward(gran):
+@pytest.mark.parametrize("gran,pow2", [(Q.TENSOR, False), (Q.ROWWISE, False), (Q.BLOCK, False),
+                                       (Q.BLOCK, True)])
+def test_fp8_backward_within_quantisation_error_of_exact_backward(gran, pow2):
     # dh = sum_v P W and dW = sum_t P^T h with every operand quantised: the
     # difference to the exact contraction is bounded term by term by the E4M3
     # rounding of both factors.  A dropped or misplaced scale, a transposed
     # operand or a wrong block index breaks the bound by orders of magnitude.
-    rng = np.random.default_rng(72 + gran)
+    # Power-of-two scales keep |x / S| <= 448, so the same bound holds.
+    rng = np.random.default_rng(72 + gran + 7 * pow2)
     T, H, V = 130, 256, 300
     h = rng.normal(0, 1, (T, H)).astype(np.float32)
     W = (rng.normal(0, 0.05, (V, H))).astype(np.float32)
-    hq, hs = Q.quantize(h, gran, Q.ACT)
-    wq, ws = Q.quantize(W, gran, Q.WEIGHT)
+    hq, hs = Q.quantize(h, gran, Q.ACT, pow2=pow2)
+    wq, ws = Q.quantize(W, gran, Q.WEIGHT, pow2=pow2)
     y = rng.integers(0, V, T)
     g = rng.normal(0, 1, T) / T
     ref = L.lm_head_backward(hq, hs, wq, ws, gran, y, g, h, W)
-    out = L.lm_head_backward_fp8(hq, hs, wq, ws, gran, y, g, h, W)
+    out = L.lm_head_backward_fp8(hq, hs, wq, ws, gran, y, g, h, W, pow2=pow2)
     P = out["P"].astype(np.float64)
     # per-element scales of each quantised operand
     sp = np.repeat(out["p_scales"], 128, axis=1)[:, :V]
@@ -355,3 +357,59 @@ def test_fp8_backward_zero_gradient():
     # every block of P is zero: scale 1, codes +-0 (g * -p is -0.0)
     assert np.all(out["p_scales"] == 1.0) and np.all((out["p_codes"] & 0x7F) == 0)
     assert not np.any(out["P_hat"]) and not np.any(out["Pt_hat"])
+
+
+def _is_pow2(s):
+    m, _ = np.frexp(np.asarray(s, np.float64))
+    return np.all(m == 0.5)
+
+
+def test_fp8_backward_pow2_scales_by_brute_force():
+    # The UE8M0 variant's backward: each operand's scale, found block by block
+    # with Python loops over the unquantised operand, is the smallest power of
+    # two S with amax / 448 <= S (S = 1 for a zero block), raised to 2^-127
+    # where it falls below E8M0's range; the codes are RNE(x / S).  Row 0 has
+    # g = 1e-41, so its P underflows far below 448 * 2^-127 and takes the floor.
+    rng = np.random.default_rng(74)
+    T, H, V = 130, 256, 200
+    h = rng.normal(0, 1, (T, H)).astype(np.float32)
+    W = rng.normal(0, 0.05, (V, H)).astype(np.float32)
+    hq, hs = Q.quantize(h, Q.BLOCK, Q.ACT, pow2=True)
+    wq, ws = Q.quantize(W, Q.BLOCK, Q.WEIGHT, pow2=True)
+    y = rng.integers(0, V, T)
+    g = rng.normal(0, 1, T) / T
+    g[0] = 1e-41
+    g[5] = 0.0
+    out = L.lm_head_backward_fp8(hq, hs, wq, ws, Q.BLOCK, y, g, h, W, pow2=True)
+    P = out["P"].astype(np.float64)
+
+    def expected_scale(block):
+        amax = float(np.max(np.abs(block))) if block.size else 0.0
+        if amax == 0.0:
+            return 1.0
+        t = float(np.float32(np.float32(amax) / np.float32(448.0)))
+        s = 2.0 ** -149
+        while s < t:
+            s *= 2.0
+        return max(s, 2.0 ** -127)
+
+    for t in range(T):
+        for b in range(out["p_scales"].shape[1]):
+            blk = P[t, 128 * b:128 * b + 128]
+            assert out["p_scales"][t, b] == expected_scale(blk), (t, b)
+    for vb in range(out["pt_scales"].shape[0]):
+        for tb in range(out["pt_scales"].shape[1]):
+            blk = P.T[128 * vb:128 * vb + 128, 128 * tb:128 * tb + 128]
+            assert out["pt_scales"][vb, tb] == expected_scale(blk), (vb, tb)
+    for hb in range(out["wt_scales"].shape[0]):
+        for vb in range(out["wt_scales"].shape[1]):
+            assert out["wt_scales"][hb, vb] == expected_scale(W.T[128 * hb:128 * hb + 128, 128 * vb:128 * vb + 128])
+    assert out["p_scales"][0, y[0] // 128] == 2.0 ** -127 and P[0, y[0]] != 0
+    assert np.all(out["p_scales"][5] == 1.0)
+    for k in ("p_scales", "pt_scales", "wt_scales", "ht_scales"):
+        assert _is_pow2(out[k]) and np.all(out[k] >= 2.0 ** -127), k
+    # codes: RNE(x / S) with x / S exact (S a power of two)
+    sp = np.repeat(out["p_scales"], 128, axis=1)[:, :V]
+    q = (P / sp).astype(np.float32)
+    assert np.array_equal(out["p_codes"][:, :V], e4m3.encode(q))
+    assert np.array_equal(out["P_hat"], e4m3.decode(e4m3.encode(q)) * sp)
