@@ -368,7 +368,6 @@ def run_ours(args, rank, world, local_rank):
         ue_stage /= args.steps
         ue = {"ms_per_step": u0.elapsed_time(u1) / args.steps, "gemm_ms": ue_stage[2],
               "quantize_ms": ue_stage[0] + ue_stage[1]}
-        del b3
 
     # the BF16 shadow pass on its own (same inputs; the paper reruns it every
     # 20 steps, so it is reported separately and amortised)
@@ -384,28 +383,35 @@ def run_ours(args, rank, world, local_rank):
 
     # backward through the lm_head from this step's g (dh = P W, dW = P^T h with
     # P = dLoss/dlogits recomputed from the FP8 logits), timed on its own
-    bwd = None
+    bwd = ue_bwd = None
     if not args.no_backward:
         bws = torch.empty(api.lib.fp8rl_lm_head_backward_workspace_size(T, H, V), dtype=torch.uint8, device=dev)
         bout = {"dh": torch.empty(T, H, device=dev), "dW": torch.empty(V, H, device=dev)}
 
-        def backward():
-            api.lm_head_backward(b.h_codes, b.h_scales, b.w_codes, b.w_scales, gran, y, b.lse, b.grad, h, W,
-                                 out=bout, workspace=bws)
+        def time_backward(bb, g):
+            def backward():
+                api.lm_head_backward(bb.h_codes, bb.h_scales, bb.w_codes, bb.w_scales, g, y, bb.lse, bb.grad,
+                                     h, W, out=bout, workspace=bws)
 
-        backward()
-        torch.cuda.synchronize()
-        n_bwd = 3
-        b0 = torch.cuda.Event(enable_timing=True)
-        b1 = torch.cuda.Event(enable_timing=True)
-        b0.record(stream)
-        for _ in range(n_bwd):
             backward()
-        b1.record(stream)
-        torch.cuda.synchronize()
-        api.check()
-        bwd = {"ms": b0.elapsed_time(b1) / n_bwd, "workspace_gb": bws.numel() / 1e9}
+            torch.cuda.synchronize()
+            n_bwd = 3
+            b0 = torch.cuda.Event(enable_timing=True)
+            b1 = torch.cuda.Event(enable_timing=True)
+            b0.record(stream)
+            for _ in range(n_bwd):
+                backward()
+            b1.record(stream)
+            torch.cuda.synchronize()
+            api.check()
+            return {"ms": b0.elapsed_time(b1) / n_bwd, "workspace_gb": bws.numel() / 1e9}
+
+        bwd = time_backward(b, gran)
+        if ue is not None:  # the variant's backward: power-of-two scales throughout
+            ue_bwd = time_backward(b3, api.GRAN_BLOCK_UE8M0)
         del bws, bout
+    if ue is not None:
+        del b3
     api.check()
 
     # same step through the public API with host buffers (copies inside the region)
@@ -540,6 +546,13 @@ def run_ours(args, rank, world, local_rank):
             "note": "the same step with power-of-two block scales (fp8rl_quantize_ue8m0, 1x128 / 128x128) "
                     "applied by tcgen05.mma kind::mxf8f6f4 with E8M0 scale factors in tensor memory; a "
                     "variant outside the paper (its scales are amax / 448), so not the headline value"}
+        if ue_bwd is not None:
+            ideal_ms = 3 * flops / (fp8_peak * 1e12) * 1e3
+            line["ue8m0_mma_variant"]["lm_head_backward"] = {
+                "ms": ue_bwd["ms"], "tflops": 3 * flops / (ue_bwd["ms"] * 1e-3) / 1e12,
+                "frac_of_roofline": ideal_ms / ue_bwd["ms"],
+                "note": "the variant's backward: P, P^T, W^T and h^T with power-of-two scales, the recompute "
+                        "and both contractions on the block-scaled MMA"}
     if bwd is not None:
         ideal_ms = 3 * flops / (fp8_peak * 1e12) * 1e3
         bwd.update({"tflop_per_call": 3 * flops / 1e12, "tflops": 3 * flops / (bwd["ms"] * 1e-3) / 1e12,

@@ -14,7 +14,13 @@
 //      [H][V'] and h^T [H][T'] with 128 x 128 scales (V', T' = V, T rounded
 //      up to 128; the padding holds zero codes);
 //   3. the block-scaled FP8 GEMM forms dh and dW into float32.
+// With power-of-two forward scales (the UE8M0 variant) the backward keeps that
+// format: P, P^T, W^T and h^T take power-of-two scales (floored at 2^-127),
+// and the recompute and both contractions run on the block-scaled MMA
+// (tcgen05.mma kind::mxf8f6f4), which applies them per 32-wide K step.
 #include <cuda_fp8.h>
+
+#include <algorithm>
 
 #include "common.cuh"
 #include "e4m3_encode.cuh"
@@ -28,15 +34,17 @@ __device__ uint32_t d_status;
 constexpr int kQT = 128;  // edge of a quantisation block / transpose tile
 
 // codes[c][r] = Q_FP8(in[r][c] / S) for one 128 x 128 tile of the bf16 matrix
-// in[rows][cols]: S = fl32(amax / 448) over the tile (1 when it is all zero),
-// written to scales[c / 128][r / 128] (row stride ld_out / 128).  The tile goes
+// in[rows][cols]: S = fl32(amax / 448) over the tile (1 when it is all zero;
+// with pow2 the power of two above it, floored at 2^-127), written to
+// scales[c / 128][r / 128] (row stride ld_out / 128).  The tile goes
 // through shared memory (row pitch 136 bf16, so column reads by a warp hit
 // distinct banks); each thread encodes 64 codes of one output row.  Rows of
 // `in` past `rows` read as zero, so the padding columns of the codes are zero.
 __global__ void __launch_bounds__(256) transpose_quantize_kernel(const uint16_t* __restrict__ in, int64_t rows,
                                                                  int64_t cols, int64_t ld_in,
                                                                  uint8_t* __restrict__ codes,
-                                                                 float* __restrict__ scales, int64_t ld_out) {
+                                                                 float* __restrict__ scales, int64_t ld_out,
+                                                                 int pow2) {
   constexpr int kPitch = kQT + 8;
   __shared__ __align__(16) uint16_t tile[kQT][kPitch];
   __shared__ uint32_t warp_max[8];
@@ -64,7 +72,7 @@ __global__ void __launch_bounds__(256) transpose_quantize_kernel(const uint16_t*
   uint32_t bm = warp_max[0];
 #pragma unroll
   for (int i = 1; i < 8; ++i) bm = max(bm, warp_max[i]);
-  const float s = e4m3_scale(__uint_as_float(bm), false);
+  const float s = pow2 ? e8m0_floor(e4m3_scale(__uint_as_float(bm), true)) : e4m3_scale(__uint_as_float(bm), false);
   const E4M3Enc e = e4m3_encoder(s);
   // output row c = tid / 2 (column c of the tile), codes r = 64 (tid % 2) ..
   const int c = tid >> 1, rh = (tid & 1) * 64;
@@ -110,7 +118,10 @@ BwdLayout bwd_layout(int64_t T, int64_t H, int64_t V) {
   l.wts = take(static_cast<size_t>(hb) * (l.vp / kQT) * 4);
   l.ht = take(static_cast<size_t>(H) * l.tp);
   l.hts = take(static_cast<size_t>(hb) * (l.tp / kQT) * 4);
-  l.sf = take(gemm_ue8m0_image_bytes(T, V, H));  // UE8M0 recompute only
+  // UE8M0 variant: scale images of the recompute, then of dh, then of dW
+  // (one buffer: the three GEMMs run in stream order)
+  l.sf = take(std::max({gemm_ue8m0_image_bytes(T, V, H), gemm_ue8m0_image_bytes(T, H, l.vp),
+                        gemm_ue8m0_image_bytes(V, H, l.tp)}));
   l.total = off;
   return l;
 }
@@ -130,6 +141,9 @@ cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const ui
   float* Wts = reinterpret_cast<float*>(base + l.wts);
   uint8_t* Htq = reinterpret_cast<uint8_t*>(base + l.ht);
   float* Hts = reinterpret_cast<float*>(base + l.hts);
+  const bool ue = gran == FP8RL_GRAN_BLOCK_UE8M0;
+  const int bgran = ue ? FP8RL_GRAN_BLOCK_UE8M0 : FP8RL_GRAN_BLOCK;
+  uint8_t* sf = reinterpret_cast<uint8_t*>(base + l.sf);
   // 1. recompute z (FP8), quantise P = dLoss/dz in both orientations
   GemmArgs a{};
   a.a_codes = hc;
@@ -149,18 +163,19 @@ cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const ui
   a.ptq_scales = Pts;
   a.ld_pq = l.vp;
   a.ld_ptq = l.tp;
-  a.sf_images = reinterpret_cast<uint8_t*>(base + l.sf);
+  a.sf_images = sf;
   cudaError_t e = launch_gemm_dense_dlogits(a, s);
   if (e != cudaSuccess) return e;
   if (dh) {  // 2./3. dh[T][H] = P[T][V'] . (W^T[H][V'])^T
-    e = launch_transpose_quantize(W, V, H, H, Wtq, Wts, l.vp, s);
+    e = launch_transpose_quantize(W, V, H, H, Wtq, Wts, l.vp, ue, s);
     if (e != cudaSuccess) return e;
     GemmArgs d{};
     d.a_codes = Pq;
     d.a_scales = Ps;
     d.b_codes = Wtq;
     d.b_scales = Wts;
-    d.gran = FP8RL_GRAN_BLOCK;
+    d.gran = bgran;
+    d.sf_images = sf;
     d.M = T;
     d.N = H;
     d.K = l.vp;
@@ -172,14 +187,15 @@ cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const ui
     if (e != cudaSuccess) return e;
   }
   if (dW) {  // dW[V][H] = P^T[V][T'] . (h^T[H][T'])^T
-    e = launch_transpose_quantize(h, T, H, H, Htq, Hts, l.tp, s);
+    e = launch_transpose_quantize(h, T, H, H, Htq, Hts, l.tp, ue, s);
     if (e != cudaSuccess) return e;
     GemmArgs d{};
     d.a_codes = Ptq;
     d.a_scales = Pts;
     d.b_codes = Htq;
     d.b_scales = Hts;
-    d.gran = FP8RL_GRAN_BLOCK;
+    d.gran = bgran;
+    d.sf_images = sf;
     d.M = V;
     d.N = H;
     d.K = l.tp;
@@ -194,13 +210,14 @@ cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const ui
 }
 
 cudaError_t launch_transpose_quantize(const uint16_t* in, int64_t rows, int64_t cols, int64_t ld_in,
-                                      uint8_t* codes, float* scales, int64_t ld_out, cudaStream_t s) {
+                                      uint8_t* codes, float* scales, int64_t ld_out, bool pow2,
+                                      cudaStream_t s) {
   if (rows == 0 || cols == 0) return cudaSuccess;
   if (cols % 8 != 0 || ld_in % 8 != 0 || ld_out % kQT != 0 || ld_out < rows) return cudaErrorInvalidValue;
   const int64_t gx = ld_out / kQT, gy = (cols + kQT - 1) / kQT;
   if (gx > 0x7FFFFFFF || gy > 65535) return cudaErrorInvalidValue;
   transpose_quantize_kernel<<<dim3(static_cast<unsigned>(gx), static_cast<unsigned>(gy)), 256, 0, s>>>(
-      in, rows, cols, ld_in, codes, scales, ld_out);
+      in, rows, cols, ld_in, codes, scales, ld_out, pow2 ? 1 : 0);
   return cudaGetLastError();
 }
 

@@ -70,6 +70,13 @@ __device__ __forceinline__ float pow2_ceil(float t) {
   return man == (1u << h) ? t : __uint_as_float(1u << (h + 1));
 }
 
+// A power-of-two scale that the FP8 backward forms itself, raised to 2^-127
+// (E8M0's smallest scale, a float32 subnormal) where it falls below; s >= 0
+// or NaN, which stays NaN.
+__device__ __forceinline__ float e8m0_floor(float s) {
+  return __float_as_uint(s) < 0x00400000u ? __uint_as_float(0x00400000u) : s;
+}
+
 // S = fl32(amax / 448), 1 when amax == 0 (an all-zero block keeps S = 1);
 // with pow2 (UE8M0 scales) rounded up to a power of two, so that |x / S|
 // stays within 448 and x / S is exact.

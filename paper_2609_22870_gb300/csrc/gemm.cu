@@ -206,12 +206,19 @@ __device__ __forceinline__ float fmax_nan(float a, float b) {
 //   codes of P with the 128 x 128 block scale of the tile half (the max over
 //   the four warps holding its 128 rows, exchanged through shared memory
 //   with a bounded wait), stored transposed         -> ptq_out / ptq_scales
-// Rows past M and columns past N hold 0 (the K padding of the contractions).
-// Returns false if the exchange wait expired.
+// With pow2 (the UE8M0 variant) both scales are rounded up to powers of two
+// and floored at 2^-127, the scale format of the block-scaled MMA that runs
+// the contractions.  Rows past M and columns past N hold 0 (the K padding of
+// the contractions).  Returns false if the exchange wait expired.
+__device__ __forceinline__ float p_scale(float amax, bool pow2) {
+  const float s = scale_of(amax);
+  return pow2 ? e8m0_floor(pow2_ceil(s)) : s;
+}
+
 __device__ __forceinline__ bool dense_fp8_epilogue(const Params& p, const EpiState& es, float* z, int row,
                                                    int col0, int m_blk, int rit, int half, int quarter,
                                                    int lane, int tcount, uint64_t* blk_bar, uint32_t* blk_max,
-                                                   uint64_t lim, const volatile int* abort_flag) {
+                                                   uint64_t lim, const volatile int* abort_flag, bool pow2) {
   const int ncol = min(CHUNK, p.N - col0);
   const bool row_ok = row < p.M;
   const float g = es.g;
@@ -237,7 +244,7 @@ __device__ __forceinline__ bool dense_fp8_epilogue(const Params& p, const EpiSta
   }
   uint32_t w[32];
   if (row_ok && col0 < p.ld_pq) {  // the row's block along N (K of the dh contraction)
-    const float s = scale_of(amax);
+    const float s = p_scale(amax, pow2);
     encode128(z, s, w);
     uint4* dst = reinterpret_cast<uint4*>(p.pq_out + static_cast<size_t>(row) * p.ld_pq + col0);
 #pragma unroll
@@ -258,7 +265,7 @@ __device__ __forceinline__ bool dense_fp8_epilogue(const Params& p, const EpiSta
   if (!__all_sync(0xffffffffu, mbar_wait(bar, par, lim, abort_flag))) return false;
   const uint32_t bmax = max(max(bm[0], bm[1]), max(bm[2], bm[3]));
   if (ncol <= 0) return true;
-  const float sb = scale_of(__uint_as_float(bmax));
+  const float sb = p_scale(__uint_as_float(bmax), pow2);
   encode128(z, sb, w);
   // lanes are consecutive tokens; a 4 x 4 byte transpose within each group of
   // four lanes (two exchanges) leaves lane 4a + j with column 4k + j of rows
@@ -621,7 +628,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         float* z = reinterpret_cast<float*>(z2);
         if (EPI == kEpiDenseFp8) {
           ok = dense_fp8_epilogue(p, es, z, row, col0, m_blk, rit, half, quarter, lane, tcount, blk_bar, blk_max,
-                                  lim, abort_flag);
+                                  lim, abort_flag, MODE == kUe8m0);
           if (!ok) break;
         } else {
           epi_consume128<EPI>(p, es, z, row, col0);
@@ -643,7 +650,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         aphase ^= 1;
         if (EPI == kEpiDenseFp8) {
           ok = dense_fp8_epilogue(p, es, zf, row, col0, m_blk, rit, half, quarter, lane, tcount, blk_bar, blk_max,
-                                  lim, abort_flag);
+                                  lim, abort_flag, MODE == kUe8m0);
           if (!ok) break;
         } else {
           epi_consume128<EPI>(p, es, zf, row, col0);
@@ -678,7 +685,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         ab ^= 1;
         if (ab == 0) aphase ^= 1;
         ok = dense_fp8_epilogue(p, es, zf, row, col0, m_blk, rit, half, quarter, lane, tcount, blk_bar, blk_max,
-                                lim, abort_flag);
+                                lim, abort_flag, MODE == kUe8m0);
         if (!ok) break;
       } else {
         ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&acc_full[ab]), aphase, lim, abort_flag));
@@ -938,9 +945,10 @@ cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s) {
   }
   const int64_t tiles = static_cast<int64_t>(p.num_m) * p.num_n;
   const int grid = static_cast<int>(tiles < sm_count() ? tiles : sm_count());
-  if constexpr (EPI == kEpiStore) {  // plain fp32 store: block-scaled FP8 (backward) or BF16
+  if constexpr (EPI == kEpiStore) {  // plain fp32 store: block-scaled FP8 (backward, both scale formats) or BF16
     switch (a.gran) {
       case kBlock: return launch_mode<kBlock, EPI>(ta, tb, p, grid, s);
+      case kUe8m0: return launch_mode<kUe8m0, EPI>(ta, tb, p, grid, s);
       case kBf16: return launch_mode<kBf16, EPI>(ta, tb, p, grid, s);
       default: return cudaErrorInvalidValue;
     }

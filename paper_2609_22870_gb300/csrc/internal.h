@@ -78,9 +78,11 @@ cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const ui
                                     int accumulate_dw, void* ws, cudaStream_t s);
 // codes [cols][ld_out] of the transposed bf16 matrix in [rows][ld_in] with
 // 128 x 128 E4M3 blocks, scales [ceil(cols/128)][ld_out/128]; columns
-// rows .. ld_out-1 of the codes are zero (ld_out a multiple of 128, >= rows)
+// rows .. ld_out-1 of the codes are zero (ld_out a multiple of 128, >= rows);
+// pow2: power-of-two scales floored at 2^-127
 cudaError_t launch_transpose_quantize(const uint16_t* in, int64_t rows, int64_t cols, int64_t ld_in,
-                                      uint8_t* codes, float* scales, int64_t ld_out, cudaStream_t s);
+                                      uint8_t* codes, float* scales, int64_t ld_out, bool pow2,
+                                      cudaStream_t s);
 uint32_t backward_status_take();
 cudaError_t launch_combine(const float2* partials, const float* zy, const int32_t* targets,
                            const float* logp_old, float* logp, float* lse, float* ratio,

@@ -34,11 +34,13 @@ def bf16_strip(args):
 
 def bwd_dh_strip(args):
     """Partial dh of the FP8 backward over one vocabulary strip: the oracle
-    quantises the strip of W with 128 x 128 blocks (the blocks of W^T), and
-    returns (P_hat[:, strip] @ W_hat_strip, |P_hat[:, strip]| @ |W_hat_strip|,
-    slack[:, strip] @ |W_hat_strip|) in float64."""
-    p_hat, slack, w_strip = args
-    wq, ws = OQ.quantize(w_strip, OQ.BLOCK, OQ.WEIGHT)
+    quantises the strip of W with 128 x 128 blocks (the blocks of W^T; with
+    pow2 the power-of-two scales of the UE8M0 variant, floored at 2^-127),
+    and returns (P_hat[:, strip] @ W_hat_strip, |P_hat[:, strip]| @
+    |W_hat_strip|, slack[:, strip] @ |W_hat_strip|) in float64."""
+    p_hat, slack, w_strip, pow2 = args
+    kw = {"pow2": True, "scale_floor": OQ.E8M0_MIN} if pow2 else {}
+    wq, ws = OQ.quantize(w_strip, OQ.BLOCK, OQ.WEIGHT, **kw)
     wd = OQ.dequantize(wq, ws, OQ.BLOCK, OQ.WEIGHT)
     aw = np.abs(wd)
     return p_hat @ wd, np.abs(p_hat) @ aw, slack @ aw

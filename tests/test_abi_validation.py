@@ -43,12 +43,15 @@ def test_lm_head_backward_workspace_size(api):
         return (x + a - 1) // a * a
     vp, tp, hb = up(V, 128), up(T, 128), up(H, 128) // 128
     # E4M3 codes and float scales of P [T][V'], P^T [V][T'], W^T [H][V'], h^T [H][T'],
-    # then the E8M0 scale images of a UE8M0 recompute: 512 bytes per 128 tokens,
-    # 1024 per 256 vocabulary rows, for each group of four 128-wide K blocks
-    kg = (hb + 3) // 4
+    # then the E8M0 scale images of the UE8M0 variant's GEMMs (512 bytes per 128
+    # rows of A, 1024 per 256 rows of B, for each group of four 128-wide K
+    # blocks), one buffer for the largest of the three: recompute (M T, N V,
+    # K H), dh (T, H, V'), dW (V, H, T')
+    def images(M, N, K):
+        return (up(M, 128) // 128 * 512 + up(N, 256) // 256 * 1024) * ((up(K, 128) // 128 + 3) // 4)
     parts = [T * vp, (vp // 128) * T * 4, V * tp, (tp // 128) * V * 4,
              H * vp, hb * (vp // 128) * 4, H * tp, hb * (tp // 128) * 4,
-             (up(T, 128) // 128 * 512 + up(V, 256) // 256 * 1024) * kg]
+             max(images(T, V, H), images(T, H, vp), images(V, H, tp))]
     want = sum(up(p, 256) for p in parts)
     assert api.lib.fp8rl_lm_head_backward_workspace_size(T, H, V) == want  # 5.72 GB
     assert api.lib.fp8rl_lm_head_backward_workspace_size(0, H, V) == 0

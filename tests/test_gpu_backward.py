@@ -60,22 +60,54 @@ def _flip_slack(x, s):
     return np.abs(hi - lo) * np.asarray(s, np.float64)
 
 
+def _pow2_flip_slack(x, block_rows):
+    """Power-of-two scales (the UE8M0 variant): where a block's amax / 448
+    lies within 2^-17 of a power of two, the two sides may pick scales a factor
+    of two apart and every code of the block may differ; there each element
+    may be off by the E4M3 rounding error at both scales (2 max(2^-4 |x|,
+    2^-10 S) with S the larger).  Blocks are block_rows x 128 of x (R, C),
+    C a multiple of 128; 0 elsewhere."""
+    x = np.abs(np.asarray(x, np.float64))
+    R, C = x.shape
+    out = np.zeros_like(x)
+    d = 2.0 ** -17
+    for r0 in range(0, R, block_rows):
+        for c0 in range(0, C, 128):
+            blk = x[r0:r0 + block_rows, c0:c0 + 128]
+            t = float(np.float32(np.float32(blk.max()) / np.float32(448.0))) if blk.size else 0.0
+            if t == 0.0:
+                continue
+            lo, hi = np.ceil(np.log2(t * (1 - d))), np.ceil(np.log2(t * (1 + d)))
+            if lo != hi:
+                out[r0:r0 + block_rows, c0:c0 + 128] = 2 * np.maximum(2.0 ** -4 * blk, 2.0 ** -10 * 2.0 ** hi)
+    return out
+
+
 def _oracle(h, W, y, g, gran):
+    pow2 = gran == UE
+    og = OQ.BLOCK if pow2 else gran
     h32, W32 = h.float().cpu().numpy(), W.float().cpu().numpy()
-    hq, hs = OQ.quantize(h32, gran, OQ.ACT)
-    wq, ws = OQ.quantize(W32, gran, OQ.WEIGHT)
-    ref = OL.lm_head_backward_fp8(hq, hs, wq, ws, gran, y.cpu().numpy(), g.cpu().numpy(), h32, W32)
+    hq, hs = OQ.quantize(h32, og, OQ.ACT, pow2=pow2)
+    wq, ws = OQ.quantize(W32, og, OQ.WEIGHT, pow2=pow2)
+    ref = OL.lm_head_backward_fp8(hq, hs, wq, ws, og, y.cpu().numpy(), g.cpu().numpy(), h32, W32, pow2=pow2)
     T, V = ref["P"].shape
     P = ref["P"].astype(np.float64)
     sp = np.repeat(ref["p_scales"], 128, axis=1)[:, :V]
     spt = np.repeat(np.repeat(ref["pt_scales"], 128, axis=0), 128, axis=1)[:V, :T]
     aw, ah = np.abs(ref["Wt_hat"]).T, np.abs(ref["ht_hat"]).T  # (V, H), (T, H)
-    bound_dh = REL * (np.abs(ref["P_hat"]) @ aw) + _flip_slack(P, sp) @ aw
-    bound_dW = REL * (np.abs(ref["Pt_hat"]) @ ah) + _flip_slack(P.T, spt) @ ah
+    slack_p, slack_pt = _flip_slack(P, sp), _flip_slack(P.T, spt)
+    if pow2:
+        slack_p = slack_p + _pow2_flip_slack(OL._pad_cols(ref["P"]), 1)[:, :V]
+        slack_pt = slack_pt + _pow2_flip_slack(OL._pad_cols(ref["P"].T), 128)[:, :T]
+    bound_dh = REL * (np.abs(ref["P_hat"]) @ aw) + slack_p @ aw
+    bound_dW = REL * (np.abs(ref["Pt_hat"]) @ ah) + slack_pt @ ah
     return ref, bound_dh, bound_dW
 
 
-@pytest.mark.parametrize("gran", [OQ.TENSOR, OQ.ROWWISE, OQ.BLOCK])
+UE = 3  # power-of-two block scales on the block-scaled MMA (forward and backward)
+
+
+@pytest.mark.parametrize("gran", [OQ.TENSOR, OQ.ROWWISE, OQ.BLOCK, UE])
 @pytest.mark.parametrize("T,H,V", [(300, 256, 1000), (129, 384, 1001), (1, 128, 1), (520, 128, 4096)])
 def test_backward_small_all_elements(cuda_lib, gran, T, H, V):
     h, W, y, g = _data(T, H, V, T + V)
@@ -118,10 +150,11 @@ def test_backward_accumulate_chunks_and_single_outputs(cuda_lib):
         api.lm_head_backward(hc, hs, wc, ws, gran, y, lse, g, h, W, want_dh=False, want_dw=False)
 
 
-@pytest.mark.parametrize("gran", [OQ.BLOCK, OQ.TENSOR])
+@pytest.mark.parametrize("gran", [OQ.BLOCK, OQ.TENSOR, UE])
 def test_backward_full_size_grpo8b(cuda_lib, gran):
     """grpo_8b (T 16384, H 4096, V 151936): 64 sampled rows of dh against the
-    oracle's FP8 backward; dW by bounded column sums."""
+    oracle's FP8 backward; dW by bounded column sums.  UE: power-of-two scales
+    on every operand, the contractions on the block-scaled MMA."""
     api = cuda_lib
     w = synth.WORKLOADS["grpo_8b"]
     h, W, y = synth.hidden_states(w, "cuda"), synth.lm_head_weight(w, "cuda"), synth.targets(w, "cuda")
@@ -130,13 +163,17 @@ def test_backward_full_size_grpo8b(cuda_lib, gran):
     dh = out["dh"]
     assert bool(torch.isfinite(dh).all()) and bool(torch.isfinite(out["dW"]).all())
     rows = sample_rows(w.T, 60, 9)
-    _, lse_r, z_r = oracle_logprobs_rows(h, W, gran, y, rows)
+    pow2 = gran == UE
+    _, lse_r, z_r = oracle_logprobs_rows(h, W, OQ.BLOCK if pow2 else gran, y, rows, pow2=pow2)
     P = OL.dlogits(z_r, y.cpu().numpy()[rows], lse_r, g.cpu().numpy()[rows]).astype(np.float32)
     Pp = OL._pad_cols(P)
-    pq, ps = OQ.quantize(Pp, OQ.BLOCK, OQ.ACT)
+    kw = {"pow2": True, "scale_floor": OQ.E8M0_MIN} if pow2 else {}
+    pq, ps = OQ.quantize(Pp, OQ.BLOCK, OQ.ACT, **kw)
     p_hat = OQ.dequantize(pq, ps, OQ.BLOCK, OQ.ACT)
     slack = _flip_slack(Pp, np.repeat(ps, 128, axis=1))
-    tasks = ((p_hat[:, v0:v0 + wx.shape[0]], slack[:, v0:v0 + wx.shape[0]], wx)
+    if pow2:
+        slack = slack + _pow2_flip_slack(Pp, 1)
+    tasks = ((p_hat[:, v0:v0 + wx.shape[0]], slack[:, v0:v0 + wx.shape[0]], wx, pow2)
              for v0, wx in _w_strips(W, POOL_STRIP))
     ref = np.zeros((len(rows), w.H))
     mag = np.zeros_like(ref)

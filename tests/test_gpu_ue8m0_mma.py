@@ -85,9 +85,10 @@ def test_ue8m0_mma_bit_reproducible(cuda_lib):
     assert torch.equal(a["logp"], b["logp"]) and torch.equal(a["lse"], b["lse"])
 
 
-def test_ue8m0_mma_dlogits_and_backward(cuda_lib):
-    """Dense dlogits rows and the FP8 backward run on the hardware-scaled
-    recompute too; against the promotion path on the same codes."""
+def test_ue8m0_mma_dlogits_rows(cuda_lib):
+    """Dense dlogits rows run on the hardware-scaled recompute too (the
+    variant's backward is checked against the oracle with the other backward
+    tests)."""
     api = cuda_lib
     T, H, V = 300, 256, 1100
     h, W, y = _data(T, H, V, 93)
@@ -102,12 +103,6 @@ def test_ue8m0_mma_dlogits_and_backward(cuda_lib):
     ref = OL.dlogits(z, y.cpu().numpy()[r], ref_lse, g.cpu().numpy()[r])
     gg = np.abs(g.cpu().numpy()[r])[:, None]
     assert np.all(np.abs(d.cpu().numpy() - ref) <= TOL * gg + 1e-12)
-    b_ue = api.lm_head_backward(hc, hs, wc, ws, UE, y, fwd["lse"], g, h, W)
-    b_bl = api.lm_head_backward(hc, hs, wc, ws, api.GRAN_BLOCK, y, fwd["lse"], g, h, W)
-    api.check()
-    for k in ("dh", "dW"):
-        scale = b_bl[k].abs().max().item()
-        assert (b_ue[k] - b_bl[k]).abs().max().item() <= 2.0 ** -6 * scale, k
 
 
 def test_ue8m0_mma_rejects_scales_that_are_not_powers_of_two(cuda_lib):
