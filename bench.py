@@ -388,10 +388,10 @@ def run_ours(args, rank, world, local_rank):
         bws = torch.empty(api.lib.fp8rl_lm_head_backward_workspace_size(T, H, V), dtype=torch.uint8, device=dev)
         bout = {"dh": torch.empty(T, H, device=dev), "dW": torch.empty(V, H, device=dev)}
 
-        def time_backward(bb, g):
+        def time_backward(bb, g, pow2=False):
             def backward():
                 api.lm_head_backward(bb.h_codes, bb.h_scales, bb.w_codes, bb.w_scales, g, y, bb.lse, bb.grad,
-                                     h, W, out=bout, workspace=bws)
+                                     h, W, pow2_scales=pow2, out=bout, workspace=bws)
 
             backward()
             torch.cuda.synchronize()
@@ -407,6 +407,8 @@ def run_ours(args, rank, world, local_rank):
             return {"ms": b0.elapsed_time(b1) / n_bwd, "workspace_gb": bws.numel() / 1e9}
 
         bwd = time_backward(b, gran)
+        if gran != api.GRAN_BLOCK_UE8M0:  # the backward's own operands on power-of-two scales
+            bwd["pow2_scales"] = time_backward(b, gran, pow2=True)
         if ue is not None:  # the variant's backward: power-of-two scales throughout
             ue_bwd = time_backward(b3, api.GRAN_BLOCK_UE8M0)
         del bws, bout
@@ -561,6 +563,12 @@ def run_ours(args, rank, world, local_rank):
                             "epilogue writes dlogits as E4M3 codes (1x128 along V, and 128x128 transposed), "
                             "W and h transposed and quantised (128x128), dh and dW on the block-scaled FP8 "
                             "GEMM; ideal = 6THV at the FP8 burst peak"})
+        if "pow2_scales" in bwd:
+            p2 = bwd["pow2_scales"]
+            p2.update({"tflops": 3 * flops / (p2["ms"] * 1e-3) / 1e12, "frac_of_roofline": ideal_ms / p2["ms"],
+                       "note": "FP8RL_BWD_POW2_SCALES: z recomputed from this step's codes as above, P, P^T, W^T "
+                               "and h^T with power-of-two scales (floored at 2^-127), dh and dW on the "
+                               "block-scaled MMA (kind::mxf8f6f4)"})
         line["lm_head_backward"] = bwd
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = oracle_step_estimate(w, budget_s=args.cpu_budget)

@@ -443,13 +443,20 @@ fp8rl_status fp8rl_dlogits_rows(const uint8_t* h_codes, const float* h_scales,
  * E4M3-quantised (Eq. 3) along its own K axis: P with 1x128 blocks along V
  * (dh), P^T with 128 x 128 blocks (dW), and the transposed bf16 operands
  * w_bf16^T [H][V] and h_bf16^T [H][T] with 128 x 128 blocks; float32
- * accumulation.
+ * accumulation.  The scales of these four operands are amax / 448 (the
+ * paper's format), promoted in registers per 128-wide K block; with
+ * FP8RL_BWD_POW2_SCALES (implied by FP8RL_GRAN_BLOCK_UE8M0) they are rounded
+ * up to powers of two (floored at 2^-127) and both contractions run on the
+ * block-scaled MMA (kind::mxf8f6f4), which applies them in hardware.  The
+ * recompute of z always uses the forward's codes and scales as given.
  *   h_codes ... targets   as for fp8rl_token_logprobs (any granularity)
  *   lse, grad_logp        float [T] DEVICE
  *   h_bf16, w_bf16        bf16 [T][H], [V][H], the operands the codes came from
  *   dh, dW                float out, 16-byte aligned; either may be NULL to
  *                         skip that contraction (not both)
- *   accumulate_dw         nonzero: dW += (several token chunks, one dW)
+ *   flags                 FP8RL_BWD_* bits: ACCUMULATE_DW: dW += (several
+ *                         token chunks, one dW); POW2_SCALES: as above;
+ *                         other bits give FP8RL_EINVAL
  * T and V below 2^31 - 256, else FP8RL_ESHAPE; misaligned h_bf16, w_bf16, dh,
  * dW or workspace give FP8RL_EALIGN; a non-finite h_bf16 or w_bf16 sets
  * FP8RL_EDEVICE.  The workspace holds the codes and scales of the four
@@ -461,6 +468,9 @@ fp8rl_status fp8rl_dlogits_rows(const uint8_t* h_codes, const float* h_scales,
  * and accumulate dW.  Target ids are not checked again here
  * (fp8rl_token_logprobs flags them): an id outside [0, V) adds no one-hot
  * term to its row of P. */
+#define FP8RL_BWD_ACCUMULATE_DW 1
+#define FP8RL_BWD_POW2_SCALES 2
+
 size_t fp8rl_lm_head_backward_workspace_size(int64_t T, int64_t H, int64_t V);
 
 fp8rl_status fp8rl_lm_head_backward(const uint8_t* h_codes, const float* h_scales,
@@ -469,7 +479,7 @@ fp8rl_status fp8rl_lm_head_backward(const uint8_t* h_codes, const float* h_scale
                                     const int32_t* targets, const float* lse,
                                     const float* grad_logp, const void* h_bf16,
                                     const void* w_bf16, float* dh, float* dW,
-                                    int accumulate_dw, void* workspace, size_t workspace_bytes,
+                                    int flags, void* workspace, size_t workspace_bytes,
                                     void* stream);
 
 /* ---------------------------------------------------------------------- */

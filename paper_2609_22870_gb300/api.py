@@ -22,6 +22,7 @@ OK, EINVAL, ESHAPE, EALIGN, EWORKSPACE, ECUDA, EDEVICE, ETIMEOUT = range(8)
 GRAN_TENSOR, GRAN_ROWWISE, GRAN_BLOCK = 0, 1, 2
 # block layout with power-of-two scales, applied by the block-scaled MMA (scoring calls only)
 GRAN_BLOCK_UE8M0 = 3
+BWD_ACCUMULATE_DW, BWD_POW2_SCALES = 1, 2  # fp8rl_lm_head_backward flags
 ROLE_ACT, ROLE_WEIGHT = 0, 1
 CALIB_EXACT, CALIB_GRID = 0, 1
 CLIP_HI, CLIP_LO = 1, 2
@@ -460,11 +461,13 @@ def seq_level_clipped_surrogate(logp, logp_old, adv_seq, seq_id, mask=None, lo=0
 
 
 def lm_head_backward(h_codes, h_scales, w_codes, w_scales, gran, targets, lse, grad_logp, h, W,
-                     want_dh=True, want_dw=True, accumulate_dw=False, out=None, workspace=None, stream=None):
+                     want_dh=True, want_dw=True, accumulate_dw=False, pow2_scales=False, out=None,
+                     workspace=None, stream=None):
     """fp8rl_lm_head_backward -> dict(dh=[T][H] float32, dW=[V][H] float32).
     ``h`` [T][H] and ``W`` [V][H] are the bf16 operands the codes came from;
     ``out`` may hold preallocated "dh" / "dW" (with ``accumulate_dw`` the
-    given dW is added to)."""
+    given dW is added to); ``pow2_scales``: the contractions' operands take
+    power-of-two scales on the block-scaled MMA (FP8RL_BWD_POW2_SCALES)."""
     T, H, V = _gemm_args(h_codes, h_scales, w_codes, w_scales, targets, gran)
     dev = h.device
     _dev(lse, torch.float32, "lse", T)
@@ -480,9 +483,10 @@ def lm_head_backward(h_codes, h_scales, w_codes, w_scales, gran, targets, lse, g
     _dev(dW, torch.float32, "dW", V * H)
     if workspace is None:
         workspace = _workspace(lib.fp8rl_lm_head_backward_workspace_size(T, H, V), dev)
+    flags = (BWD_ACCUMULATE_DW if accumulate_dw else 0) | (BWD_POW2_SCALES if pow2_scales else 0)
     _ok(lib.fp8rl_lm_head_backward(_ptr(h_codes), _ptr(h_scales), _ptr(w_codes), _ptr(w_scales), int(gran),
                                    T, H, V, _ptr(targets), _ptr(lse), _ptr(grad_logp), _ptr(h), _ptr(W),
-                                   _ptr(dh), _ptr(dW), int(bool(accumulate_dw)), _ptr(workspace),
+                                   _ptr(dh), _ptr(dW), flags, _ptr(workspace),
                                    workspace.numel(), _stream(stream)), "fp8rl_lm_head_backward")
     return {"dh": dh, "dW": dW}
 

@@ -461,10 +461,11 @@ fp8rl_status fp8rl_lm_head_backward(const uint8_t* hc, const float* hs, const ui
                                     const float* wsc, fp8rl_gran g, int64_t T, int64_t H, int64_t V,
                                     const int32_t* targets, const float* lse, const float* grad,
                                     const void* h_bf16, const void* w_bf16, float* dh, float* dW,
-                                    int accumulate_dw, void* ws, size_t ws_bytes, void* stream) {
+                                    int flags, void* ws, size_t ws_bytes, void* stream) {
   fp8rl_status st = check_gemm_shape(hc, hs, wc, wsc, g, T, H, V);
   if (st != FP8RL_OK) return st;
   if (!targets || !lse || !grad || !h_bf16 || !w_bf16 || (!dh && !dW)) return FP8RL_EINVAL;
+  if (flags & ~(FP8RL_BWD_ACCUMULATE_DW | FP8RL_BWD_POW2_SCALES)) return FP8RL_EINVAL;
   if (T > kMaxBwdRows || V > kMaxBwdRows) return FP8RL_ESHAPE;
   if (!aligned16(h_bf16) || !aligned16(w_bf16) || (dh && !aligned16(dh)) || (dW && !aligned16(dW)))
     return FP8RL_EALIGN;
@@ -472,7 +473,9 @@ fp8rl_status fp8rl_lm_head_backward(const uint8_t* hc, const float* hs, const ui
   if (!aligned16(ws)) return FP8RL_EALIGN;
   cudaError_t e = launch_lm_head_backward(hc, hs, wc, wsc, g, T, H, V, targets, lse, grad,
                                           static_cast<const uint16_t*>(h_bf16),
-                                          static_cast<const uint16_t*>(w_bf16), dh, dW, accumulate_dw,
+                                          static_cast<const uint16_t*>(w_bf16), dh, dW,
+                                          (flags & FP8RL_BWD_ACCUMULATE_DW) != 0,
+                                          (flags & FP8RL_BWD_POW2_SCALES) != 0,
                                           ws, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? FP8RL_OK : cuda_fail(e);
 }

@@ -14,10 +14,11 @@
 //      [H][V'] and h^T [H][T'] with 128 x 128 scales (V', T' = V, T rounded
 //      up to 128; the padding holds zero codes);
 //   3. the block-scaled FP8 GEMM forms dh and dW into float32.
-// With power-of-two forward scales (the UE8M0 variant) the backward keeps that
-// format: P, P^T, W^T and h^T take power-of-two scales (floored at 2^-127),
-// and the recompute and both contractions run on the block-scaled MMA
-// (tcgen05.mma kind::mxf8f6f4), which applies them per 32-wide K step.
+// With pow2_scales (implied by power-of-two forward scales, the UE8M0
+// variant) P, P^T, W^T and h^T take power-of-two scales (floored at 2^-127)
+// and both contractions run on the block-scaled MMA (tcgen05.mma
+// kind::mxf8f6f4), which applies them per 32-wide K step; the recompute runs
+// in the forward's own mode.
 #include <cuda_fp8.h>
 
 #include <algorithm>
@@ -130,7 +131,7 @@ cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const ui
                                     const float* wsc, int gran, int64_t T, int64_t H, int64_t V,
                                     const int32_t* targets, const float* lse, const float* grad,
                                     const uint16_t* h, const uint16_t* W, float* dh, float* dW,
-                                    int accumulate_dw, void* ws, cudaStream_t s) {
+                                    bool accumulate_dw, bool pow2_scales, void* ws, cudaStream_t s) {
   const BwdLayout l = bwd_layout(T, H, V);
   char* base = static_cast<char*>(ws);
   uint8_t* Pq = reinterpret_cast<uint8_t*>(base + l.p);
@@ -141,7 +142,7 @@ cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const ui
   float* Wts = reinterpret_cast<float*>(base + l.wts);
   uint8_t* Htq = reinterpret_cast<uint8_t*>(base + l.ht);
   float* Hts = reinterpret_cast<float*>(base + l.hts);
-  const bool ue = gran == FP8RL_GRAN_BLOCK_UE8M0;
+  const bool ue = pow2_scales || gran == FP8RL_GRAN_BLOCK_UE8M0;
   const int bgran = ue ? FP8RL_GRAN_BLOCK_UE8M0 : FP8RL_GRAN_BLOCK;
   uint8_t* sf = reinterpret_cast<uint8_t*>(base + l.sf);
   // 1. recompute z (FP8), quantise P = dLoss/dz in both orientations
@@ -164,6 +165,7 @@ cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const ui
   a.ld_pq = l.vp;
   a.ld_ptq = l.tp;
   a.sf_images = sf;
+  a.p_pow2 = ue ? 1 : 0;
   cudaError_t e = launch_gemm_dense_dlogits(a, s);
   if (e != cudaSuccess) return e;
   if (dh) {  // 2./3. dh[T][H] = P[T][V'] . (W^T[H][V'])^T
@@ -203,7 +205,7 @@ cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const ui
     d.ldb = l.tp;
     d.c_out = dW;
     d.ld_c = H;
-    d.accumulate = accumulate_dw;
+    d.accumulate = accumulate_dw ? 1 : 0;
     e = launch_gemm_store(d, s);
   }
   return e;

@@ -206,9 +206,9 @@ __device__ __forceinline__ float fmax_nan(float a, float b) {
 //   codes of P with the 128 x 128 block scale of the tile half (the max over
 //   the four warps holding its 128 rows, exchanged through shared memory
 //   with a bounded wait), stored transposed         -> ptq_out / ptq_scales
-// With pow2 (the UE8M0 variant) both scales are rounded up to powers of two
-// and floored at 2^-127, the scale format of the block-scaled MMA that runs
-// the contractions.  Rows past M and columns past N hold 0 (the K padding of
+// With p.p_pow2 both scales are rounded up to powers of two and floored at
+// 2^-127, the scale format of the block-scaled MMA that then runs the
+// contractions.  Rows past M and columns past N hold 0 (the K padding of
 // the contractions).  Returns false if the exchange wait expired.
 __device__ __forceinline__ float p_scale(float amax, bool pow2) {
   const float s = scale_of(amax);
@@ -218,7 +218,8 @@ __device__ __forceinline__ float p_scale(float amax, bool pow2) {
 __device__ __forceinline__ bool dense_fp8_epilogue(const Params& p, const EpiState& es, float* z, int row,
                                                    int col0, int m_blk, int rit, int half, int quarter,
                                                    int lane, int tcount, uint64_t* blk_bar, uint32_t* blk_max,
-                                                   uint64_t lim, const volatile int* abort_flag, bool pow2) {
+                                                   uint64_t lim, const volatile int* abort_flag) {
+  const bool pow2 = p.p_pow2 != 0;
   const int ncol = min(CHUNK, p.N - col0);
   const bool row_ok = row < p.M;
   const float g = es.g;
@@ -628,7 +629,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         float* z = reinterpret_cast<float*>(z2);
         if (EPI == kEpiDenseFp8) {
           ok = dense_fp8_epilogue(p, es, z, row, col0, m_blk, rit, half, quarter, lane, tcount, blk_bar, blk_max,
-                                  lim, abort_flag, MODE == kUe8m0);
+                                  lim, abort_flag);
           if (!ok) break;
         } else {
           epi_consume128<EPI>(p, es, z, row, col0);
@@ -650,7 +651,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         aphase ^= 1;
         if (EPI == kEpiDenseFp8) {
           ok = dense_fp8_epilogue(p, es, zf, row, col0, m_blk, rit, half, quarter, lane, tcount, blk_bar, blk_max,
-                                  lim, abort_flag, MODE == kUe8m0);
+                                  lim, abort_flag);
           if (!ok) break;
         } else {
           epi_consume128<EPI>(p, es, zf, row, col0);
@@ -685,7 +686,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         ab ^= 1;
         if (ab == 0) aphase ^= 1;
         ok = dense_fp8_epilogue(p, es, zf, row, col0, m_blk, rit, half, quarter, lane, tcount, blk_bar, blk_max,
-                                lim, abort_flag, MODE == kUe8m0);
+                                lim, abort_flag);
         if (!ok) break;
       } else {
         ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&acc_full[ab]), aphase, lim, abort_flag));
@@ -919,6 +920,7 @@ cudaError_t launch_gemm(const GemmArgs& a, cudaStream_t s) {
   p.c_out = a.c_out;
   p.ld_c = a.ld_c;
   p.accumulate = a.accumulate;
+  p.p_pow2 = a.p_pow2;
   p.M = static_cast<int>(a.M);
   p.N = static_cast<int>(a.N);
   p.K = static_cast<int>(a.K);

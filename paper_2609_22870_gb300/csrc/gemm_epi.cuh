@@ -44,6 +44,7 @@ struct Params {
   float* c_out;      // kEpiStore: fp32 [M][ld_c]
   int64_t ld_c;
   int accumulate;
+  int p_pow2;        // kEpiDenseFp8: power-of-two scales for P and P^T
   int M, N, K;
   int num_m, num_n, num_kb;
   int band_m;  // row blocks per band of the tile order

@@ -48,6 +48,7 @@ struct GemmArgs {
   float* c_out;             // [M][ld_c], 16-byte aligned, ld_c % 4 == 0
   int64_t ld_c;
   int accumulate;           // add to c_out instead of overwriting it
+  int p_pow2;               // dense FP8 dlogits: power-of-two scales for P and P^T
   // FP8RL_GRAN_BLOCK_UE8M0: device scratch of gemm_ue8m0_image_bytes(M, N, K)
   // bytes (16-byte aligned) for the E8M0 scale-factor images
   uint8_t* sf_images;
@@ -75,7 +76,7 @@ cudaError_t launch_lm_head_backward(const uint8_t* hc, const float* hs, const ui
                                     const float* wsc, int gran, int64_t T, int64_t H, int64_t V,
                                     const int32_t* targets, const float* lse, const float* grad,
                                     const uint16_t* h, const uint16_t* W, float* dh, float* dW,
-                                    int accumulate_dw, void* ws, cudaStream_t s);
+                                    bool accumulate_dw, bool pow2_scales, void* ws, cudaStream_t s);
 // codes [cols][ld_out] of the transposed bf16 matrix in [rows][ld_in] with
 // 128 x 128 E4M3 blocks, scales [ceil(cols/128)][ld_out/128]; columns
 // rows .. ld_out-1 of the codes are zero (ld_out a multiple of 128, >= rows);

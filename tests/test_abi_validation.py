@@ -29,10 +29,10 @@ ODD = ctypes.c_void_p(4096 + 8)
 NULL = None
 
 
-def _bwd(api, T=64, H=128, V=256, gran=2, h=P, dh=P, dW=P, ws=P, ws_bytes=None, hc=P, lse=P):
+def _bwd(api, T=64, H=128, V=256, gran=2, h=P, dh=P, dW=P, ws=P, ws_bytes=None, hc=P, lse=P, flags=0):
     if ws_bytes is None:
         ws_bytes = api.lib.fp8rl_lm_head_backward_workspace_size(T, H, V)
-    return api.lib.fp8rl_lm_head_backward(hc, P, P, P, gran, T, H, V, P, lse, P, h, P, dh, dW, 0, ws,
+    return api.lib.fp8rl_lm_head_backward(hc, P, P, P, gran, T, H, V, P, lse, P, h, P, dh, dW, flags, ws,
                                           ws_bytes, NULL)
 
 
@@ -60,6 +60,8 @@ def test_lm_head_backward_workspace_size(api):
 
 def test_lm_head_backward_rejects_bad_arguments(api):
     assert _bwd(api, hc=NULL) == api.EINVAL
+    assert _bwd(api, flags=4) == api.EINVAL  # unknown flag bit
+    assert _bwd(api, flags=api.BWD_ACCUMULATE_DW | api.BWD_POW2_SCALES, hc=NULL) == api.EINVAL
     assert _bwd(api, lse=NULL) == api.EINVAL
     assert _bwd(api, dh=NULL, dW=NULL) == api.EINVAL
     assert _bwd(api, gran=7) == api.EINVAL

@@ -83,12 +83,13 @@ def _pow2_flip_slack(x, block_rows):
     return out
 
 
-def _oracle(h, W, y, g, gran):
-    pow2 = gran == UE
-    og = OQ.BLOCK if pow2 else gran
+def _oracle(h, W, y, g, gran, bwd_pow2=False):
+    fwd_pow2 = gran == UE
+    pow2 = fwd_pow2 or bwd_pow2
+    og = OQ.BLOCK if fwd_pow2 else gran
     h32, W32 = h.float().cpu().numpy(), W.float().cpu().numpy()
-    hq, hs = OQ.quantize(h32, og, OQ.ACT, pow2=pow2)
-    wq, ws = OQ.quantize(W32, og, OQ.WEIGHT, pow2=pow2)
+    hq, hs = OQ.quantize(h32, og, OQ.ACT, pow2=fwd_pow2)
+    wq, ws = OQ.quantize(W32, og, OQ.WEIGHT, pow2=fwd_pow2)
     ref = OL.lm_head_backward_fp8(hq, hs, wq, ws, og, y.cpu().numpy(), g.cpu().numpy(), h32, W32, pow2=pow2)
     T, V = ref["P"].shape
     P = ref["P"].astype(np.float64)
@@ -107,12 +108,15 @@ def _oracle(h, W, y, g, gran):
 UE = 3  # power-of-two block scales on the block-scaled MMA (forward and backward)
 
 
-@pytest.mark.parametrize("gran", [OQ.TENSOR, OQ.ROWWISE, OQ.BLOCK, UE])
+@pytest.mark.parametrize("gran,bwd_pow2", [(OQ.TENSOR, False), (OQ.ROWWISE, False), (OQ.BLOCK, False),
+                                           (UE, False), (OQ.BLOCK, True), (OQ.ROWWISE, True)])
 @pytest.mark.parametrize("T,H,V", [(300, 256, 1000), (129, 384, 1001), (1, 128, 1), (520, 128, 4096)])
-def test_backward_small_all_elements(cuda_lib, gran, T, H, V):
+def test_backward_small_all_elements(cuda_lib, gran, bwd_pow2, T, H, V):
+    """bwd_pow2: the paper-scale forward with the backward's own operands on
+    power-of-two scales (FP8RL_BWD_POW2_SCALES); UE implies it."""
     h, W, y, g = _data(T, H, V, T + V)
-    out, _ = _forward_backward(cuda_lib, h, W, y, g, gran)
-    ref, bh, bw = _oracle(h, W, y, g, gran)
+    out, _ = _forward_backward(cuda_lib, h, W, y, g, gran, pow2_scales=bwd_pow2)
+    ref, bh, bw = _oracle(h, W, y, g, gran, bwd_pow2)
     dh = out["dh"].cpu().numpy().astype(np.float64)
     dW = out["dW"].cpu().numpy().astype(np.float64)
     assert np.all(np.abs(dh - ref["dh"]) <= bh + 1e-30)
@@ -150,21 +154,22 @@ def test_backward_accumulate_chunks_and_single_outputs(cuda_lib):
         api.lm_head_backward(hc, hs, wc, ws, gran, y, lse, g, h, W, want_dh=False, want_dw=False)
 
 
-@pytest.mark.parametrize("gran", [OQ.BLOCK, OQ.TENSOR, UE])
-def test_backward_full_size_grpo8b(cuda_lib, gran):
+@pytest.mark.parametrize("gran,bwd_pow2", [(OQ.BLOCK, False), (OQ.TENSOR, False), (UE, False), (OQ.BLOCK, True)])
+def test_backward_full_size_grpo8b(cuda_lib, gran, bwd_pow2):
     """grpo_8b (T 16384, H 4096, V 151936): 64 sampled rows of dh against the
     oracle's FP8 backward; dW by bounded column sums.  UE: power-of-two scales
-    on every operand, the contractions on the block-scaled MMA."""
+    on every operand, the contractions on the block-scaled MMA; bwd_pow2: the
+    same for the backward's operands after a paper-scale forward."""
     api = cuda_lib
     w = synth.WORKLOADS["grpo_8b"]
     h, W, y = synth.hidden_states(w, "cuda"), synth.lm_head_weight(w, "cuda"), synth.targets(w, "cuda")
     g = (torch.randn(w.T, generator=torch.Generator().manual_seed(8)) / w.T).float().cuda()
-    out, _ = _forward_backward(api, h, W, y, g, gran)
+    out, _ = _forward_backward(api, h, W, y, g, gran, pow2_scales=bwd_pow2)
     dh = out["dh"]
     assert bool(torch.isfinite(dh).all()) and bool(torch.isfinite(out["dW"]).all())
     rows = sample_rows(w.T, 60, 9)
-    pow2 = gran == UE
-    _, lse_r, z_r = oracle_logprobs_rows(h, W, OQ.BLOCK if pow2 else gran, y, rows, pow2=pow2)
+    pow2 = gran == UE or bwd_pow2
+    _, lse_r, z_r = oracle_logprobs_rows(h, W, OQ.BLOCK if gran == UE else gran, y, rows, pow2=gran == UE)
     P = OL.dlogits(z_r, y.cpu().numpy()[rows], lse_r, g.cpu().numpy()[rows]).astype(np.float32)
     Pp = OL._pad_cols(P)
     kw = {"pow2": True, "scale_floor": OQ.E8M0_MIN} if pow2 else {}
