@@ -241,10 +241,11 @@ def kernels_per_step(gran, mode, T):
     """Kernel launches of one FP8 step: quantise h and W (amax + encode each
     for per-tensor scaling), the GEMM, the combine, calibration (one
     cooperative launch up to 2^18 tokens, else a pass and a decide launch per
-    stage: 9 stages exact, 3 grid), valid-token count and surrogate."""
+    stage: 9 stages exact, 3 grid) and the surrogate (which takes the
+    calibration's count of valid tokens, so it makes no counting pass)."""
     q = 2 if gran == 0 else 1
     calib = 1 if T <= (1 << 18) else (6 if mode == 1 else 18)
-    return 2 * q + 1 + 1 + calib + 2
+    return 2 * q + 1 + 1 + calib + 1
 
 
 def run_ours(args, rank, world, local_rank):
@@ -298,7 +299,8 @@ def run_ours(args, rank, world, local_rank):
                 ev[5].record(stream)
             api.clipped_surrogate(bb.ratio, adv_d, mask_d, None, bounds=api.bounds_view(bb.cal_res),
                                   stats=bb.stats, workspace=bb.sur_ws,
-                                  out={"grad": bb.grad, "clip_mask": bb.clip_mask})
+                                  out={"grad": bb.grad, "clip_mask": bb.clip_mask},
+                                  n_valid=api.n_valid_view(bb.cal_res))
             if record:
                 ev[6].record(stream)
         return step

@@ -269,6 +269,8 @@ typedef struct fp8rl_calib_result {
   int64_t sum_pos_fp8;    /* P     = sum_{A>0, r_fp8 < H*} q                          */
   double rho_bf16;        /* N_bf / D_bf                                              */
   double rho_fp8;         /* P / D_fp8                                                */
+  int64_t n_valid;        /* valid tokens (mask != 0; T without a mask), for the
+                             surrogate's token mean (fp8rl_clipped_surrogate)         */
 } fp8rl_calib_result;
 
 #define FP8RL_CALIB_FLAG_NO_NEG 1       /* no A<0 token: L* = c_lo (clamped to I_L) */
@@ -342,6 +344,10 @@ size_t fp8rl_surrogate_workspace_size(int64_t T);
  *   r, adv       float [T];  mask uint8 [T] or NULL;  w_tis float [T] or NULL (1)
  *   lo, hi       bounds by value, used when `bounds` is NULL
  *   bounds       DEVICE float[2] {L, H} or NULL (e.g. a fp8rl_calib_result*)
+ *   n_valid      DEVICE int64, the number of valid tokens of `mask` when the
+ *                caller has it (e.g. &result->n_valid of fp8rl_calibrate_clip_bounds
+ *                on the same mask), read at run time; NULL: the call counts
+ *                them in a pass of its own.  Ignored without a mask (T).
  *   grad_logp    float [T] out or NULL: dloss/dlogp_t = -w A r / n_valid on
  *                unclipped valid tokens, 0 elsewhere.  With lse from
  *                fp8rl_token_logprobs this is dLoss/dlogits in factored form:
@@ -350,7 +356,8 @@ size_t fp8rl_surrogate_workspace_size(int64_t T);
  *   stats        DEVICE pointer to one fp8rl_clip_stats */
 fp8rl_status fp8rl_clipped_surrogate(const float* r, const float* adv, const uint8_t* mask,
                                      const float* w_tis, int64_t T, float lo, float hi,
-                                     const float* bounds, float* grad_logp, uint8_t* clip_mask,
+                                     const float* bounds, const int64_t* n_valid,
+                                     float* grad_logp, uint8_t* clip_mask,
                                      fp8rl_clip_stats* stats,
                                      void* workspace, size_t workspace_bytes, void* stream);
 

@@ -279,6 +279,7 @@ def calibrate_clip_bounds(r_fp8, r_bf16, adv, mask, coef, eps_low, eps_high, opt
         "hi_new": smooth_update(o["hi_old"], hi_star, o["delta_hi"]),
         "c_lo": c_lo, "c_hi": c_hi,
         "n_neg": n_neg, "n_pos": n_pos, "k_bf16": k,
+        "n_valid": int(mask.sum()),  # every valid token, any advantage (the surrogate's mean)
         "k_fp8": int(np.sum(neg & (r_fp8 <= lo_star))),
         "shift": s,
         "sum_pos_bf16": n_bf, "sum_neg_bf16": d_bf,

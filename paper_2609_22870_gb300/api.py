@@ -46,7 +46,8 @@ class CalibResult(ctypes.Structure):
                 ("k_bf16", ctypes.c_int64), ("k_fp8", ctypes.c_int64),
                 ("sum_pos_bf16", ctypes.c_int64), ("sum_neg_bf16", ctypes.c_int64),
                 ("sum_neg_fp8", ctypes.c_int64), ("sum_pos_fp8", ctypes.c_int64),
-                ("rho_bf16", ctypes.c_double), ("rho_fp8", ctypes.c_double)]
+                ("rho_bf16", ctypes.c_double), ("rho_fp8", ctypes.c_double),
+                ("n_valid", ctypes.c_int64)]
 
 
 class ClipStats(ctypes.Structure):
@@ -95,7 +96,7 @@ _SIGS = {
     "fp8rl_calibrate_clip_bounds": (_i, [_p, _p, _p, _p, _p, _i64, _f, _f, ctypes.POINTER(CalibOpts),
                                          _p, _p, _sz, _p]),
     "fp8rl_surrogate_workspace_size": (_sz, [_i64]),
-    "fp8rl_clipped_surrogate": (_i, [_p, _p, _p, _p, _i64, _f, _f, _p, _p, _p, _p, _p, _sz, _p]),
+    "fp8rl_clipped_surrogate": (_i, [_p, _p, _p, _p, _i64, _f, _f, _p, _p, _p, _p, _p, _p, _sz, _p]),
     "fp8rl_dlogits_workspace_size": (_sz, [_i64, _i64, _i64, _i]),
     "fp8rl_dlogits_rows": (_i, [_p, _p, _p, _p, _i, _i64, _i64, _i64, _p, _p, _p, _p, _i64, _p, _p,
                                 _sz, _p]),
@@ -377,14 +378,23 @@ def bounds_view(buf):
     return buf[:8].view(torch.float32)
 
 
+def n_valid_view(buf):
+    """The valid-token count inside a device fp8rl_calib_result buffer (int64
+    [1]), for clipped_surrogate(n_valid=...)."""
+    off = CalibResult.n_valid.offset
+    return buf[off:off + 8].view(torch.int64)
+
+
 # ------------------------------------------------------------------ surrogate
 def surrogate_workspace_size(T):
     return int(lib.fp8rl_surrogate_workspace_size(T))
 
 
 def clipped_surrogate(r, adv, mask=None, w_tis=None, lo=0.8, hi=1.2, bounds=None, want_grad=True,
-                      want_clip_mask=True, stats=None, workspace=None, out=None, stream=None):
-    """fp8rl_clipped_surrogate -> dict(stats=<device buffer>, grad, clip_mask)."""
+                      want_clip_mask=True, stats=None, workspace=None, out=None, stream=None, n_valid=None):
+    """fp8rl_clipped_surrogate -> dict(stats=<device buffer>, grad, clip_mask).
+    ``n_valid``: device int64 [1] count of the mask's valid tokens when known
+    (n_valid_view of the calibration's result on the same mask), else counted."""
     T = r.numel()
     dev = r.device
     _dev(r, torch.float32, "r")
@@ -392,6 +402,7 @@ def clipped_surrogate(r, adv, mask=None, w_tis=None, lo=0.8, hi=1.2, bounds=None
     _dev(mask, torch.uint8, "mask", T)
     _dev(w_tis, torch.float32, "w_tis", T)
     _dev(bounds, torch.float32, "bounds", 2)
+    _dev(n_valid, torch.int64, "n_valid", 1)
     o = out or {}
     grad = o.get("grad", torch.empty(T, dtype=torch.float32, device=dev)) if want_grad else None
     cm = o.get("clip_mask", torch.empty(T, dtype=torch.uint8, device=dev)) if want_clip_mask else None
@@ -399,8 +410,9 @@ def clipped_surrogate(r, adv, mask=None, w_tis=None, lo=0.8, hi=1.2, bounds=None
     if workspace is None:
         workspace = _workspace(surrogate_workspace_size(T), dev)
     _ok(lib.fp8rl_clipped_surrogate(_ptr(r), _ptr(adv), _ptr(mask), _ptr(w_tis), T, lo, hi,
-                                    _ptr(bounds), _ptr(grad), _ptr(cm), _ptr(stats), _ptr(workspace),
-                                    workspace.numel(), _stream(stream)), "fp8rl_clipped_surrogate")
+                                    _ptr(bounds), _ptr(n_valid), _ptr(grad), _ptr(cm), _ptr(stats),
+                                    _ptr(workspace), workspace.numel(), _stream(stream)),
+        "fp8rl_clipped_surrogate")
     return {"stats": stats, "grad": grad, "clip_mask": cm}
 
 
@@ -622,8 +634,9 @@ def score_calibrate_loss(h, W, targets, logp_old, r_bf16, adv, mask, coef, gran,
                          opts=None, buffers=None, stream=None):
     """One pass of the whole hot path through the C ABI, in order:
     quantize(h), quantize(W), token_logprobs (+ ratios), calibrate_clip_bounds,
-    clipped_surrogate with the new bounds.  Returns the buffers object whose
-    fields hold every output (device-resident)."""
+    clipped_surrogate with the new bounds (and the calibration's count of valid
+    tokens, so the surrogate makes no counting pass).  Returns the buffers
+    object whose fields hold every output (device-resident)."""
     T, H = h.shape
     V = W.shape[0]
     b = buffers or StepBuffers(T, H, V, gran, h.device)
@@ -634,5 +647,6 @@ def score_calibrate_loss(h, W, targets, logp_old, r_bf16, adv, mask, coef, gran,
     calibrate_clip_bounds(b.ratio, r_bf16, adv, mask, coef, eps_low, eps_high, opts, b.cal_res,
                           b.cal_ws, stream)
     clipped_surrogate(b.ratio, adv, mask, None, bounds=bounds_view(b.cal_res), stats=b.stats,
-                      workspace=b.sur_ws, out={"grad": b.grad, "clip_mask": b.clip_mask}, stream=stream)
+                      workspace=b.sur_ws, out={"grad": b.grad, "clip_mask": b.clip_mask}, stream=stream,
+                      n_valid=n_valid_view(b.cal_res))
     return b

@@ -313,14 +313,14 @@ size_t fp8rl_surrogate_workspace_size(int64_t T) { return T < 0 ? 0 : surrogate_
 
 fp8rl_status fp8rl_clipped_surrogate(const float* r, const float* adv, const uint8_t* mask,
                                      const float* w_tis, int64_t T, float lo, float hi,
-                                     const float* bounds, float* grad, uint8_t* clip_mask,
-                                     fp8rl_clip_stats* stats, void* ws, size_t ws_bytes,
-                                     void* stream) {
+                                     const float* bounds, const int64_t* n_valid, float* grad,
+                                     uint8_t* clip_mask, fp8rl_clip_stats* stats, void* ws,
+                                     size_t ws_bytes, void* stream) {
   if (!stats || (T > 0 && (!r || !adv))) return FP8RL_EINVAL;
   if (T < 0) return FP8RL_ESHAPE;
   if (!ws || ws_bytes < surrogate_workspace_bytes(T)) return FP8RL_EWORKSPACE;
-  cudaError_t e = launch_surrogate(r, adv, mask, w_tis, T, lo, hi, bounds, grad, clip_mask, stats, ws,
-                                   static_cast<cudaStream_t>(stream));
+  cudaError_t e = launch_surrogate(r, adv, mask, w_tis, T, lo, hi, bounds, n_valid, grad, clip_mask,
+                                   stats, ws, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? FP8RL_OK : cuda_fail(e);
 }
 

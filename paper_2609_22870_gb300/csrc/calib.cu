@@ -83,6 +83,7 @@ struct State {
   unsigned int h_mp_inv;        // ~min{key in I_H : q != 0}
   unsigned int h_Mp1;           // 1 + max{key in I_H : q != 0}
   unsigned int pad2;
+  unsigned long long n_valid;   // valid tokens (any advantage), for the surrogate's mean
   // written by decide steps
   int shift;
   int found;
@@ -287,6 +288,7 @@ struct PassAcc {
   long long h_below;
   unsigned l_nb_below1, l_nb_above_inv, l_mp_inv, l_Mp1;
   unsigned h_nb_below1, h_nb_above_inv, h_top1, h_mp_inv, h_Mp1;
+  unsigned long long n_valid;  // last: zero from the initialiser's omitted tail
 };
 
 // Constants of one pass.
@@ -310,6 +312,7 @@ __device__ __forceinline__ int pass_token(const Args& a, const PassCtx& x, const
     if (!(isfinite(A) && isfinite(rf) && isfinite(rb) && isfinite(c)) || rf < 0.f || rb < 0.f ||
         c < 0.f)
       acc.bad = 1;
+    acc.n_valid += valid;
     if (neg) {
       ++acc.n_neg;
       if (rb <= a.c_lo) ++acc.k_bf;
@@ -593,7 +596,8 @@ __device__ void pass_body(const Args& a, ShHist& sh, float* sh_cand) {
     else if (hist_mode == 3) hist_add_lane(sh, d, w);
   }
   if (to_list && lane == 0) (stage == kPrep ? a.l_cnt : a.h_cnt)[seg] = seg_fill;
-  unsigned long long n_neg = acc.n_neg, n_pos = acc.n_pos, k_bf = acc.k_bf, k_fp = acc.k_fp;
+  unsigned long long n_neg = acc.n_neg, n_pos = acc.n_pos, k_bf = acc.k_bf, k_fp = acc.k_fp,
+                     n_valid = acc.n_valid;
   long long s_pos_bf = acc.s_pos_bf, s_neg_bf = acc.s_neg_bf, s_neg_fp = acc.s_neg_fp,
             s_pos_fp = acc.s_pos_fp;
   unsigned emax = acc.emax, bad = acc.bad;
@@ -604,6 +608,7 @@ __device__ void pass_body(const Args& a, ShHist& sh, float* sh_cand) {
   // ---- flush: warp-aggregated scalars, then the block histogram
   n_neg = warp_sum(n_neg);
   n_pos = warp_sum(n_pos);
+  n_valid = warp_sum(n_valid);
   k_bf = warp_sum(k_bf);
   k_fp = warp_sum(k_fp);
   s_pos_bf = warp_sum(s_pos_bf);
@@ -634,6 +639,7 @@ __device__ void pass_body(const Args& a, ShHist& sh, float* sh_cand) {
     if (h_below) atomicAdd(&st->h_below, static_cast<unsigned long long>(h_below));
     if (n_neg) atomicAdd(&st->n_neg, n_neg);
     if (n_pos) atomicAdd(&st->n_pos, n_pos);
+    if (n_valid) atomicAdd(&st->n_valid, n_valid);
     if (k_bf) atomicAdd(&st->k_bf16, k_bf);
     if (k_fp) atomicAdd(&st->k_fp8, k_fp);
     if (s_pos_bf) atomicAdd(&st->s_pos_bf, static_cast<unsigned long long>(s_pos_bf));
@@ -938,6 +944,7 @@ __device__ void write_result(const Args& a, State* st) {
   r.sum_pos_fp8 = static_cast<int64_t>(st->s_pos_fp);
   r.rho_bf16 = r.sum_neg_bf16 ? static_cast<double>(r.sum_pos_bf16) / static_cast<double>(r.sum_neg_bf16) : NAN;
   r.rho_fp8 = r.sum_neg_fp8 ? static_cast<double>(r.sum_pos_fp8) / static_cast<double>(r.sum_neg_fp8) : NAN;
+  r.n_valid = static_cast<int64_t>(st->n_valid);
   *a.out = r;
 }
 

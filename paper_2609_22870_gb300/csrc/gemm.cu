@@ -166,8 +166,23 @@ __host__ __device__ constexpr uint32_t idesc_mx_e4m3(uint32_t M, uint32_t N) {
 }
 
 // E4M3 codes Q_FP8(fl32(v_i / S)) of 128 floats, four per word (byte i % 4 of
-// word i / 4), in the packed arithmetic of the quantiser.
-__device__ __forceinline__ void encode128(const float* v, float s, uint32_t (&w)[32]) {
+// word i / 4), in the packed arithmetic of the quantiser.  With pow2 (S a
+// power of two in [2^-127, 2^120]) 1 / S is exact and so is v * (1 / S)
+// wherever it is at least 2^-126; below that both forms give code 0 of v's
+// sign, so one packed multiply replaces the corrected quotient.
+__device__ __forceinline__ void encode128(const float* v, float s, uint32_t (&w)[32], bool pow2) {
+  if (pow2) {
+    const float r = __frcp_rn(s);
+    const uint64_t r2 = f32x2(r, r);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      uint64_t q0, q1;
+      asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(q0) : "l"(f32x2(v[4 * i], v[4 * i + 1])), "l"(r2));
+      asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(q1) : "l"(f32x2(v[4 * i + 2], v[4 * i + 3])), "l"(r2));
+      w[i] = cvt_e4m3x2(q0) | (cvt_e4m3x2(q1) << 16);
+    }
+    return;
+  }
   const E4M3Enc e = e4m3_encoder(s);
   if (!e.divide) {
 #pragma unroll
@@ -246,7 +261,7 @@ __device__ __forceinline__ bool dense_fp8_epilogue(const Params& p, const EpiSta
   uint32_t w[32];
   if (row_ok && col0 < p.ld_pq) {  // the row's block along N (K of the dh contraction)
     const float s = p_scale(amax, pow2);
-    encode128(z, s, w);
+    encode128(z, s, w, pow2);
     uint4* dst = reinterpret_cast<uint4*>(p.pq_out + static_cast<size_t>(row) * p.ld_pq + col0);
 #pragma unroll
     for (int q = 0; q < 8; ++q) dst[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
@@ -267,7 +282,7 @@ __device__ __forceinline__ bool dense_fp8_epilogue(const Params& p, const EpiSta
   const uint32_t bmax = max(max(bm[0], bm[1]), max(bm[2], bm[3]));
   if (ncol <= 0) return true;
   const float sb = p_scale(__uint_as_float(bmax), pow2);
-  encode128(z, sb, w);
+  encode128(z, sb, w, pow2);
   // lanes are consecutive tokens; a 4 x 4 byte transpose within each group of
   // four lanes (two exchanges) leaves lane 4a + j with column 4k + j of rows
   // 4a .. 4a + 3, so each store writes four bytes and each column of P^T gets

@@ -109,10 +109,11 @@ uint32_t calib_status_take();
 
 // ----------------------------------------------------------------- loss.cu
 size_t surrogate_workspace_bytes(int64_t T);
+// n_valid: device count of the mask's valid tokens, or NULL to count them
 cudaError_t launch_surrogate(const float* r, const float* adv, const uint8_t* mask,
                              const float* w, int64_t T, float lo, float hi, const float* bounds,
-                             float* grad, uint8_t* clip_mask, fp8rl_clip_stats* stats, void* ws,
-                             cudaStream_t s);
+                             const int64_t* n_valid, float* grad, uint8_t* clip_mask,
+                             fp8rl_clip_stats* stats, void* ws, cudaStream_t s);
 size_t seq_level_workspace_bytes(int64_t T, int64_t n_seq);
 cudaError_t launch_seq_level(const float* logp, const float* logp_old, const float* adv_seq,
                              const uint8_t* mask, const int32_t* sid, int64_t n_seq, int64_t T,

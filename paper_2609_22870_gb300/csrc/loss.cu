@@ -8,7 +8,8 @@
 //   g_t = dloss/dlogp_t = -w_t A_t r_t / n_valid on unclipped valid tokens
 //
 // Two grid-stride passes: the valid-token count (g needs it; skipped without
-// a mask), then the fused per-token pass writing g and the clip mask, four
+// a mask, or when the caller passes the count, e.g. the calibration's, which
+// reads the same mask), then the fused per-token pass writing g and the clip mask, four
 // tokens per thread and step with 16-byte loads when the arrays allow.  Terms
 // are float32 (two roundings of the exact product); each thread sums its
 // terms with an error-free two-sum compensation (Knuth), so its partial is
@@ -153,14 +154,16 @@ __global__ void __launch_bounds__(kThreads) surrogate_kernel(
     const float* __restrict__ r, const float* __restrict__ adv, const uint8_t* __restrict__ mask,
     const float* __restrict__ wts, int64_t T, float lo_arg, float hi_arg,
     const float* __restrict__ bounds, float* __restrict__ grad, uint8_t* __restrict__ clip_mask,
-    fp8rl_clip_stats* __restrict__ stats, Work* w, bool vec) {
+    fp8rl_clip_stats* __restrict__ stats, Work* w, const int64_t* __restrict__ nv_in, bool vec) {
   __shared__ double sh_d[kThreads / 32];
   __shared__ unsigned long long sh_u[kThreads / 32];
   __shared__ bool last;
   Bounds b;
   b.lo = bounds ? bounds[0] : lo_arg;
   b.hi = bounds ? bounds[1] : hi_arg;
-  const unsigned long long n_valid = mask ? w->n_valid : static_cast<unsigned long long>(T);
+  const unsigned long long n_valid =
+      !mask ? static_cast<unsigned long long>(T)
+            : (nv_in ? static_cast<unsigned long long>(*nv_in) : w->n_valid);
   b.inv_n = n_valid ? 1.0f / static_cast<float>(n_valid) : 0.f;
   Acc a;
   const int64_t tid = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
@@ -675,17 +678,17 @@ size_t surrogate_workspace_bytes(int64_t T) {
 
 cudaError_t launch_surrogate(const float* r, const float* adv, const uint8_t* mask,
                              const float* w, int64_t T, float lo, float hi, const float* bounds,
-                             float* grad, uint8_t* clip_mask, fp8rl_clip_stats* stats, void* ws,
-                             cudaStream_t s) {
+                             const int64_t* n_valid, float* grad, uint8_t* clip_mask,
+                             fp8rl_clip_stats* stats, void* ws, cudaStream_t s) {
   Work* work = static_cast<Work*>(ws);
   cudaError_t e = cudaMemsetAsync(work, 0, sizeof(Work), s);
   if (e != cudaSuccess) return e;
   const int grid = grid_of(T);
-  if (mask) count_valid_kernel<<<grid, kThreads, 0, s>>>(mask, T, work);
+  if (mask && !n_valid) count_valid_kernel<<<grid, kThreads, 0, s>>>(mask, T, work);
   const bool vec = aligned(r, 16) && aligned(adv, 16) && aligned(w, 16) && aligned(grad, 16) &&
                    aligned(mask, 4) && aligned(clip_mask, 4);
   surrogate_kernel<<<grid, kThreads, 0, s>>>(r, adv, mask, w, T, lo, hi, bounds, grad, clip_mask,
-                                              stats, work, vec);
+                                              stats, work, n_valid, vec);
   return cudaGetLastError();
 }
 

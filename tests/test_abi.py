@@ -126,3 +126,37 @@ int main(void) {
     assert r.returncode == 0, r.stderr
     run = subprocess.run([str(exe)], capture_output=True, text=True, timeout=60)
     assert run.returncode == 0 and run.stdout.strip() == "ok", run.stdout + run.stderr
+
+
+def _prototypes():
+    """name -> list of parameter declarations, from the header's prototypes."""
+    text = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    out = {}
+    for m in re.finditer(r"\b(?:fp8rl_status|size_t|void|uint32_t|int64_t|int|const char\s*\*)\s*(fp8rl_[a-z0-9_]+)\s*\(([^;{]*?)\)\s*;",
+                         text, flags=re.S):
+        params = [p.strip() for p in m.group(2).split(",")]
+        out[m.group(1)] = [] if params == ["void"] else params
+    return out
+
+
+def _ctype_of(param):
+    if "*" in param:
+        return "ptr"
+    base = param.rsplit(None, 1)[0]
+    return {"int64_t": "i64", "uint64_t": "u64", "float": "f32", "size_t": "u64", "int": "i32",
+            "fp8rl_gran": "i32", "fp8rl_role": "i32", "int32_t": "i32", "fp8rl_status": "i32",
+            "fp8rl_calib_mode": "i32"}[base]
+
+
+def test_binding_signatures_match_the_header(libpath):
+    """Every ctypes signature of the Python binding has the header's parameter
+    count and kinds (a missing or extra argument would shift every later one)."""
+    from paper_2609_22870_gb300 import api
+    kinds = {ctypes.c_void_p: "ptr", ctypes.c_int64: "i64", ctypes.c_uint64: "u64", ctypes.c_float: "f32",
+             ctypes.c_size_t: "u64", ctypes.c_int: "i32"}  # size_t is uint64 here
+    protos = _prototypes()
+    for name, (_, args) in api._SIGS.items():
+        assert name in protos, name
+        want = [_ctype_of(p) for p in protos[name]]
+        got = [kinds.get(a, "ptr") for a in args]  # POINTER(struct) types are pointers
+        assert got == want, (name, got, want)

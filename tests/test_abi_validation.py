@@ -99,6 +99,17 @@ def test_seq_mean_surrogate_rejects_bad_arguments(api):
     assert f(P, P, NULL, NULL, P, 10, 100, 0.8, 1.2, NULL, NULL, NULL, P, NULL, ws, NULL) == api.EWORKSPACE
 
 
+def test_token_mean_surrogate_rejects_bad_arguments(api):
+    # (r, adv, mask, w, T, lo, hi, bounds, n_valid, grad, clip_mask, stats, ws, ws_bytes, stream):
+    # the binding's signature table must match the header's, argument for argument
+    f = api.lib.fp8rl_clipped_surrogate
+    ws = api.lib.fp8rl_surrogate_workspace_size(100)
+    assert f(P, P, NULL, NULL, 100, 0.8, 1.2, NULL, P, NULL, NULL, NULL, P, ws, NULL) == api.EINVAL
+    assert f(NULL, P, NULL, NULL, 100, 0.8, 1.2, NULL, NULL, NULL, NULL, P, P, ws, NULL) == api.EINVAL
+    assert f(P, P, NULL, NULL, -1, 0.8, 1.2, NULL, NULL, NULL, NULL, P, P, ws, NULL) == api.ESHAPE
+    assert f(P, P, NULL, NULL, 100, 0.8, 1.2, NULL, P, NULL, NULL, P, NULL, ws, NULL) == api.EWORKSPACE
+
+
 def test_quantize_ue8m0_rejects_bad_arguments(api):
     f = api.lib.fp8rl_quantize_ue8m0
     assert f(NULL, 4, 128, 128, 2, 0, P, P, NULL, 0, NULL) == api.EINVAL      # no input

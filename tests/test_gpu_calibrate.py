@@ -41,8 +41,8 @@ def _ref(r_fp, r_bf, adv, mask, coef, eps_low, eps_high, **opts):
 def _compare(got, ref):
     for k in ("lo_star", "hi_star", "lo_new", "hi_new", "c_lo", "c_hi"):
         assert np.float32(got[k]) == ref[k] or (np.isnan(got[k]) and np.isnan(ref[k])), (k, got[k], ref[k])
-    for k in ("n_neg", "n_pos", "k_bf16", "k_fp8", "flags", "shift", "sum_pos_bf16", "sum_neg_bf16",
-              "sum_neg_fp8", "sum_pos_fp8"):
+    for k in ("n_neg", "n_pos", "n_valid", "k_bf16", "k_fp8", "flags", "shift", "sum_pos_bf16",
+              "sum_neg_bf16", "sum_neg_fp8", "sum_pos_fp8"):
         assert got[k] == ref[k], (k, got[k], ref[k])
     for k in ("rho_bf16", "rho_fp8"):
         if np.isnan(ref[k]):

@@ -68,6 +68,34 @@ def test_surrogate_nullable_and_empty(cuda_lib):
     assert st["loss"] == 0 and st["flags"] == 1
 
 
+def test_surrogate_with_the_calibrations_valid_count(cuda_lib):
+    """The step passes the calibration's count of valid tokens (same mask), so
+    the surrogate skips its counting pass: results identical to the counting
+    call.  A count of twice the valid tokens halves the gradient and the loss
+    exactly (the pointer is read); without a mask it is ignored."""
+    api = cuda_lib
+    T = 70000
+    r, adv, mask, w = (t.cuda() for t in _inputs(T, 21))
+    r_bf = (r * 1.01).contiguous()
+    cal = api.calibrate_clip_bounds(r, r_bf, adv, mask, None, 0.2, 0.2)
+    nv = api.n_valid_view(cal)
+    assert int(nv.item()) == int(mask.sum().item()) == api.read_calib_result(cal)["n_valid"]
+    b = api.bounds_view(cal)
+    ref = api.clipped_surrogate(r, adv, mask, w, bounds=b)
+    got = api.clipped_surrogate(r, adv, mask, w, bounds=b, n_valid=nv)
+    api.check()
+    assert torch.equal(ref["grad"], got["grad"]) and torch.equal(ref["clip_mask"], got["clip_mask"])
+    assert api.read_clip_stats(ref["stats"]) == api.read_clip_stats(got["stats"])
+    twice = (2 * nv).contiguous()
+    half = api.clipped_surrogate(r, adv, mask, w, bounds=b, n_valid=twice)
+    api.check()
+    assert torch.equal(half["grad"] * 2, ref["grad"])
+    assert api.read_clip_stats(half["stats"])["loss"] * 2 == api.read_clip_stats(ref["stats"])["loss"]
+    nomask = api.clipped_surrogate(r, adv, None, w, bounds=b, n_valid=twice)
+    api.check()
+    assert api.read_clip_stats(nomask["stats"])["n_valid"] == T
+
+
 def test_surrogate_deterministic(cuda_lib):
     r, adv, mask, w = (t.cuda() for t in _inputs(100000, 9))
     a = cuda_lib.read_clip_stats(cuda_lib.clipped_surrogate(r, adv, mask, w)["stats"])

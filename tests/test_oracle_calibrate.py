@@ -194,6 +194,13 @@ def test_degenerate_inputs():
     assert res["flags"] & C.FLAG_NO_POS and res["hi_star"] == F32(1.2)
     res = C.calibrate_clip_bounds(r, r, adv, np.zeros(8, np.uint8), None, 0.2, 0.2)
     assert res["flags"] & C.FLAG_NO_NEG and res["flags"] & C.FLAG_NO_POS
+    # n_valid counts valid tokens of any advantage sign (zero included): here
+    # tokens 0, 2, 3 and 5 are valid, with A = +1, -1, 0, 0
+    a = np.array([1, 5, -1, 0, 2, 0, 3, 4], np.float32)
+    m = np.array([1, 0, 1, 1, 0, 1, 0, 0], np.uint8)
+    res = C.calibrate_clip_bounds(r, r, a, m, None, 0.2, 0.2)
+    assert (res["n_valid"], res["n_pos"], res["n_neg"]) == (4, 1, 1)
+    assert C.calibrate_clip_bounds(r, r, a, None, None, 0.2, 0.2)["n_valid"] == 8
 
 
 @pytest.mark.parametrize("scale", [1e-30, 1e-5, 1.0, 1e5, 1e30])
