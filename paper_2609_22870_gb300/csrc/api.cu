@@ -5,6 +5,7 @@
 #include <cmath>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 
 #include "common.cuh"
 #include "internal.h"
@@ -75,6 +76,26 @@ int sm_count() {
     cached[dev] = n > 0 ? n : 1;
   }
   return cached[dev];
+}
+
+int resident_ctas(const void* kernel, int threads) {
+  struct Entry {
+    int dev;
+    const void* fn;
+    int threads, n;
+  };
+  static std::mutex mu;
+  static Entry table[64];
+  static int used = 0;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  std::lock_guard<std::mutex> lock(mu);
+  for (int i = 0; i < used; ++i)
+    if (table[i].dev == dev && table[i].fn == kernel && table[i].threads == threads) return table[i].n;
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kernel, threads, 0) != cudaSuccess || n < 1) n = 1;
+  if (used < 64) table[used++] = Entry{dev, kernel, threads, n};
+  return n;
 }
 
 }  // namespace fp8rl

@@ -138,6 +138,10 @@ cudaError_t launch_tis(const float* lp_old, const float* lp_samp, int64_t T, flo
 
 // SM count of the current device (cached per device).
 int sm_count();
+// CTAs of `threads` threads of `kernel` that one SM holds at once (cached per
+// device and kernel; at least 1): grids of kernels that give every CTA the
+// same share of the work are sized to one full wave with it.
+int resident_ctas(const void* kernel, int threads);
 
 // Records `e` as the text fp8rl_last_cuda_error() returns on this thread.
 void record_cuda_error(cudaError_t e);

@@ -63,6 +63,15 @@ int grid_of(int64_t T) {
   return static_cast<int>(want < 1 ? 1 : (want > cap ? cap : want));
 }
 
+// The launch grid of a kernel whose CTAs each take an equal share of the
+// work: `grid` (what the workspace was sized for) capped at one full wave of
+// the CTAs the SMs hold at once, so no CTA waits for a second wave.
+template <typename Kernel>
+int wave_grid(Kernel* kernel, int grid) {
+  const int cap = sm_count() * min(kCtasPerSm, resident_ctas(reinterpret_cast<const void*>(kernel), kThreads));
+  return grid < cap ? grid : cap;
+}
+
 // Number of non-zero bytes of a word.
 __device__ __forceinline__ uint32_t nonzero_bytes(uint32_t w) {
   return __popc((((w & 0x7F7F7F7Fu) + 0x7F7F7F7Fu) | w) & 0x80808080u);
@@ -683,8 +692,8 @@ cudaError_t launch_surrogate(const float* r, const float* adv, const uint8_t* ma
   Work* work = static_cast<Work*>(ws);
   cudaError_t e = cudaMemsetAsync(work, 0, sizeof(Work), s);
   if (e != cudaSuccess) return e;
-  const int grid = grid_of(T);
-  if (mask && !n_valid) count_valid_kernel<<<grid, kThreads, 0, s>>>(mask, T, work);
+  const int grid = wave_grid(surrogate_kernel, grid_of(T));
+  if (mask && !n_valid) count_valid_kernel<<<wave_grid(count_valid_kernel, grid_of(T)), kThreads, 0, s>>>(mask, T, work);
   const bool vec = aligned(r, 16) && aligned(adv, 16) && aligned(w, 16) && aligned(grad, 16) &&
                    aligned(mask, 4) && aligned(clip_mask, 4);
   surrogate_kernel<<<grid, kThreads, 0, s>>>(r, adv, mask, w, T, lo, hi, bounds, grad, clip_mask,
@@ -706,11 +715,13 @@ cudaError_t launch_seq_surrogate(const float* r, const float* adv, const uint8_t
   cudaError_t e = cudaMemsetAsync(work, 0, sizeof(SeqWork), s);
   if (e == cudaSuccess && n_seq > 0) e = cudaMemsetAsync(cnt, 0, static_cast<size_t>(n_seq) * 4, s);
   if (e != cudaSuccess) return e;
-  const int grid = grid_of(T);
+  const int grid = wave_grid(seq_surrogate_kernel, grid_of(T));
   if (aligned(sid, 16) && aligned(mask, 4))
-    seq_accum_kernel<true, false><<<grid, kThreads, 0, s>>>(nullptr, nullptr, mask, sid, T, n_seq, nullptr, cnt, work);
+    seq_accum_kernel<true, false><<<wave_grid(seq_accum_kernel<true, false, SeqWork>, grid_of(T)), kThreads, 0, s>>>(
+        nullptr, nullptr, mask, sid, T, n_seq, nullptr, cnt, work);
   else
-    seq_accum_kernel<false, false><<<grid, kThreads, 0, s>>>(nullptr, nullptr, mask, sid, T, n_seq, nullptr, cnt, work);
+    seq_accum_kernel<false, false><<<wave_grid(seq_accum_kernel<false, false, SeqWork>, grid_of(T)), kThreads, 0, s>>>(
+        nullptr, nullptr, mask, sid, T, n_seq, nullptr, cnt, work);
   const bool vec = aligned(r, 16) && aligned(adv, 16) && aligned(sid, 16) && aligned(w, 16) &&
                    aligned(grad, 16) && aligned(mask, 4) && aligned(clip_mask, 4);
   seq_surrogate_kernel<<<grid, kThreads, 0, s>>>(r, adv, mask, w, sid, T, n_seq, cnt, lo, hi, bounds,
@@ -736,14 +747,17 @@ cudaError_t launch_seq_level(const float* logp, const float* logp_old, const flo
   if (e != cudaSuccess) return e;
   const bool vec4 = aligned(logp, 16) && aligned(logp_old, 16) && aligned(sid, 16) && aligned(mask, 4);
   if (vec4)
-    seq_accum_kernel<true, true><<<grid_of(T), kThreads, 0, s>>>(logp, logp_old, mask, sid, T, n_seq, q, cnt, work);
+    seq_accum_kernel<true, true><<<wave_grid(seq_accum_kernel<true, true, SeqLvlWork>, grid_of(T)), kThreads, 0, s>>>(
+        logp, logp_old, mask, sid, T, n_seq, q, cnt, work);
   else
-    seq_accum_kernel<false, true><<<grid_of(T), kThreads, 0, s>>>(logp, logp_old, mask, sid, T, n_seq, q, cnt, work);
-  seq_lvl_seq_kernel<<<seq_grid_of(n_seq), kThreads, 0, s>>>(adv_seq, n_seq, q, cnt, lo, hi, bounds,
+    seq_accum_kernel<false, true><<<wave_grid(seq_accum_kernel<false, true, SeqLvlWork>, grid_of(T)), kThreads, 0, s>>>(
+        logp, logp_old, mask, sid, T, n_seq, q, cnt, work);
+  seq_lvl_seq_kernel<<<wave_grid(seq_lvl_seq_kernel, seq_grid_of(n_seq)), kThreads, 0, s>>>(adv_seq, n_seq, q, cnt, lo, hi, bounds,
                                                              seq_ratio, seq_clip, coef, part, stats, work);
   if (grad) {
     const bool vec = aligned(sid, 16) && aligned(grad, 16) && aligned(mask, 4);
-    seq_lvl_grad_kernel<<<grid_of(T), kThreads, 0, s>>>(mask, sid, T, n_seq, coef, grad, vec);
+    seq_lvl_grad_kernel<<<wave_grid(seq_lvl_grad_kernel, grid_of(T)), kThreads, 0, s>>>(mask, sid, T, n_seq, coef,
+                                                                                     grad, vec);
   }
   return cudaGetLastError();
 }
