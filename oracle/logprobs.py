@@ -53,11 +53,7 @@ multiples of 128 along K.
 With power-of-two (UE8M0) forward scales the backward keeps that scale format
 for its own four operands (the scales of the hardware's block-scaled MMA):
 each S is the smallest power of two not below fl32(amax / 448), raised to
-2^-127 where it falls below E8M0's range.  P^T is then requantised from the
-E4M3 P (its dequantised values P_hat), not from the float32 P: with
-power-of-two scales P_hat / S differs from P / S only by the first rounding,
-so the 128 x 128 codes are those of P except for ties below E4M3's normal
-range, and the transpose reads one byte per element instead of four.
+2^-127 where it falls below E8M0's range.
 """
 
 import numpy as np
@@ -166,9 +162,9 @@ def lm_head_backward_fp8(h_codes, h_scales, w_codes, w_scales, gran, targets, g,
     with 128 x 128 blocks (A operand of dW = P^T h); W^T [H][V] and h^T [H][T]
     are quantised from the bf16 values with 128 x 128 blocks (B operands).
     ``pow2``: the four take power-of-two scales floored at 2^-127 (the
-    backward of the UE8M0 variant), and P^T is requantised from P_hat.  The
-    products of the dequantised operands are summed in float64.  Returns the
-    quantised operands too (codes and scales in natural shape)."""
+    backward of the UE8M0 variant).  The products of the dequantised operands
+    are summed in float64.  Returns the quantised operands too (codes and
+    scales in natural shape)."""
     y = np.asarray(targets, np.int64)
     gg = np.asarray(g, np.float64)
     z = logits(h_codes, h_scales, w_codes, w_scales, gran)
@@ -177,9 +173,7 @@ def lm_head_backward_fp8(h_codes, h_scales, w_codes, w_scales, gran, targets, g,
     T, V = P32.shape
     kw = {"pow2": True, "scale_floor": Q.E8M0_MIN} if pow2 else {}
     pq, ps = Q.quantize(_pad_cols(P32), Q.BLOCK, Q.ACT, **kw)              # (T, V') codes, (T, V'/128)
-    # P^T: from P in float32, or with pow2 from the E4M3 P (exact in float32)
-    src_t = Q.dequantize(pq, ps, Q.BLOCK, Q.ACT)[:, :V].astype(np.float32).T if pow2 else P32.T
-    ptq, pts = Q.quantize(_pad_cols(src_t), Q.BLOCK, Q.WEIGHT, **kw)       # (V, T'),  (ceil(V/128), T'/128)
+    ptq, pts = Q.quantize(_pad_cols(P32.T), Q.BLOCK, Q.WEIGHT, **kw)       # (V, T'),  (ceil(V/128), T'/128)
     wtq, wts = Q.quantize(_pad_cols(np.asarray(W, np.float32).T), Q.BLOCK, Q.WEIGHT, **kw)   # (H, V')
     htq, hts = Q.quantize(_pad_cols(np.asarray(h, np.float32).T), Q.BLOCK, Q.WEIGHT, **kw)   # (H, T')
     P_hat = Q.dequantize(pq, ps, Q.BLOCK, Q.ACT)

@@ -330,8 +330,6 @@ def test_fp8_backward_within_quantisation_error_of_exact_backward(gran, pow2):
     swt = np.repeat(np.repeat(out["wt_scales"], 128, axis=0), 128, axis=1)[:H, :V]
     sht = np.repeat(np.repeat(out["ht_scales"], 128, axis=0), 128, axis=1)[:H, :T]
     ep, ept = _e4m3_abs_err_bound(P, sp), _e4m3_abs_err_bound(P.T, spt)
-    if pow2:  # P^T requantised from P_hat: both roundings
-        ept = ep.T + _e4m3_abs_err_bound(out["P_hat"].T, spt)
     ew, eh = _e4m3_abs_err_bound(W.T, swt), _e4m3_abs_err_bound(h.T, sht)
     assert np.all(np.abs(out["P_hat"] - P) <= ep) and np.all(np.abs(out["Wt_hat"] - W.T) <= ew)
     assert np.all(np.abs(out["Pt_hat"] - P.T) <= ept) and np.all(np.abs(out["ht_hat"] - h.T) <= eh)
@@ -399,11 +397,9 @@ def test_fp8_backward_pow2_scales_by_brute_force():
         for b in range(out["p_scales"].shape[1]):
             blk = P[t, 128 * b:128 * b + 128]
             assert out["p_scales"][t, b] == expected_scale(blk), (t, b)
-    # P^T is requantised from the E4M3 P: its block scales come from P_hat
-    P_hat = out["P_hat"]
     for vb in range(out["pt_scales"].shape[0]):
         for tb in range(out["pt_scales"].shape[1]):
-            blk = P_hat.T[128 * vb:128 * vb + 128, 128 * tb:128 * tb + 128]
+            blk = P.T[128 * vb:128 * vb + 128, 128 * tb:128 * tb + 128]
             assert out["pt_scales"][vb, tb] == expected_scale(blk), (vb, tb)
     for hb in range(out["wt_scales"].shape[0]):
         for vb in range(out["wt_scales"].shape[1]):
@@ -417,12 +413,3 @@ def test_fp8_backward_pow2_scales_by_brute_force():
     q = (P / sp).astype(np.float32)
     assert np.array_equal(out["p_codes"][:, :V], e4m3.encode(q))
     assert np.array_equal(out["P_hat"], e4m3.decode(e4m3.encode(q)) * sp)
-    # with power-of-two scales the requantised P^T codes are the codes of P^T
-    # quantised directly wherever the block-scaled value is at least 2^-5 (in
-    # E4M3's normal range scaling by a power of two commutes with rounding);
-    # below that the two roundings may meet a tie
-    spt = np.repeat(np.repeat(out["pt_scales"], 128, axis=0), 128, axis=1)[:V, :T]
-    direct = e4m3.encode((P.T / spt).astype(np.float32))
-    big = np.abs(P_hat.T / spt) >= 2.0 ** -5
-    assert np.array_equal(out["pt_codes"][:, :T][big], direct[big]) and big.sum() > 1000
-    assert np.array_equal(out["Pt_hat"], e4m3.decode(out["pt_codes"][:, :T]) * spt)
