@@ -39,15 +39,16 @@ __global__ void __launch_bounds__(kTok * kWarps) combine_kernel(
   const int64_t t = blockIdx.x * static_cast<int64_t>(kTok) + lane;
   float m = -INFINITY, s = 0.f;
   if (t < M) {
-    // eight loads in flight per lane: the grid has only T / 32 CTAs, so the
-    // bytes in flight come from depth per thread rather than from occupancy
+    // sixteen loads in flight per lane: the grid has only T / 32 CTAs, so
+    // the bytes in flight come from depth per thread rather than from occupancy
+    constexpr int kDepth = 16;
     int64_t c = w;
-    for (; c + 7 * kWarps < n_chunks; c += 8 * kWarps) {
-      float2 q[8];
+    for (; c + (kDepth - 1) * kWarps < n_chunks; c += kDepth * kWarps) {
+      float2 q[kDepth];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) q[u] = __ldg(partials + (c + u * kWarps) * M + t);
+      for (int u = 0; u < kDepth; ++u) q[u] = __ldg(partials + (c + u * kWarps) * M + t);
 #pragma unroll
-      for (int u = 0; u < 8; ++u) merge(m, s, q[u]);
+      for (int u = 0; u < kDepth; ++u) merge(m, s, q[u]);
     }
     for (; c < n_chunks; c += kWarps) merge(m, s, __ldg(partials + c * M + t));
   }

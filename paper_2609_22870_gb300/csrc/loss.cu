@@ -518,6 +518,19 @@ __global__ void __launch_bounds__(kThreads) seq_accum_kernel(
     for (int k = 0; k < 4; ++k) on[k] = ((mv >> (8 * k)) & 0xFFu) != 0;
   };
   int64_t base = beg;
+  // without the sums a step loads only ids and mask (5 B a token): four full
+  // steps' loads in flight before any is processed
+  if (VEC && !SUMS) {
+    for (; base + 511 < end; base += 512) {
+      int id[4][4];
+      float lp[4][4], lo[4][4];
+      bool on[4][4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) load_vec(base + 128 * k + 4 * lane, id[k], lp[k], lo[k], on[k]);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) step(id[k], lp[k], lo[k], on[k], base + 128 * k + 4 * lane);
+    }
+  }
   // two full steps' loads in flight before either is processed
   if (VEC) {
     for (; base + 255 < end; base += 256) {
