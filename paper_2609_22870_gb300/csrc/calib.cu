@@ -200,8 +200,8 @@ __device__ __forceinline__ unsigned term_exponent(float c, float r, float a) {
   return static_cast<unsigned>(64 - __clzll(static_cast<long long>(m)) + e + kEBias);
 }
 
-// q_t = RNE(fl64(fl64(c r) a) 2^s) as int64.
-__device__ __forceinline__ long long fixed_term(float c, float r, float a, int s) {
+// q_t = RNE(fl64(fl64(c r) a) 2^s) as int64, on the exact integer significands.
+__device__ __forceinline__ long long fixed_term_exact(float c, float r, float a, int s) {
   unsigned long long m;
   int e;
   term53(c, r, a, m, e);
@@ -222,6 +222,44 @@ __device__ __forceinline__ long long fixed_term(float c, float r, float a, int s
     }
   }
   return a < 0.f ? -static_cast<long long>(q) : static_cast<long long>(q);
+}
+
+// The same q_t from float32 arithmetic wherever that decides it; false sends
+// the token to fixed_term_exact.  With V = c r |a| 2^s (c, r >= 0):
+//   hi + lo = c r exactly (lo = fma(c, r, -hi), exact for |hi| >= 2^-102),
+//   p1 + e1 = hi |a| exactly (the same for |p1| >= 2^-102),
+//   A = p1 2^s (exact: a power-of-two scale, s in [-126, 127]),
+//   B = fl(e1 + fl(lo |a|)) 2^s, with A + B within 2^-46 |A| of V;
+//   Ai = rint(A) and f = fl((A - Ai) + B) (A - Ai exact).
+// For |A| < 2^35, Ai + f lies within 2^-11 + 2^-12 of V, and fl64(V) within
+// 2^-53 |V| <= 2^-18 of V, so both are within 2^-10 of each other.  When f is
+// more than 2^-9 from the nearest half-integer, no integer rounding boundary
+// lies between them, and RNE(fl64(V)) = Ai + rint(f).  Ties, huge, tiny,
+// zero and non-finite products take the exact path.
+__device__ __forceinline__ bool fixed_term_fast(float c, float r, float a, int s, long long& q) {
+  const float ca = fabsf(a);
+  const float hi = c * r;
+  const float p1 = hi * ca;
+  if (!(hi >= 0x1p-102f && p1 >= 0x1p-102f) || s < -126 || s > 127) return false;
+  const float lo = fmaf(c, r, -hi);
+  const float e1 = fmaf(hi, ca, -p1);
+  const float sc = __int_as_float((s + 127) << 23);
+  const float A = p1 * sc;
+  if (!(A < 0x1p35f)) return false;  // also catches an infinite product
+  const float B = (e1 + lo * ca) * sc;
+  const float Ai = rintf(A);
+  const float f = (A - Ai) + B;
+  const float fi = rintf(f);
+  if (!(fabsf(fabsf(f - fi) - 0.5f) > 0x1p-9f)) return false;
+  const long long m = static_cast<long long>(Ai) + static_cast<long long>(fi);
+  q = a < 0.f ? -m : m;
+  return true;
+}
+
+__device__ __forceinline__ long long fixed_term(float c, float r, float a, int s) {
+  long long q;
+  if (fixed_term_fast(c, r, a, s, q)) return q;
+  return fixed_term_exact(c, r, a, s);
 }
 
 __device__ __forceinline__ bool digit_match(unsigned key, int digit, unsigned prefix) {

@@ -186,3 +186,42 @@ def test_calibrate_crossings_outside_the_interval(cuda_lib, mode, T, case):
     interval ends; bit-exact against the oracle."""
     args = _interval_case(case, T, 400 + T % 97)
     _compare(_run(cuda_lib, *args, 0.2, 0.2, mode=mode), _ref(*args, 0.2, 0.2, mode=mode))
+
+
+@pytest.mark.parametrize("T", [5000, 300000])
+def test_calibrate_eq5_terms_on_rounding_ties(cuda_lib, T):
+    """Eq. 5 terms placed on and next to the rounding ties of q = RNE(e 2^s).
+    The kernel decides most terms in float32 and sends those within 2^-9 of a
+    tie to its exact integer path; every field must still match the oracle
+    bit for bit.  Exact ties: r = 1, |A| = 1, coef = (k + 1/2) 2^-s.  Near
+    ties: coef = fl32((k + 1/2 + d) / (r |A| 2^s)) for d = +-3 2^-9 .. +-2^-22,
+    which lands e 2^s within 2^-20 of its target.  The shift s is unchanged
+    (these terms are far below max |e|)."""
+    r_fp, r_bf, adv, mask, coef = (t.clone() for t in _inputs(T, 41))
+    s = _ref(r_fp, r_bf, adv, mask, coef, 0.2, 0.2)["shift"]
+    rng = np.random.default_rng(43)
+    cand = np.nonzero((mask.numpy() != 0) & (adv.numpy() != 0))[0]
+    pick = rng.choice(cand, size=max(64, T // 40), replace=False)
+    rf, rb, a, c = r_fp.numpy(), r_bf.numpy(), adv.numpy(), coef.numpy()
+    # the kernel's float32 path takes terms more than 2^-9 from a tie: 2^-8 and
+    # 3 2^-9 land just outside that margin, the rest inside it
+    deltas = [2.0 ** -9, -2.0 ** -9, 2.0 ** -10, -2.0 ** -10, 2.0 ** -12, -2.0 ** -12, 2.0 ** -22, -2.0 ** -22,
+              2.0 ** -8, -2.0 ** -8, 3 * 2.0 ** -9, -3 * 2.0 ** -9]
+    for j, i in enumerate(pick):
+        k = int(rng.integers(0, 60))
+        if j % 3 == 0:  # an exact tie on both ratios' terms
+            rf[i] = rb[i] = 1.0
+            a[i] = np.float32(1.0 if a[i] > 0 else -1.0)
+            c[i] = np.float32(np.ldexp(k + 0.5, -s))
+        else:  # near a tie, on the BF16 term (j odd) or the FP8 term (j even)
+            r = float(rb[i] if j % 2 else rf[i])
+            target = k + 0.5 + deltas[j % len(deltas)]
+            c[i] = np.float32(target / (r * abs(float(a[i])) * 2.0 ** s))
+    ref = _ref(r_fp, r_bf, adv, mask, coef, 0.2, 0.2)
+    assert ref["shift"] == s
+    # the planted terms do sit on or next to ties
+    e = OC.update_terms(c[pick], rb[pick], a[pick])
+    frac = np.abs(np.ldexp(np.abs(e), s) % 1.0 - 0.5)
+    assert np.sum(frac == 0) >= len(pick) // 3 and np.sum(frac < 2.0 ** -8) >= len(pick) // 2
+    got = _run(cuda_lib, r_fp, r_bf, adv, mask, coef, 0.2, 0.2)
+    _compare(got, ref)
