@@ -357,7 +357,9 @@ __device__ __forceinline__ int pass_token(const Args& a, const PassCtx& x, const
     }
     if (pos) ++acc.n_pos;
     if (neg || pos) {
-      acc.emax = max(acc.emax, max(term_exponent_fast(c, rb, A), term_exponent_fast(c, rf, A)));
+      // |fl64(fl64(c r) A)| is non-decreasing in r (c r is exact, the rounding
+      // monotone), so the larger ratio gives the larger of the two exponents
+      acc.emax = max(acc.emax, term_exponent_fast(c, fmaxf(rb, rf), A));
     }
     if (!neg) return -1;
     w = 1;
