@@ -106,6 +106,9 @@ class ClockSampler:
         self.index = index
         self.sm, self.reasons = [], set()
         self.smax = None
+        self.power_limit_w = None
+        self.region = None
+        self.by_region = {}  # region -> ([sm MHz], [power W])
         self._on = threading.Event()
         self._stop = threading.Event()
         self.src = None
@@ -131,6 +134,9 @@ class ClockSampler:
             mx = ctypes.c_uint()
             if lib.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0:  # 1 = NVML_CLOCK_SM
                 self.smax = float(mx.value)
+            lim = ctypes.c_uint()
+            if lib.nvmlDeviceGetEnforcedPowerLimit(h, ctypes.byref(lim)) == 0:  # mW, read only
+                self.power_limit_w = lim.value / 1000.0
             return (lib, h)
         except OSError:
             return None
@@ -139,12 +145,17 @@ class ClockSampler:
         import ctypes
         lib, h = self.nvml
         clk = ctypes.c_uint()
+        mw = ctypes.c_uint()
         rs = ctypes.c_ulonglong()
         while not self._stop.is_set():
             if not self._on.wait(0.05):
                 continue
+            reg = self.by_region.setdefault(self.region, ([], []))
             if lib.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(clk)) == 0:
                 self.sm.append(float(clk.value))
+                reg[0].append(float(clk.value))
+            if lib.nvmlDeviceGetPowerUsage(h, ctypes.byref(mw)) == 0:
+                reg[1].append(mw.value / 1000.0)
             if lib.nvmlDeviceGetCurrentClocksThrottleReasons(h, ctypes.byref(rs)) == 0:
                 for bit, name in self.REASONS.items():
                     if rs.value & bit:
@@ -152,10 +163,12 @@ class ClockSampler:
             time.sleep(0.005)
 
     class _Active:
-        def __init__(self, outer):
+        def __init__(self, outer, region):
             self.o = outer
+            self.region = region
 
         def __enter__(self):
+            self.o.region = self.region
             self.o._on.set()
             if self.o.nvml is None and self.o.proc is None:
                 self.o._start_smi()
@@ -164,8 +177,10 @@ class ClockSampler:
             self.o._on.clear()
             return False
 
-    def active(self):
-        return self._Active(self)
+    def active(self, region="step"):
+        """Samples while the block runs; `region` names it in the per-region
+        medians (SM clock and board power)."""
+        return self._Active(self, region)
 
     def _start_smi(self):
         fields = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -210,9 +225,15 @@ class ClockSampler:
                 self.proc.kill()
         if self.src is None:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no NVML and no nvidia-smi"]}
-        return {"sm_mhz": statistics.median(self.sm) if self.sm else None,
-                "sm_max_mhz": self.smax, "reasons": sorted(self.reasons), "samples": len(self.sm),
-                "source": self.src}
+        out = {"sm_mhz": statistics.median(self.sm) if self.sm else None,
+               "sm_max_mhz": self.smax, "reasons": sorted(self.reasons), "samples": len(self.sm),
+               "source": self.src}
+        if self.by_region:
+            out["power_limit_w"] = self.power_limit_w
+            out["by_region"] = {r: {"sm_mhz": statistics.median(c) if c else None,
+                                    "power_w": statistics.median(p) if p else None, "samples": len(c)}
+                                for r, (c, p) in self.by_region.items()}
+        return out
 
 
 def pci_bus_id(dev):
@@ -355,7 +376,7 @@ def run_ours(args, rank, world, local_rank):
         u0 = torch.cuda.Event(enable_timing=True)
         u1 = torch.cuda.Event(enable_timing=True)
         ue_events = []
-        with clocks.active():
+        with clocks.active("ue8m0_variant"):
             u0.record(stream)
             for _ in range(args.steps):
                 ev[:] = [torch.cuda.Event(enable_timing=True) for _ in range(7)]
@@ -450,7 +471,7 @@ def run_ours(args, rank, world, local_rank):
         dist.barrier()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
-    with clocks.active():
+    with clocks.active("e2e"):
         e0.record(stream)
         e2e_run(args.steps)
         e1.record(stream)
