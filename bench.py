@@ -135,10 +135,11 @@ class ClockSampler:
             if lib.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0:  # 1 = NVML_CLOCK_SM
                 self.smax = float(mx.value)
             lim = ctypes.c_uint()
-            if lib.nvmlDeviceGetEnforcedPowerLimit(h, ctypes.byref(lim)) == 0:  # mW, read only
+            get_lim = getattr(lib, "nvmlDeviceGetEnforcedPowerLimit", None)
+            if get_lim is not None and get_lim(h, ctypes.byref(lim)) == 0:  # mW, read only
                 self.power_limit_w = lim.value / 1000.0
             return (lib, h)
-        except OSError:
+        except (OSError, AttributeError):
             return None
 
     def _nvml_loop(self):
@@ -147,6 +148,7 @@ class ClockSampler:
         clk = ctypes.c_uint()
         mw = ctypes.c_uint()
         rs = ctypes.c_ulonglong()
+        get_power = getattr(lib, "nvmlDeviceGetPowerUsage", None)
         while not self._stop.is_set():
             if not self._on.wait(0.05):
                 continue
@@ -154,7 +156,7 @@ class ClockSampler:
             if lib.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(clk)) == 0:
                 self.sm.append(float(clk.value))
                 reg[0].append(float(clk.value))
-            if lib.nvmlDeviceGetPowerUsage(h, ctypes.byref(mw)) == 0:
+            if get_power is not None and get_power(h, ctypes.byref(mw)) == 0:
                 reg[1].append(mw.value / 1000.0)
             if lib.nvmlDeviceGetCurrentClocksThrottleReasons(h, ctypes.byref(rs)) == 0:
                 for bit, name in self.REASONS.items():
