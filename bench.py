@@ -366,6 +366,48 @@ def run_ours(args, rank, world, local_rank):
             step()
         torch.cuda.synchronize()
 
+    # the same step captured once into a CUDA graph and replayed: the six
+    # kernels launch from the device-side graph, not one host launch each
+    # (this matters where the step is short; the results must equal the
+    # eager step's bit for bit)
+    graph = None
+    if not args.no_graph:
+        try:
+            step()
+            torch.cuda.synchronize()
+            eager = [t.clone() for t in (b.logp, b.ratio, b.grad, b.clip_mask, b.cal_res, b.stats)]
+            cg = torch.cuda.CUDAGraph()
+            side = torch.cuda.Stream()
+            side.wait_stream(torch.cuda.current_stream())
+            with torch.cuda.stream(side):
+                step()
+            torch.cuda.current_stream().wait_stream(side)
+            with torch.cuda.graph(cg):
+                step()
+            cg.replay()
+            torch.cuda.synchronize()
+            api.check()
+            same = all(torch.equal(a, c) for a, c in
+                       zip(eager, (b.logp, b.ratio, b.grad, b.clip_mask, b.cal_res, b.stats)))
+            for _ in range(args.warmup):
+                cg.replay()
+            g0 = torch.cuda.Event(enable_timing=True)
+            g1 = torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize()
+            g0.record()
+            for _ in range(args.steps):
+                cg.replay()
+            g1.record()
+            torch.cuda.synchronize()
+            api.check()
+            gms = g0.elapsed_time(g1) / args.steps
+            graph = {"ms_per_step": gms, "value": whole_job_rate(T, 1, gms), "unit": "tokens/s",
+                     "matches_eager": same,
+                     "note": "the step captured once into a CUDA graph and replayed (torch.cuda.CUDAGraph)"}
+            del cg
+        except Exception as exc:  # a capture the driver refuses: report it, keep the eager figures
+            graph = {"unavailable": f"{type(exc).__name__}: {str(exc)[:160]}"}
+
     # the same step with power-of-two block scales applied by the tensor
     # cores' block-scaled MMA (a variant outside the paper; block layout only)
     ue = None
@@ -564,6 +606,8 @@ def run_ours(args, rank, world, local_rank):
                                              "clipped_hi_fp8", "clipped_lo_bf16", "clipped_hi_bf16",
                                              "nmae_prob", "nmae_ratio")},
     }
+    if graph is not None:
+        line["cuda_graph"] = graph
     if ue is not None:
         ue_tf = flops / (ue["gemm_ms"] * 1e-3) / 1e12
         line["ue8m0_mma_variant"] = {
@@ -877,6 +921,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-backward", action="store_true", help="skip timing the lm_head backward")
     ap.add_argument("--no-fp8-peak", action="store_true", help="skip measuring the vendor FP8 GEMM rate")
+    ap.add_argument("--no-graph", action="store_true", help="skip timing the step replayed from a CUDA graph")
     ap.add_argument("--no-variants", action="store_true",
                     help="skip timing the step with power-of-two scales on the block-scaled MMA")
     ap.add_argument("--kernels", action="store_true",
