@@ -17,7 +17,11 @@
  * negative inputs where the method forbids them, an expired bounded wait) set
  * a device status word and never trap; fp8rl_check() reports and clears it.
  * Outputs of a call that flagged an error are unspecified (NaN where noted).
- * No C++ exception crosses this interface.
+ * No C++ exception crosses this interface.  No compute call synchronises with
+ * the host or allocates device memory, so a sequence of calls (e.g. one
+ * training step) can be captured into a CUDA graph and replayed, once each
+ * call has run outside the capture on the device (the first call sets kernel
+ * attributes and looks up library addresses).
  *
  * Paper references are to sections, equations and Algorithm 1 of the paper.
  */
