@@ -38,8 +38,8 @@ GRAN_NAMES = {0: "tensor", 1: "row", 2: "block"}
 # DRAM bytes (read + write) per launch of the GEMM kernel on the default
 # workload, from one ncu capture of this kernel source at that workload
 # (dram__bytes_read.sum + dram__bytes_write.sum); reported only while the
-# kernel source is the one that was measured.
-GEMM_TRAFFIC = {"workload": "grpo_8b", "bytes": 1.934e9, "gemm_cu_sha256_prefix": "2b24cd50159400e4"}
+# kernel sources (gemm.cu, gemm_epi.cuh) are the ones that were measured.
+GEMM_TRAFFIC = {"workload": "grpo_8b", "bytes": None, "gemm_sources_sha256_prefix": None}
 
 
 def max_over_ranks(values, world, device="cpu"):
@@ -69,12 +69,18 @@ def load_peaks():
     return dict(FALLBACK_PEAKS), "fallback"
 
 
-def measured_gemm_traffic(w):
+def gemm_source_digest():
+    """sha256 prefix over the GEMM kernel's sources (gemm.cu, then gemm_epi.cuh)."""
     import hashlib
-    src = os.path.join(ROOT, "paper_2609_22870_gb300", "csrc", "gemm.cu")
-    with open(src, "rb") as f:
-        digest = hashlib.sha256(f.read()).hexdigest()[:16]
-    if w.name == GEMM_TRAFFIC["workload"] and digest == GEMM_TRAFFIC["gemm_cu_sha256_prefix"]:
+    h = hashlib.sha256()
+    for name in ("gemm.cu", "gemm_epi.cuh"):
+        with open(os.path.join(ROOT, "paper_2609_22870_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def measured_gemm_traffic(w):
+    if w.name == GEMM_TRAFFIC["workload"] and gemm_source_digest() == GEMM_TRAFFIC["gemm_sources_sha256_prefix"]:
         return GEMM_TRAFFIC["bytes"]
     return None
 

@@ -74,6 +74,16 @@ __device__ __forceinline__ void tile_coords(int tile, const Params& p, int& m_bl
   n_blk = local / band_m;
 }
 
+// 2^x on the special-function unit with a subnormal result flushed to zero
+// (PTX ex2.approx.ftz.f32).  The logsumexp terms are exp(z - max) <= 1 summed
+// into a total of at least 1 (the maximum's own term), so a flushed term, below
+// 2^-126, changes no bit of the sum.
+__device__ __forceinline__ float exp2_ftz(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // Running epilogue state of one thread: row `row`, vocabulary columns
 // [col0, col0 + 128) consumed 32 at a time (values already scaled).
 struct EpiState {
@@ -117,8 +127,8 @@ __device__ __forceinline__ void epi_consume32(const Params& p, EpiState& e, cons
     float acc = 0.f;
 #pragma unroll
     for (int i = 0; i < 32; ++i)
-      if (i < ncol) acc += exp2f(fmaf(z[i], kLog2e, -mb));
-    e.s = e.s * exp2f((e.m - mn) * kLog2e) + acc;
+      if (i < ncol) acc += exp2_ftz(fmaf(z[i], kLog2e, -mb));
+    e.s = e.s * exp2_ftz((e.m - mn) * kLog2e) + acc;
     e.m = mn;
     const int jj = e.j - base;
     if (jj >= 0 && jj < 32) {
@@ -179,7 +189,7 @@ __device__ __forceinline__ void epi_consume128(const Params& p, EpiState& e, con
   const float mb = mn * kLog2e;
   float a4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-  for (int i = 0; i < CHUNK; ++i) a4[i & 3] += exp2f(fmaf(z[i], kLog2e, -mb));
+  for (int i = 0; i < CHUNK; ++i) a4[i & 3] += exp2_ftz(fmaf(z[i], kLog2e, -mb));
   e.s = (a4[0] + a4[1]) + (a4[2] + a4[3]);
   e.m = mn;
   if (e.j >= 0 && e.j < CHUNK) {
