@@ -79,6 +79,35 @@ def test_struct_layouts_match_binding(libpath, tmp_path):
                      ctypes.sizeof(api.ClipStats)]
 
 
+def test_struct_field_offsets_match_binding(libpath, tmp_path):
+    """Every field of the binding's ctypes structs sits at the header's offset
+    (the readers and api.n_valid_view index the device buffers by them)."""
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no gcc")
+    import importlib.util
+    spec = importlib.util.spec_from_file_location("_api_probe2", os.path.join(
+        ROOT, "paper_2609_22870_gb300", "api.py"))
+    api = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(api)  # loads the library; calls nothing on the GPU
+    structs = {"fp8rl_calib_opts": api.CalibOpts, "fp8rl_calib_result": api.CalibResult,
+               "fp8rl_clip_stats": api.ClipStats, "fp8rl_clip_diag": api.ClipDiag}
+    lines = []
+    for cname, cls in structs.items():
+        for fname, _ in cls._fields_:
+            lines.append(f'printf("{cname}.{fname} %zu\\n", offsetof({cname}, {fname}));')
+    src = tmp_path / "o.c"
+    src.write_text('#include <stdio.h>\n#include <stddef.h>\n#include "fp8rl.h"\nint main(void){' +
+                   "".join(lines) + "return 0;}\n")
+    exe = tmp_path / "o"
+    subprocess.run([gcc, "-std=c99", str(src), "-I", os.path.join(ROOT, "include"), "-o", str(exe)],
+                   check=True)
+    got = dict(l.split() for l in subprocess.run([str(exe)], capture_output=True, text=True).stdout.splitlines())
+    for cname, cls in structs.items():
+        for fname, _ in cls._fields_:
+            assert int(got[f"{cname}.{fname}"]) == getattr(cls, fname).offset, (cname, fname)
+
+
 def test_c_program_links_and_runs(libpath, tmp_path):
     """A plain C consumer links against libfp8rl.so and uses the host-side part
     of the ABI: paper defaults, status strings, size queries and the argument
